@@ -1,0 +1,155 @@
+/*
+ * graphpo.h -- C ABI of the GB300 (sm_103a) GraphPO advantage-construction path.
+ *
+ * One call turns a batch of sampled rollout groups into per-token advantages:
+ *
+ *   state embeddings z_v, step boundaries, step lengths, binary rewards
+ *     -> cosine similarity of every comparable state pair of a prompt group
+ *        (tcgen05 tensor cores for bf16 embeddings)              GraphPO Sec. 4.2
+ *     -> pairs with sim >= kappa linked into equivalence classes
+ *        (union-find, class label = smallest state index)       Sec. 4.2, Alg. S.1
+ *     -> pooled node scores S(v), Eq. (combain); step rewards
+ *        r_step = (S(v) - S(p(v))) (1 - max(0, sim(p(v), v)))   Sec. 4.3
+ *     -> correctness advantages over E_cor(u), efficiency advantages
+ *        A_eff on every edge of the routes a_Q -> v              Sec. 4.4
+ *     -> A_dual = A_cor + lambda_eff * A_eff on every token      Sec. 4.5
+ *
+ * Batch layout ("chain layout"): prompt group g owns rollouts
+ * [group_rollout_off[g], group_rollout_off[g+1]); rollout r owns states
+ * [rollout_step_off[r], rollout_step_off[r+1]) in step order (at least one);
+ * state v is the node reached after the step that enters it, and that step is
+ * the generated edge (p(v), v) with step_len[v] >= 1 tokens.  Its tokens are
+ * packed per rollout: rollout r covers tokens [rollout_token_off[r],
+ * rollout_token_off[r+1]) and the spans of its steps follow each other in step
+ * order, so rollout_token_off[r+1] - rollout_token_off[r] = sum of its
+ * step_len.  rollout_step_off[0] = rollout_token_off[0] = 0.
+ *
+ * Memory: every array pointer in gpo_batch and gpo_outputs is DEVICE memory of
+ * the current CUDA device, owned by the caller; the library never allocates
+ * on the compute path.  The caller also provides the workspace
+ * (gpo_workspace_size bytes, 256-byte aligned).  A context owns only a few
+ * host-side bytes and one pinned status word.
+ *
+ * Errors: host-checkable problems (NULL pointers, bad sizes, parameters out of
+ * range, misaligned embeddings, a too small workspace, a group larger than
+ * GPO_MAX_GROUP_STATES) make gpo_compute return an error before anything is
+ * enqueued.  Problems that need the device arrays (non-monotone offsets, step
+ * lengths that do not tile a rollout's tokens, rewards outside {0,1},
+ * non-finite embeddings) are found by the kernels, which then skip the rest
+ * of the work; gpo_sync_status returns them.  Outputs are undefined after any
+ * error.  No C++ exception, abort or device trap crosses this interface.
+ *
+ * Threading: a context may be used by one host thread at a time; calls on
+ * one context and one stream are ordered by the stream.  Calls that share a
+ * workspace must be ordered on the GPU.
+ */
+#ifndef GRAPHPO_H
+#define GRAPHPO_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define GPO_MAX_GROUP_STATES 4096 /* states of one prompt group (one CTA holds a group) */
+
+typedef enum {
+  GPO_OK = 0,
+  GPO_ERR_INVALID_ARG = 1, /* NULL pointer, negative size, parameter out of range */
+  GPO_ERR_SHAPE = 2,       /* offsets / step lengths / token spans inconsistent */
+  GPO_ERR_BAD_REWARD = 3,  /* a reward is not 0 or 1 (GraphPO Sec. 4.3: R(z) in {0,1}) */
+  GPO_ERR_NONFINITE = 4,   /* an embedding row is non-finite (or its squared norm overflows fp32) */
+  GPO_ERR_UNSUPPORTED = 5, /* e.g. a group above GPO_MAX_GROUP_STATES, misaligned embeddings */
+  GPO_ERR_CUDA = 6,        /* a CUDA runtime call failed; see gpo_last_error */
+  GPO_ERR_TIMEOUT = 7,     /* a device-side wait gave up (the kernel returned cleanly) */
+  GPO_ERR_WORKSPACE = 8    /* workspace missing or smaller than gpo_workspace_size */
+} gpo_status;
+
+typedef enum {
+  GPO_MERGE_NONCAUSAL = 0, /* compare every pair not in an ancestor-descendant relation
+                              (Sec. 4.2); in chain layout: states of different rollouts */
+  GPO_MERGE_SAME_DEPTH = 1 /* additionally require equal step depth (layer-wise merging) */
+} gpo_merge_rule;
+
+typedef enum { GPO_EMB_BF16 = 0, GPO_EMB_F32 = 1 } gpo_emb_dtype;
+
+typedef struct {
+  double kappa;      /* merge threshold: linked when sim >= kappa (Sec. 4.2; paper uses 0.92) */
+  double w;          /* pooling coefficient in [0,1], Eq. (combain) (paper uses 0.7) */
+  double lambda_eff; /* >= 0, weight of A_eff in A_dual (Sec. 4.5; paper gives no value) */
+  double std_eps;    /* >= 0, added to every standard deviation (GRPO convention 1e-6) */
+  int32_t std_ddof;  /* 1: sample standard deviation, 0: population */
+  int32_t merge_rule;/* gpo_merge_rule */
+  int32_t flags;     /* GPO_FLAG_* bits, 0 by default */
+} gpo_params;
+
+/* Compute the pairwise similarities of bf16 embeddings on the CUDA cores (fp32
+ * FMA) instead of the tcgen05 tensor cores; fp32 embeddings always use them. */
+#define GPO_FLAG_SIMT_SIMILARITY 1
+
+typedef struct {
+  int32_t num_groups;     /* G >= 0 */
+  int32_t num_rollouts;   /* R >= 0 */
+  int32_t num_states;     /* N >= 0 */
+  int32_t d;              /* embedding width >= 1 */
+  int32_t emb_dtype;      /* gpo_emb_dtype */
+  int32_t max_states_per_group; /* upper bound on any group's state count (sizes the workspace) */
+  int64_t emb_row_stride; /* elements between rows; row bytes must be a multiple of 16 */
+  int64_t total_tokens;   /* T = rollout_token_off[R] */
+  const int32_t* group_rollout_off; /* [G+1] */
+  const int32_t* rollout_step_off;  /* [R+1] */
+  const int32_t* step_len;          /* [N] */
+  const int64_t* rollout_token_off; /* [R+1] */
+  const void* emb;                  /* [N x emb_row_stride], 16-byte aligned */
+  const uint8_t* reward;            /* [R] verifier rewards in {0,1} */
+  const void* root_emb;             /* optional [G x emb_row_stride] prompt embeddings; NULL:
+                                       eta on the first step of every rollout is 0 */
+} gpo_batch;
+
+typedef struct {
+  float* adv;         /* [T] required: A_dual of the edge holding each token */
+  float* adv_cor;     /* [T] optional: A_cor of the edge */
+  float* adv_eff;     /* [T] optional: efficiency advantage routed through the edge (no lambda) */
+  uint8_t* eff_mask;  /* [T] optional: 1 where some route a_Q -> v covers the edge */
+  int32_t* class_id;  /* [N] optional: smallest state index of the state's class */
+  float* node_score;  /* [N] optional: pooled score S(v) */
+  float* edge_adv;    /* [N] optional: A_dual of the edge entering each state */
+} gpo_outputs;
+
+typedef struct gpo_ctx gpo_ctx;
+
+/* Creates a context for the current CUDA device.  Returns GPO_ERR_INVALID_ARG
+ * for parameters out of range, GPO_ERR_UNSUPPORTED if the device is not
+ * sm_103, GPO_ERR_CUDA if the runtime fails. */
+gpo_status gpo_create(gpo_ctx** ctx, const gpo_params* params);
+
+/* Bytes of device workspace gpo_compute needs for batches of this shape
+ * (reads only the host-side sizes of `batch`). */
+gpo_status gpo_workspace_size(const gpo_ctx* ctx, const gpo_batch* batch, size_t* bytes);
+
+/* Enqueues the whole path on `stream` (a cudaStream_t; NULL = legacy default
+ * stream).  Asynchronous: returns once the kernels are enqueued. */
+gpo_status gpo_compute(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* out,
+                       void* workspace, size_t workspace_bytes, void* stream);
+
+/* Waits for `stream` and returns the first error the kernels of the last
+ * gpo_compute on this context reported (GPO_OK if none). */
+gpo_status gpo_sync_status(gpo_ctx* ctx, void* stream);
+
+/* Static description of a status code. */
+const char* gpo_status_string(gpo_status status);
+
+/* Last error message recorded on the context (never NULL). */
+const char* gpo_last_error(const gpo_ctx* ctx);
+
+/* Library version string. */
+const char* gpo_version(void);
+
+void gpo_destroy(gpo_ctx* ctx);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* GRAPHPO_H */

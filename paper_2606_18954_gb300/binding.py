@@ -1,0 +1,280 @@
+"""ctypes binding of libgraphpo (include/graphpo.h).
+
+Argument marshalling only: every step of the path runs in the library's CUDA
+kernels.  PyTorch supplies device memory (inputs, outputs, workspace) and the
+current CUDA stream.  There is no CPU fallback: if the library is not built or
+no sm_103 GPU is present the calls raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import dataclasses
+import os
+import threading
+from typing import Optional
+
+import numpy as np
+
+from . import buildlib as _build
+
+GPO_OK = 0
+STATUS_NAMES = {0: "ok", 1: "invalid argument", 2: "shape", 3: "bad reward", 4: "non-finite",
+                5: "unsupported", 6: "cuda", 7: "timeout", 8: "workspace"}
+MERGE_RULES = {"noncausal": 0, "same_depth": 1}
+FLAG_SIMT_SIMILARITY = 1
+EMB_BF16, EMB_F32 = 0, 1
+
+
+class GraphPOError(RuntimeError):
+    def __init__(self, code: int, msg: str = ""):
+        super().__init__(f"graphpo status {code} ({STATUS_NAMES.get(code, '?')}): {msg}")
+        self.code = code
+
+
+class Params(ctypes.Structure):
+    _fields_ = [("kappa", ctypes.c_double), ("w", ctypes.c_double), ("lambda_eff", ctypes.c_double),
+                ("std_eps", ctypes.c_double), ("std_ddof", ctypes.c_int32), ("merge_rule", ctypes.c_int32),
+                ("flags", ctypes.c_int32)]
+
+
+class CBatch(ctypes.Structure):
+    _fields_ = [("num_groups", ctypes.c_int32), ("num_rollouts", ctypes.c_int32),
+                ("num_states", ctypes.c_int32), ("d", ctypes.c_int32), ("emb_dtype", ctypes.c_int32),
+                ("max_states_per_group", ctypes.c_int32), ("emb_row_stride", ctypes.c_int64),
+                ("total_tokens", ctypes.c_int64),
+                ("group_rollout_off", ctypes.c_void_p), ("rollout_step_off", ctypes.c_void_p),
+                ("step_len", ctypes.c_void_p), ("rollout_token_off", ctypes.c_void_p),
+                ("emb", ctypes.c_void_p), ("reward", ctypes.c_void_p), ("root_emb", ctypes.c_void_p)]
+
+
+class COutputs(ctypes.Structure):
+    _fields_ = [("adv", ctypes.c_void_p), ("adv_cor", ctypes.c_void_p), ("adv_eff", ctypes.c_void_p),
+                ("eff_mask", ctypes.c_void_p), ("class_id", ctypes.c_void_p),
+                ("node_score", ctypes.c_void_p), ("edge_adv", ctypes.c_void_p)]
+
+
+EXPORTS = ["gpo_create", "gpo_workspace_size", "gpo_compute", "gpo_sync_status", "gpo_status_string",
+           "gpo_last_error", "gpo_version", "gpo_destroy"]
+
+_lib = None
+_lock = threading.Lock()
+
+
+def lib_path() -> str:
+    return _build.LIB
+
+
+def load(build_if_missing: bool = False):
+    """Load libgraphpo.so (optionally building it first)."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        path = _build.LIB
+        if not os.path.exists(path):
+            if not build_if_missing:
+                raise RuntimeError(f"{path} is missing: build it with paper_2606_18954_gb300.build()")
+            _build.build()
+        L = ctypes.CDLL(path)
+        L.gpo_create.argtypes = [ctypes.POINTER(ctypes.c_void_p), ctypes.POINTER(Params)]
+        L.gpo_create.restype = ctypes.c_int
+        L.gpo_workspace_size.argtypes = [ctypes.c_void_p, ctypes.POINTER(CBatch), ctypes.POINTER(ctypes.c_size_t)]
+        L.gpo_workspace_size.restype = ctypes.c_int
+        L.gpo_compute.argtypes = [ctypes.c_void_p, ctypes.POINTER(CBatch), ctypes.POINTER(COutputs),
+                                  ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]
+        L.gpo_compute.restype = ctypes.c_int
+        L.gpo_sync_status.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
+        L.gpo_sync_status.restype = ctypes.c_int
+        L.gpo_status_string.argtypes = [ctypes.c_int]
+        L.gpo_status_string.restype = ctypes.c_char_p
+        L.gpo_last_error.argtypes = [ctypes.c_void_p]
+        L.gpo_last_error.restype = ctypes.c_char_p
+        L.gpo_version.argtypes = []
+        L.gpo_version.restype = ctypes.c_char_p
+        L.gpo_destroy.argtypes = [ctypes.c_void_p]
+        L.gpo_destroy.restype = None
+        _lib = L
+        return L
+
+
+def _ptr(t) -> Optional[int]:
+    return None if t is None else t.data_ptr()
+
+
+@dataclasses.dataclass
+class Batch:
+    """Device tensors of one batch in chain layout (see include/graphpo.h)."""
+    group_rollout_off: "torch.Tensor"   # int32 [G+1]
+    rollout_step_off: "torch.Tensor"    # int32 [R+1]
+    step_len: "torch.Tensor"            # int32 [N]
+    rollout_token_off: "torch.Tensor"   # int64 [R+1]
+    emb: "torch.Tensor"                 # bf16 or fp32 [N, d], unit stride in d
+    reward: "torch.Tensor"              # uint8 [R]
+    total_tokens: int
+    max_states_per_group: int
+    root_emb: "Optional[torch.Tensor]" = None
+
+    @property
+    def num_groups(self):
+        return self.group_rollout_off.numel() - 1
+
+    @property
+    def num_rollouts(self):
+        return self.rollout_step_off.numel() - 1
+
+    @property
+    def num_states(self):
+        return self.emb.shape[0]
+
+    def c_struct(self) -> CBatch:
+        import torch
+        e = self.emb
+        assert e.dim() == 2 and e.stride(1) == 1, "embeddings must be [N, d] with unit inner stride"
+        dt = EMB_BF16 if e.dtype == torch.bfloat16 else EMB_F32
+        if e.dtype not in (torch.bfloat16, torch.float32):
+            raise TypeError("embeddings must be bfloat16 or float32")
+        return CBatch(self.num_groups, self.num_rollouts, e.shape[0], e.shape[1], dt,
+                      int(self.max_states_per_group), e.stride(0) if e.shape[0] > 1 else e.shape[1],
+                      int(self.total_tokens),
+                      _ptr(self.group_rollout_off), _ptr(self.rollout_step_off),
+                      _ptr(self.step_len) if self.step_len.numel() else None, _ptr(self.rollout_token_off),
+                      _ptr(e) if e.numel() else None, _ptr(self.reward) if self.reward.numel() else None,
+                      _ptr(self.root_emb))
+
+    @staticmethod
+    def from_arrays(arrs: dict, device="cuda", pin: bool = False) -> "Batch":
+        """From the numpy dict layout of `workloads.make_batch` (copied to `device`)."""
+        import torch
+
+        def t(a, dt):
+            x = torch.from_numpy(np.ascontiguousarray(a).astype(dt, copy=False))
+            if pin and device == "cpu":
+                x = x.pin_memory()
+            return x.to(device) if device != "cpu" else x
+
+        if arrs["emb_dtype"] == "bf16":
+            emb = t(np.asarray(arrs["emb"], np.uint16).view(np.int16), np.int16).view(torch.bfloat16)
+            root = arrs.get("root_emb")
+            root = t(np.asarray(root, np.uint16).view(np.int16), np.int16).view(torch.bfloat16) if root is not None else None
+        else:
+            emb = t(arrs["emb"], np.float32)
+            root = arrs.get("root_emb")
+            root = t(root, np.float32) if root is not None else None
+        go = np.asarray(arrs["group_rollout_off"])
+        so = np.asarray(arrs["rollout_step_off"])
+        ng = so[go[1:]] - so[go[:-1]] if len(go) > 1 else np.zeros(0)
+        return Batch(t(go, np.int32), t(so, np.int32), t(arrs["step_len"], np.int32),
+                     t(arrs["rollout_token_off"], np.int64), emb, t(arrs["reward"], np.uint8),
+                     int(arrs["rollout_token_off"][-1]) if len(arrs["rollout_token_off"]) else 0,
+                     int(ng.max()) if len(ng) else 0, root)
+
+    def to(self, device, non_blocking=False) -> "Batch":
+        f = lambda x: None if x is None else x.to(device, non_blocking=non_blocking)
+        return Batch(f(self.group_rollout_off), f(self.rollout_step_off), f(self.step_len),
+                     f(self.rollout_token_off), f(self.emb), f(self.reward), self.total_tokens,
+                     self.max_states_per_group, f(self.root_emb))
+
+
+class GraphPO:
+    """One context of the advantage path on the current CUDA device.
+
+    gp = GraphPO(kappa=0.92, w=0.7, lambda_eff=1.0)
+    out = gp(batch)            # dict of device tensors; enqueued on the current stream
+    gp.check()                 # waits and raises GraphPOError on a device-side error
+    """
+
+    def __init__(self, kappa=0.92, w=0.7, lambda_eff=1.0, std_eps=1e-6, std_ddof=1,
+                 merge_rule="noncausal", flags=0):
+        self._lib = load()
+        self.params = Params(float(kappa), float(w), float(lambda_eff), float(std_eps), int(std_ddof),
+                             MERGE_RULES[merge_rule] if isinstance(merge_rule, str) else int(merge_rule),
+                             int(flags))
+        h = ctypes.c_void_p()
+        code = self._lib.gpo_create(ctypes.byref(h), ctypes.byref(self.params))
+        if code != GPO_OK:
+            raise GraphPOError(code, "gpo_create")
+        self._h = h
+        self._ws = None
+
+    def close(self):
+        if getattr(self, "_h", None) and self._h.value:
+            self._lib.gpo_destroy(self._h)
+            self._h = ctypes.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def last_error(self) -> str:
+        return self._lib.gpo_last_error(self._h).decode()
+
+    def workspace_size(self, batch: Batch) -> int:
+        n = ctypes.c_size_t()
+        cb = batch.c_struct()
+        code = self._lib.gpo_workspace_size(self._h, ctypes.byref(cb), ctypes.byref(n))
+        if code != GPO_OK:
+            raise GraphPOError(code, self.last_error())
+        return n.value
+
+    def workspace(self, batch: Batch):
+        import torch
+        need = self.workspace_size(batch)
+        if self._ws is None or self._ws.numel() < need or self._ws.device != batch.emb.device:
+            self._ws = torch.empty(max(need, 256), dtype=torch.uint8, device=batch.emb.device)
+        return self._ws
+
+    def alloc_outputs(self, batch: Batch, components=False, nodes=False) -> dict:
+        import torch
+        dev = batch.emb.device
+        T, N = batch.total_tokens, batch.num_states
+        out = {"adv": torch.empty(max(T, 1), dtype=torch.float32, device=dev)[:T]}
+        if components:
+            out["adv_cor"] = torch.empty(max(T, 1), dtype=torch.float32, device=dev)[:T]
+            out["adv_eff"] = torch.empty(max(T, 1), dtype=torch.float32, device=dev)[:T]
+            out["eff_mask"] = torch.empty(max(T, 4), dtype=torch.uint8, device=dev)[:T]
+        if nodes:
+            out["class_id"] = torch.empty(max(N, 1), dtype=torch.int32, device=dev)[:N]
+            out["node_score"] = torch.empty(max(N, 1), dtype=torch.float32, device=dev)[:N]
+            out["edge_adv"] = torch.empty(max(N, 1), dtype=torch.float32, device=dev)[:N]
+        return out
+
+    def compute_into(self, batch: Batch, out: dict, workspace=None, stream=None) -> None:
+        import torch
+        ws = self.workspace(batch) if workspace is None else workspace
+        if stream is None:
+            stream = torch.cuda.current_stream(batch.emb.device)
+        co = COutputs(*[_ptr(out.get(k)) if out.get(k) is not None and out[k].numel() else None
+                        for k in ("adv", "adv_cor", "adv_eff", "eff_mask", "class_id", "node_score", "edge_adv")])
+        cb = batch.c_struct()
+        code = self._lib.gpo_compute(self._h, ctypes.byref(cb), ctypes.byref(co), ws.data_ptr(), ws.numel(),
+                                     ctypes.c_void_p(stream.cuda_stream))
+        if code != GPO_OK:
+            raise GraphPOError(code, self.last_error())
+
+    def __call__(self, batch: Batch, components=False, nodes=False, stream=None) -> dict:
+        out = self.alloc_outputs(batch, components, nodes)
+        self.compute_into(batch, out, stream=stream)
+        return out
+
+    def check(self, stream=None) -> None:
+        import torch
+        if stream is None:
+            stream = torch.cuda.current_stream()
+        code = self._lib.gpo_sync_status(self._h, ctypes.c_void_p(stream.cuda_stream))
+        if code != GPO_OK:
+            raise GraphPOError(code, self.last_error())
+
+    def compute_host(self, host_batch: Batch, stream=None) -> "torch.Tensor":
+        """End-to-end call on HOST tensors (ideally pinned): copies the inputs to the
+        current device, runs the path, copies the per-token advantages back."""
+        import torch
+        dev = torch.device("cuda", torch.cuda.current_device())
+        db = host_batch.to(dev, non_blocking=True)
+        out = self.alloc_outputs(db)
+        self.compute_into(db, out, stream=stream)
+        host = torch.empty(out["adv"].shape, dtype=torch.float32, pin_memory=True)
+        host.copy_(out["adv"], non_blocking=True)
+        self.check(stream)
+        return host

@@ -1,0 +1,320 @@
+// Host implementation of the C ABI declared in include/graphpo.h: argument
+// checks, workspace layout, TMA descriptor encoding and the launch sequence
+//   prep (validate + plan) -> row stats -> similarity merge -> per-group
+//   advantages -> per-token scatter
+// all on the caller's stream.  Nothing here allocates device memory.
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+
+#include "gpo_internal.cuh"
+
+struct gpo_ctx {
+  gpo_params params;
+  int device;
+  int num_sms;
+  uint32_t* host_status;      // pinned copy of the workspace status words
+  const uint32_t* last_status; // device status words of the last gpo_compute
+  char msg[512];
+};
+
+namespace gpo {
+namespace {
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+void set_msg(gpo_ctx* c, const char* fmt, ...) {
+  if (!c) return;
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(c->msg, sizeof c->msg, fmt, ap);
+  va_end(ap);
+}
+
+constexpr size_t kAlign = 256;
+inline size_t up(size_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
+
+int64_t max_items_for(int64_t N, int64_t G, int64_t maxn) {
+  // sum over groups of items_for(n) <= sum n^2/32768 + 3n/256 + 1
+  return N * maxn / 32768 + (3 * N) / 256 + G + 8;
+}
+
+struct Layout {
+  size_t status, items, group_items, groups, state_meta, rollout_group, nrm2, dotp, rn, root_n2, edge_count,
+      edges, e_adv, e_cor, e_eff, e_mask, tok_start, total;
+  int max_items;
+};
+
+bool layout(const gpo_batch& b, Layout& L) {
+  const int64_t G = b.num_groups, R = b.num_rollouts, N = b.num_states;
+  const int64_t mi = max_items_for(N, G, b.max_states_per_group);
+  if (mi > (1 << 30)) return false;
+  L.max_items = (int)mi;
+  size_t o = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = o;
+    o = up(o + bytes);
+    return at;
+  };
+  L.status = take(sizeof(uint32_t) * kStatusWords);
+  L.items = take(sizeof(Item) * mi);
+  L.group_items = take(sizeof(int) * (G + 1));
+  L.groups = take(sizeof(GroupInfo) * G);
+  L.state_meta = take(sizeof(int2) * N);
+  L.rollout_group = take(sizeof(int) * R);
+  L.nrm2 = take(sizeof(float) * N);
+  L.dotp = take(sizeof(float) * N);
+  L.rn = take(sizeof(float) * N);
+  L.root_n2 = take(sizeof(float) * G);
+  L.edge_count = take(sizeof(int) * mi);
+  L.edges = take(sizeof(int2) * (size_t)kEdgeCap * mi);
+  L.e_adv = take(sizeof(float) * N);
+  L.e_cor = take(sizeof(float) * N);
+  L.e_eff = take(sizeof(float) * N);
+  L.e_mask = take(N);
+  L.tok_start = take(sizeof(int64_t) * N);
+  L.total = o;
+  return true;
+}
+
+Ws workspace_views(void* base, const Layout& L) {
+  unsigned char* p = static_cast<unsigned char*>(base);
+  Ws w;
+  w.status = reinterpret_cast<uint32_t*>(p + L.status);
+  w.items = reinterpret_cast<Item*>(p + L.items);
+  w.group_items = reinterpret_cast<int*>(p + L.group_items);
+  w.groups = reinterpret_cast<GroupInfo*>(p + L.groups);
+  w.state_meta = reinterpret_cast<int2*>(p + L.state_meta);
+  w.rollout_group = reinterpret_cast<int*>(p + L.rollout_group);
+  w.nrm2 = reinterpret_cast<float*>(p + L.nrm2);
+  w.dotp = reinterpret_cast<float*>(p + L.dotp);
+  w.rn = reinterpret_cast<float*>(p + L.rn);
+  w.root_n2 = reinterpret_cast<float*>(p + L.root_n2);
+  w.edge_count = reinterpret_cast<int*>(p + L.edge_count);
+  w.edges = reinterpret_cast<int2*>(p + L.edges);
+  w.e_adv = reinterpret_cast<float*>(p + L.e_adv);
+  w.e_cor = reinterpret_cast<float*>(p + L.e_cor);
+  w.e_eff = reinterpret_cast<float*>(p + L.e_eff);
+  w.e_mask = p + L.e_mask;
+  w.tok_start = reinterpret_cast<int64_t*>(p + L.tok_start);
+  w.max_items = L.max_items;
+  return w;
+}
+
+gpo_status check_params(const gpo_params& p) {
+  if (!std::isfinite(p.kappa) || !(p.w >= 0.0 && p.w <= 1.0) || !(p.lambda_eff >= 0.0) ||
+      !std::isfinite(p.lambda_eff) || !(p.std_eps >= 0.0) || !std::isfinite(p.std_eps) || p.std_ddof < 0 ||
+      p.std_ddof > 1 || p.merge_rule < 0 || p.merge_rule > 1 || (p.flags & ~GPO_FLAG_SIMT_SIMILARITY))
+    return GPO_ERR_INVALID_ARG;
+  return GPO_OK;
+}
+
+inline bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
+
+gpo_status check_batch(gpo_ctx* c, const gpo_batch* b) {
+  if (!b) return set_msg(c, "batch is NULL"), GPO_ERR_INVALID_ARG;
+  if (b->num_groups < 0 || b->num_rollouts < 0 || b->num_states < 0 || b->total_tokens < 0 || b->d < 1 ||
+      b->max_states_per_group < 0)
+    return set_msg(c, "negative size or d < 1"), GPO_ERR_INVALID_ARG;
+  if (b->emb_dtype != GPO_EMB_BF16 && b->emb_dtype != GPO_EMB_F32)
+    return set_msg(c, "unknown emb_dtype %d", b->emb_dtype), GPO_ERR_INVALID_ARG;
+  if (b->max_states_per_group > GPO_MAX_GROUP_STATES)
+    return set_msg(c, "max_states_per_group %d above %d", b->max_states_per_group, GPO_MAX_GROUP_STATES),
+           GPO_ERR_UNSUPPORTED;
+  if (b->num_states > 0 && b->max_states_per_group < 1)
+    return set_msg(c, "max_states_per_group must be >= 1"), GPO_ERR_INVALID_ARG;
+  if (b->num_rollouts > b->num_states) return set_msg(c, "more rollouts than states"), GPO_ERR_SHAPE;
+  if (b->emb_row_stride < b->d) return set_msg(c, "emb_row_stride < d"), GPO_ERR_INVALID_ARG;
+  const int64_t esz = b->emb_dtype == GPO_EMB_BF16 ? 2 : 4;
+  if ((b->emb_row_stride * esz) % 16 != 0)
+    return set_msg(c, "embedding row bytes must be a multiple of 16"), GPO_ERR_UNSUPPORTED;
+  if (!b->group_rollout_off || !b->rollout_step_off || !b->rollout_token_off)
+    return set_msg(c, "offset array is NULL"), GPO_ERR_INVALID_ARG;
+  if (b->num_states > 0 && (!b->step_len || !b->emb)) return set_msg(c, "step_len/emb NULL"), GPO_ERR_INVALID_ARG;
+  if (b->num_rollouts > 0 && !b->reward) return set_msg(c, "reward NULL"), GPO_ERR_INVALID_ARG;
+  if ((b->emb && !aligned(b->emb, 16)) || (b->root_emb && !aligned(b->root_emb, 16)))
+    return set_msg(c, "embeddings must be 16-byte aligned"), GPO_ERR_UNSUPPORTED;
+  if ((int64_t)b->num_states * b->emb_row_stride >= (int64_t)1 << 40)
+    return set_msg(c, "embedding matrix too large"), GPO_ERR_UNSUPPORTED;
+  return GPO_OK;
+}
+
+gpo_status check_outputs(gpo_ctx* c, const gpo_batch* b, const gpo_outputs* o) {
+  if (!o) return set_msg(c, "outputs is NULL"), GPO_ERR_INVALID_ARG;
+  if (b->total_tokens > 0 && !o->adv) return set_msg(c, "adv output is NULL"), GPO_ERR_INVALID_ARG;
+  if (!aligned(o->adv, 16) || !aligned(o->adv_cor, 16) || !aligned(o->adv_eff, 16) || !aligned(o->eff_mask, 4))
+    return set_msg(c, "token outputs must be 16-byte (eff_mask 4-byte) aligned"), GPO_ERR_UNSUPPORTED;
+  return GPO_OK;
+}
+
+}  // namespace
+}  // namespace gpo
+
+using namespace gpo;
+
+extern "C" {
+
+const char* gpo_version(void) { return "graphpo-gb300 0.1 (sm_103a)"; }
+
+const char* gpo_status_string(gpo_status s) {
+  switch (s) {
+    case GPO_OK: return "ok";
+    case GPO_ERR_INVALID_ARG: return "invalid argument";
+    case GPO_ERR_SHAPE: return "inconsistent offsets, step lengths or token spans";
+    case GPO_ERR_BAD_REWARD: return "reward outside {0,1}";
+    case GPO_ERR_NONFINITE: return "non-finite embedding";
+    case GPO_ERR_UNSUPPORTED: return "unsupported input or device";
+    case GPO_ERR_CUDA: return "CUDA runtime error";
+    case GPO_ERR_TIMEOUT: return "device-side wait timed out";
+    case GPO_ERR_WORKSPACE: return "workspace missing or too small";
+  }
+  return "unknown status";
+}
+
+const char* gpo_last_error(const gpo_ctx* ctx) { return ctx ? ctx->msg : "no context"; }
+
+gpo_status gpo_create(gpo_ctx** out, const gpo_params* params) {
+  if (!out || !params) return GPO_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (check_params(*params) != GPO_OK) return GPO_ERR_INVALID_ARG;
+  gpo_ctx* c = new (std::nothrow) gpo_ctx();
+  if (!c) return GPO_ERR_CUDA;
+  c->params = *params;
+  c->last_status = nullptr;
+  c->msg[0] = 0;
+  cudaDeviceProp prop;
+  if (cudaGetDevice(&c->device) != cudaSuccess || cudaGetDeviceProperties(&prop, c->device) != cudaSuccess) {
+    delete c;
+    return GPO_ERR_CUDA;
+  }
+  if (!(prop.major == 10 && prop.minor == 3)) {
+    delete c;
+    return GPO_ERR_UNSUPPORTED;
+  }
+  c->num_sms = prop.multiProcessorCount;
+  if (setup_sim_tc() != cudaSuccess || setup_groups() != cudaSuccess ||
+      cudaMallocHost(&c->host_status, sizeof(uint32_t) * kStatusWords) != cudaSuccess) {
+    cudaGetLastError();
+    delete c;
+    return GPO_ERR_CUDA;
+  }
+  *out = c;
+  return GPO_OK;
+}
+
+void gpo_destroy(gpo_ctx* ctx) {
+  if (!ctx) return;
+  if (ctx->host_status) cudaFreeHost(ctx->host_status);
+  delete ctx;
+}
+
+gpo_status gpo_workspace_size(const gpo_ctx* ctx, const gpo_batch* batch, size_t* bytes) {
+  if (!ctx || !bytes) return GPO_ERR_INVALID_ARG;
+  gpo_status s = check_batch(const_cast<gpo_ctx*>(ctx), batch);
+  if (s != GPO_OK) return s;
+  Layout L;
+  if (!layout(*batch, L)) return GPO_ERR_UNSUPPORTED;
+  *bytes = L.total;
+  return GPO_OK;
+}
+
+gpo_status gpo_compute(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* out, void* workspace,
+                       size_t workspace_bytes, void* stream) {
+  if (!ctx) return GPO_ERR_INVALID_ARG;
+  ctx->msg[0] = 0;
+  gpo_status s = check_batch(ctx, batch);
+  if (s != GPO_OK) return s;
+  s = check_outputs(ctx, batch, out);
+  if (s != GPO_OK) return s;
+  Layout L;
+  if (!layout(*batch, L)) return set_msg(ctx, "batch too large"), GPO_ERR_UNSUPPORTED;
+  if (!workspace || !aligned(workspace, kAlign) || workspace_bytes < L.total)
+    return set_msg(ctx, "workspace needs %zu bytes, 256-byte aligned", L.total), GPO_ERR_WORKSPACE;
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev != ctx->device)
+    return set_msg(ctx, "current device differs from the context's"), GPO_ERR_INVALID_ARG;
+
+  const gpo_batch& b = *batch;
+  const gpo_params& p = ctx->params;
+  Sizes sz;
+  sz.G = b.num_groups;
+  sz.R = b.num_rollouts;
+  sz.N = b.num_states;
+  sz.d = b.d;
+  sz.T = b.total_tokens;
+  sz.stride = b.emb_row_stride;
+  sz.maxn = b.max_states_per_group;
+  Params pp;
+  pp.kappa = p.kappa;
+  pp.w = p.w;
+  pp.lambda_eff = p.lambda_eff;
+  pp.eps = p.std_eps;
+  pp.ddof = p.std_ddof;
+  pp.rule = p.merge_rule;
+  const Ws ws = workspace_views(workspace, L);
+  LaunchCtx lc;
+  lc.stream = static_cast<cudaStream_t>(stream);
+  lc.num_sms = ctx->num_sms;
+
+  const bool use_tc = b.emb_dtype == GPO_EMB_BF16 && !(p.flags & GPO_FLAG_SIMT_SIMILARITY) && sz.N > 0;
+  CUtensorMap map;
+  memset(&map, 0, sizeof map);
+  if (use_tc) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return set_msg(ctx, "cuTensorMapEncodeTiled unavailable"), GPO_ERR_CUDA;
+    const cuuint64_t dims[2] = {(cuuint64_t)sz.d, (cuuint64_t)sz.N};
+    const cuuint64_t strides[1] = {(cuuint64_t)(sz.stride * 2)};
+    const cuuint32_t box[2] = {(cuuint32_t)kTileK, (cuuint32_t)kTileM};
+    const cuuint32_t estr[2] = {1, 1};
+    const CUresult r = enc(&map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(b.emb), dims, strides, box,
+                           estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return set_msg(ctx, "cuTensorMapEncodeTiled failed (%d)", (int)r), GPO_ERR_UNSUPPORTED;
+  }
+
+  cudaError_t e = cudaMemsetAsync(ws.status, 0, sizeof(uint32_t) * kStatusWords, lc.stream);
+  if (e == cudaSuccess) e = launch_prep(lc, b, sz, ws);
+  if (e == cudaSuccess && sz.N > 0) {
+    e = launch_row_stats(lc, b, sz, ws);
+    if (e == cudaSuccess) e = use_tc ? launch_sim_tc(lc, map, sz, ws, pp) : launch_sim_simt(lc, b, sz, ws, pp);
+    if (e == cudaSuccess) e = launch_groups(lc, b, *out, sz, ws, pp);
+    if (e == cudaSuccess) e = launch_tokens(lc, *out, sz, ws);
+  }
+  ctx->last_status = ws.status;
+  if (e != cudaSuccess) return set_msg(ctx, "launch failed: %s", cudaGetErrorString(e)), GPO_ERR_CUDA;
+  return GPO_OK;
+}
+
+gpo_status gpo_sync_status(gpo_ctx* ctx, void* stream) {
+  if (!ctx) return GPO_ERR_INVALID_ARG;
+  cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return set_msg(ctx, "stream error: %s", cudaGetErrorString(e)), GPO_ERR_CUDA;
+  if (!ctx->last_status) return GPO_OK;
+  e = cudaMemcpy(ctx->host_status, ctx->last_status, sizeof(uint32_t) * kStatusWords, cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return set_msg(ctx, "status read failed: %s", cudaGetErrorString(e)), GPO_ERR_CUDA;
+  const uint32_t code = ctx->host_status[kStError];
+  if (code != 0)
+    set_msg(ctx, "%s (kernel %u, index %u)", gpo_status_string((gpo_status)code), ctx->host_status[kStWhere],
+            ctx->host_status[kStDetail]);
+  return (gpo_status)code;
+}
+
+}  // extern "C"

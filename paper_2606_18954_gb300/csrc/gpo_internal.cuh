@@ -1,0 +1,273 @@
+// Internal declarations shared by the translation units of libgraphpo.
+// Device-side workspace layout, error reporting, and the inline-PTX wrappers
+// for mbarrier, TMA (cp.async.bulk.tensor) and tcgen05 used by the kernels.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/graphpo.h"
+
+namespace gpo {
+
+// ------------------------------------------------------------------ sizes
+
+constexpr int kTileM = 128;          // rows of one similarity tile (tcgen05 M)
+constexpr int kTileN = 256;          // max columns of one work item (tcgen05 N)
+constexpr int kTileK = 64;           // bf16 elements per 128-byte swizzle row
+constexpr int kEdgeCap = 384;        // spanning-forest edges one item can emit (< rows+cols)
+constexpr int kStatusWords = 16;
+
+// status words (uint32) at the head of the workspace
+enum : int {
+  kStError = 0,     // first gpo_status reported by any kernel
+  kStAbort = 1,     // nonzero: kernels stop early
+  kStItems = 2,     // number of similarity work items planned
+  kStTicket = 3,    // last-block ticket of the prep kernel
+  kStDetail = 4,    // first failing index (debug aid)
+  kStWhere = 5,     // kernel that reported the error (debug aid)
+};
+
+// A similarity work item: rows [row0, row0+128) of one prompt group against
+// columns [col0, col0+ncols) of the same group (col0 >= row0).
+struct Item {
+  int row0, col0, ncols, group;
+};
+
+struct GroupInfo {
+  int s0, n;        // states [s0, s0+n)
+  int r0, nr;       // rollouts [r0, r0+nr)
+};
+
+// Device pointers into the caller's workspace (computed on the host).
+struct Ws {
+  uint32_t* status;      // [kStatusWords]
+  Item* items;           // [max_items]
+  int* group_items;      // [G+1]
+  GroupInfo* groups;     // [G]
+  int2* state_meta;      // [N] {rollout, depth}
+  int* rollout_group;    // [R]
+  float* nrm2;           // [N] squared norm (fp32 accumulation)
+  float* dotp;           // [N] <z_{p(v)}, z_v> (root embedding for depth 1 if given)
+  float* rn;             // [N] 1/|z| (0 for a zero row)
+  float* root_n2;        // [G]
+  int* edge_count;       // [max_items]
+  int2* edges;           // [max_items * kEdgeCap]
+  float* e_adv;          // [N] A_dual per edge
+  float* e_cor;          // [N] A_cor per edge
+  float* e_eff;          // [N] routed efficiency advantage per edge
+  uint8_t* e_mask;       // [N]
+  int64_t* tok_start;    // [N] first token of each edge
+  int max_items;
+};
+
+struct Sizes {
+  int G, R, N, d;
+  int64_t T;
+  int64_t stride;        // embedding row stride in elements
+  int maxn;              // max states per group (host bound)
+};
+
+struct Params {
+  double kappa, w, lambda_eff, eps;
+  int ddof, rule;
+};
+
+// ------------------------------------------------------------------ errors
+
+__device__ __forceinline__ void report(uint32_t* st, int code, int where, int detail) {
+  if (atomicCAS(&st[kStError], 0u, (uint32_t)code) == 0u) {
+    st[kStWhere] = (uint32_t)where;
+    st[kStDetail] = (uint32_t)detail;
+  }
+  atomicExch(&st[kStAbort], 1u);
+}
+
+__device__ __forceinline__ bool aborted(const uint32_t* st) {
+  return *((volatile const uint32_t*)&st[kStAbort]) != 0u;
+}
+
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// ------------------------------------------------------------------ PTX: smem / mbarrier
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Waits for the phase with the given parity.  Gives up after `limit_ns` of
+// wall time or when another thread raised the abort flag: then it reports
+// GPO_ERR_TIMEOUT (first time) and returns false so that the caller can wind
+// down cleanly instead of hanging the GPU.
+// Wind-down waits (copies or MMAs still in flight before the CTA exits) pass
+// honor_abort = false so that they only stop at their time limit.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32_t* st, int where,
+                                          uint64_t limit_ns = 2000000000ull, bool honor_abort = true) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t it = 1;; ++it) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((it & 255u) == 0u) {
+      if (honor_abort && aborted(st)) return false;
+      if (globaltimer_ns() - t0 > limit_ns) {
+        report(st, GPO_ERR_TIMEOUT, where, 0);
+        return false;
+      }
+    }
+  }
+}
+
+// ------------------------------------------------------------------ PTX: TMA
+
+__device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
+// 2-D tiled bulk tensor load into shared memory; completion is signalled as
+// transaction bytes on `bar`.  x is the innermost (element) coordinate.
+__device__ __forceinline__ void tma_load_2d(void* smem_dst, const CUtensorMap* map, uint64_t* bar, int x,
+                                            int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], "
+      "[%2];" ::"r"(smem_u32(smem_dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y)
+      : "memory");
+}
+
+// ------------------------------------------------------------------ PTX: tcgen05
+
+__device__ __forceinline__ void tmem_alloc(uint32_t* dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(dst_smem)),
+               "r"(ncols)
+               : "memory");
+}
+
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// D[tmem] (+)= A[smem] * B[smem]^T, bf16 inputs, fp32 accumulation, one CTA.
+__device__ __forceinline__ void mma_bf16_ss(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                            uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrives once on `bar` when every tcgen05 operation issued so far by this
+// thread has completed.
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                   smem_u32(bar))
+               : "memory");
+}
+
+// 32 lanes x 32 consecutive fp32 columns: thread t of the warp receives TMEM
+// lane (base lane + t), columns [col, col+32).
+__device__ __forceinline__ void tmem_ld_32x32b_x32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
+        "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]),
+        "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]),
+        "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+}
+
+__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+
+// Shared-memory matrix descriptor for a K-major operand stored as rows of 128
+// bytes with the 128-byte swizzle (8-row atoms of 1024 bytes, stacked densely):
+// start address, leading offset (unused for this layout, encoded 1), stride
+// offset 1024 bytes between 8-row groups, descriptor version 1, swizzle mode 2.
+__device__ __forceinline__ uint64_t smem_desc_k128(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)1u << 16;             // leading byte offset >> 4
+  d |= (uint64_t)(1024u >> 4) << 32;   // stride byte offset >> 4
+  d |= (uint64_t)1u << 46;             // descriptor version
+  d |= (uint64_t)2u << 61;             // 128-byte swizzle
+  return d;
+}
+
+// Instruction descriptor of kind::f16: fp32 accumulator, bf16 A and B, both
+// K-major, shape M x N.
+__host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+// ------------------------------------------------------------------ launchers (host)
+
+struct LaunchCtx {
+  cudaStream_t stream;
+  int num_sms;
+};
+
+cudaError_t launch_prep(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws);
+cudaError_t launch_row_stats(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws);
+cudaError_t launch_sim_tc(const LaunchCtx& lc, const CUtensorMap& map, const Sizes& sz, const Ws& ws,
+                          const Params& p);
+cudaError_t launch_sim_simt(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws,
+                            const Params& p);
+cudaError_t launch_groups(const LaunchCtx& lc, const gpo_batch& b, const gpo_outputs& o, const Sizes& sz,
+                          const Ws& ws, const Params& p);
+cudaError_t launch_tokens(const LaunchCtx& lc, const gpo_outputs& o, const Sizes& sz, const Ws& ws);
+
+cudaError_t setup_sim_tc();
+cudaError_t setup_groups();
+size_t sim_tc_smem_bytes();
+size_t groups_smem_bytes(int maxn);
+
+}  // namespace gpo

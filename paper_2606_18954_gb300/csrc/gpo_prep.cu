@@ -1,0 +1,337 @@
+// Validation and planning (first kernel), per-state row statistics, and the
+// per-token advantage scatter (last kernel) of the GraphPO path.
+#include "gpo_internal.cuh"
+
+namespace gpo {
+
+constexpr int kPlanThreads = 1024;
+constexpr int kTokChunk = 4096;   // tokens handled by one block of the scatter kernel
+
+// Similarity work items of a group with n states: row blocks of 128 states,
+// each against the columns at or after its own first state, in chunks of 256.
+__host__ __device__ inline int items_for(int n) {
+  int c = 0;
+  for (int rb = 0; rb * kTileM < n; ++rb) c += (n - rb * kTileM + kTileN - 1) / kTileN;
+  return c;
+}
+
+// Inclusive scan of one int per thread across a block of kPlanThreads.
+__device__ int block_incl_scan(int x, int* warp_tot) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) warp_tot[wid] = x;
+  __syncthreads();
+  if (wid == 0) {
+    int t = warp_tot[lane];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      int y = __shfl_up_sync(0xffffffffu, t, o);
+      if (lane >= o) t += y;
+    }
+    warp_tot[lane] = t;
+  }
+  __syncthreads();
+  const int add = wid > 0 ? warp_tot[wid - 1] : 0;
+  const int res = x + add;
+  __syncthreads();
+  return res;
+}
+
+// ---------------------------------------------------------------------------
+// K0: validate the offset arrays, rewards and step lengths; write per-state
+// (rollout, depth) and per-rollout group; the last block to finish plans the
+// similarity work items.  Nothing is dereferenced before its range is checked.
+__global__ void __launch_bounds__(kPlanThreads) prep_kernel(gpo_batch b, Sizes sz, Ws ws) {
+  uint32_t* st = ws.status;
+  const int tid = blockIdx.x * blockDim.x + threadIdx.x;
+  const int nth = gridDim.x * blockDim.x;
+  const int32_t* go = b.group_rollout_off;
+  const int32_t* so = b.rollout_step_off;
+  const int64_t* to = b.rollout_token_off;
+
+  if (tid == 0) {
+    if (go[0] != 0 || go[sz.G] != sz.R) report(st, GPO_ERR_SHAPE, 0, 0);
+    if (so[0] != 0 || so[sz.R] != sz.N) report(st, GPO_ERR_SHAPE, 0, 1);
+    if (to[0] != 0 || to[sz.R] != sz.T) report(st, GPO_ERR_SHAPE, 0, 2);
+  }
+  for (int g = tid; g < sz.G; g += nth) {
+    const int a = go[g], c = go[g + 1];
+    if (a < 0 || c < a || c > sz.R) {
+      report(st, GPO_ERR_SHAPE, 0, 3);
+      continue;
+    }
+    for (int r = a; r < c; ++r) ws.rollout_group[r] = g;
+  }
+  for (int r = tid; r < sz.R; r += nth) {
+    const int s = so[r], e = so[r + 1];
+    if (s < 0 || e <= s || e > sz.N) {  // every rollout has at least one step
+      report(st, GPO_ERR_SHAPE, 0, 4);
+      continue;
+    }
+    if (b.reward[r] > 1) report(st, GPO_ERR_BAD_REWARD, 0, r);
+    int64_t sum = 0;
+    for (int v = s; v < e; ++v) {
+      const int L = b.step_len[v];
+      if (L < 1) report(st, GPO_ERR_SHAPE, 0, 5);
+      sum += L;
+      ws.state_meta[v] = make_int2(r, v - s + 1);
+    }
+    const int64_t t0 = to[r], t1 = to[r + 1];
+    if (t0 < 0 || t1 > sz.T || t1 - t0 != sum) report(st, GPO_ERR_SHAPE, 0, 6);
+  }
+
+  // ---- last block: plan the work items
+  __shared__ int s_last;
+  __shared__ int s_warp[32];
+  __shared__ int s_carry;
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = atomicAdd(&st[kStTicket], 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  if (threadIdx.x == 0) s_carry = 0;
+  __syncthreads();
+  const bool ok = !aborted(st);
+  for (int base = 0; base < sz.G; base += kPlanThreads) {
+    const int g = base + threadIdx.x;
+    int cnt = 0, s0 = 0, n = 0, r0 = 0;
+    if (ok && g < sz.G) {
+      r0 = go[g];
+      const int r1 = go[g + 1];
+      s0 = so[r0];
+      n = so[r1] - s0;
+      if (n > sz.maxn || n > GPO_MAX_GROUP_STATES) report(st, GPO_ERR_UNSUPPORTED, 0, g);
+      GroupInfo gi;
+      gi.s0 = s0;
+      gi.n = n;
+      gi.r0 = r0;
+      gi.nr = r1 - r0;
+      ws.groups[g] = gi;
+      cnt = items_for(n);
+    }
+    const int incl = block_incl_scan(cnt, s_warp);
+    const int first = s_carry + incl - cnt;
+    if (ok && g < sz.G) {
+      ws.group_items[g] = first;
+      int k = first;
+      for (int rb = 0; rb * kTileM < n; ++rb)
+        for (int c0 = rb * kTileM; c0 < n; c0 += kTileN) {
+          if (k < ws.max_items) {
+            Item it;
+            it.row0 = s0 + rb * kTileM;
+            it.col0 = s0 + c0;
+            it.ncols = min(kTileN, n - c0);
+            it.group = g;
+            ws.items[k] = it;
+            ws.edge_count[k] = 0;
+          }
+          ++k;
+        }
+    }
+    __syncthreads();
+    if (threadIdx.x == kPlanThreads - 1) s_carry += incl;
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    int total = s_carry;
+    if (ok) ws.group_items[sz.G] = total;
+    if (total > ws.max_items) report(st, GPO_ERR_WORKSPACE, 0, total);
+    st[kStItems] = aborted(st) ? 0u : (uint32_t)total;
+  }
+}
+
+cudaError_t launch_prep(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws) {
+  const int64_t work = (int64_t)sz.R + sz.G + 1;
+  int blocks = (int)((work + kPlanThreads - 1) / kPlanThreads);
+  blocks = blocks < 1 ? 1 : (blocks > 4 * lc.num_sms ? 4 * lc.num_sms : blocks);
+  prep_kernel<<<blocks, kPlanThreads, 0, lc.stream>>>(b, sz, ws);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// K1a: per state, |z_v|^2 and <z_{p(v)}, z_v> with fp32 accumulation (one warp
+// per row: lane partial sums over a strided set of elements, then a shuffle
+// tree).  p(v) is the previous state of the rollout, or the prompt embedding
+// for the first step when one is given.  Extra warps compute |root|^2.
+
+template <bool kBf16>
+__device__ __forceinline__ void load8(const void* base, int64_t elem, float (&x)[8]) {
+  if (kBf16) {
+    const uint4 u = *reinterpret_cast<const uint4*>(reinterpret_cast<const uint16_t*>(base) + elem);
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      x[2 * i] = __uint_as_float(w[i] << 16);
+      x[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+    }
+  } else {
+    const float4* p = reinterpret_cast<const float4*>(reinterpret_cast<const float*>(base) + elem);
+    const float4 a = p[0], c = p[1];
+    x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w;
+    x[4] = c.x; x[5] = c.y; x[6] = c.z; x[7] = c.w;
+  }
+}
+
+template <bool kBf16>
+__device__ __forceinline__ float load1(const void* base, int64_t elem) {
+  if (kBf16) return __uint_as_float((uint32_t)(reinterpret_cast<const uint16_t*>(base)[elem]) << 16);
+  return reinterpret_cast<const float*>(base)[elem];
+}
+
+template <bool kBf16>
+__global__ void __launch_bounds__(256) row_stats_kernel(gpo_batch b, Sizes sz, Ws ws) {
+  if (aborted(ws.status)) return;
+  const int lane = threadIdx.x & 31;
+  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  const int nroot = b.root_emb ? sz.G : 0;
+  const int d = sz.d, nvec = d / 8;
+  for (int64_t job = warp; job < (int64_t)sz.N + nroot; job += nwarps) {
+    const void* rowp;
+    const void* parp = nullptr;
+    int64_t row, prow = 0;
+    if (job < sz.N) {
+      row = job;
+      rowp = b.emb;
+      const int2 m = ws.state_meta[job];
+      if (m.y > 1) {
+        parp = b.emb;
+        prow = job - 1;
+      } else if (b.root_emb) {
+        parp = b.root_emb;
+        prow = ws.rollout_group[m.x];
+      }
+    } else {
+      row = job - sz.N;
+      rowp = b.root_emb;
+    }
+    const int64_t rb = row * sz.stride, pb = prow * sz.stride;
+    float s2 = 0.f, sd = 0.f;
+    for (int k = lane; k < nvec; k += 32) {
+      float x[8];
+      load8<kBf16>(rowp, rb + 8 * k, x);
+      if (parp) {
+        float y[8];
+        load8<kBf16>(parp, pb + 8 * k, y);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) sd = fmaf(x[i], y[i], sd);
+      }
+#pragma unroll
+      for (int i = 0; i < 8; ++i) s2 = fmaf(x[i], x[i], s2);
+    }
+    for (int k = nvec * 8 + lane; k < d; k += 32) {
+      const float x = load1<kBf16>(rowp, rb + k);
+      s2 = fmaf(x, x, s2);
+      if (parp) sd = fmaf(x, load1<kBf16>(parp, pb + k), sd);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      s2 += __shfl_xor_sync(0xffffffffu, s2, o);
+      sd += __shfl_xor_sync(0xffffffffu, sd, o);
+    }
+    if (lane == 0) {
+      if (!isfinite(s2) || !isfinite(sd)) report(ws.status, GPO_ERR_NONFINITE, 1, (int)job);
+      if (job < sz.N) {
+        ws.nrm2[row] = s2;
+        ws.dotp[row] = sd;
+        ws.rn[row] = s2 > 0.f ? 1.0f / sqrtf(s2) : 0.f;
+      } else {
+        ws.root_n2[row] = s2;
+      }
+    }
+  }
+}
+
+cudaError_t launch_row_stats(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws) {
+  const int64_t jobs = (int64_t)sz.N + (b.root_emb ? sz.G : 0);
+  if (jobs == 0) return cudaSuccess;
+  int64_t blocks = (jobs * 32 + 255) / 256;
+  const int64_t cap = (int64_t)lc.num_sms * 8;
+  if (blocks > cap) blocks = cap;
+  if (b.emb_dtype == GPO_EMB_BF16)
+    row_stats_kernel<true><<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
+  else
+    row_stats_kernel<false><<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// K3: every token of edge e receives e's advantage (Sec. 4.5).  Block c owns
+// tokens [c*kTokChunk, (c+1)*kTokChunk); the edges that overlap it are found
+// by a short binary search over the edges' first tokens.  Each thread writes
+// four consecutive tokens with one 16-byte store per output.
+
+__global__ void __launch_bounds__(256) tokens_kernel(gpo_outputs o, Sizes sz, Ws ws) {
+  if (aborted(ws.status)) return;
+  const int64_t t0 = (int64_t)blockIdx.x * kTokChunk;
+  const int64_t t1 = min(sz.T, t0 + kTokChunk);
+  // first edge of the chunk: last v with tok_start[v] <= t0
+  __shared__ int s_lo, s_hi;
+  if (threadIdx.x == 0) {
+    int lo = 0, hi = sz.N - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (ws.tok_start[mid] <= t0) lo = mid; else hi = mid - 1;
+    }
+    s_lo = lo;
+    int lo2 = lo, hi2 = sz.N - 1;
+    while (lo2 < hi2) {
+      const int mid = (lo2 + hi2 + 1) >> 1;
+      if (ws.tok_start[mid] <= t1 - 1) lo2 = mid; else hi2 = mid - 1;
+    }
+    s_hi = lo2;
+  }
+  __syncthreads();
+  const int vlo = s_lo, vhi = s_hi;
+  for (int64_t t = t0 + 4 * (int64_t)threadIdx.x; t < t1; t += 4 * (int64_t)blockDim.x) {
+    // edge of token t
+    int lo = vlo, hi = vhi;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (ws.tok_start[mid] <= t) lo = mid; else hi = mid - 1;
+    }
+    int v[4];
+    v[0] = lo;
+#pragma unroll
+    for (int j = 1; j < 4; ++j) {
+      int u = v[j - 1];
+      while (u < vhi && ws.tok_start[u + 1] <= t + j) ++u;
+      v[j] = u;
+    }
+    if (t + 4 <= sz.T) {
+      *reinterpret_cast<float4*>(o.adv + t) =
+          make_float4(ws.e_adv[v[0]], ws.e_adv[v[1]], ws.e_adv[v[2]], ws.e_adv[v[3]]);
+      if (o.adv_cor)
+        *reinterpret_cast<float4*>(o.adv_cor + t) =
+            make_float4(ws.e_cor[v[0]], ws.e_cor[v[1]], ws.e_cor[v[2]], ws.e_cor[v[3]]);
+      if (o.adv_eff)
+        *reinterpret_cast<float4*>(o.adv_eff + t) =
+            make_float4(ws.e_eff[v[0]], ws.e_eff[v[1]], ws.e_eff[v[2]], ws.e_eff[v[3]]);
+      if (o.eff_mask)
+        *reinterpret_cast<uint32_t*>(o.eff_mask + t) =
+            (uint32_t)ws.e_mask[v[0]] | ((uint32_t)ws.e_mask[v[1]] << 8) | ((uint32_t)ws.e_mask[v[2]] << 16) |
+            ((uint32_t)ws.e_mask[v[3]] << 24);
+    } else {
+      for (int j = 0; j < 4 && t + j < sz.T; ++j) {
+        o.adv[t + j] = ws.e_adv[v[j]];
+        if (o.adv_cor) o.adv_cor[t + j] = ws.e_cor[v[j]];
+        if (o.adv_eff) o.adv_eff[t + j] = ws.e_eff[v[j]];
+        if (o.eff_mask) o.eff_mask[t + j] = ws.e_mask[v[j]];
+      }
+    }
+  }
+}
+
+cudaError_t launch_tokens(const LaunchCtx& lc, const gpo_outputs& o, const Sizes& sz, const Ws& ws) {
+  if (sz.T == 0 || sz.N == 0) return cudaSuccess;
+  const int64_t blocks = (sz.T + kTokChunk - 1) / kTokChunk;
+  tokens_kernel<<<(unsigned)blocks, 256, 0, lc.stream>>>(o, sz, ws);
+  return cudaGetLastError();
+}
+
+}  // namespace gpo
