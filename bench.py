@@ -1,0 +1,374 @@
+#!/usr/bin/env python3
+"""Throughput of the GraphPO advantage path on GB300.
+
+A step = one pass of the whole path (validation/planning, row statistics,
+similarity merge, per-group scores and advantages, per-token scatter) over one
+synthetic batch with the shape of the math RLVR workload (128 prompts x 16
+rollouts, ~16 steps, lognormal lengths with a 2k-token median, bf16 d=1024
+state embeddings); `--config` picks another shape.  Inputs are resident in HBM;
+L2 is flushed (a 256 MiB write) before every timed step; every step is timed on
+the device with CUDA events on the launching stream.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--config math]
+
+Multi-GPU (torchrun, one rank per GPU): every rank runs its own batch of the same
+shape (weak scaling, no collective on the data path); value = tokens of all ranks
+divided by the slowest rank's time.  `--impl reference` times the CPU oracle.
+Prints one JSON line on rank 0.
+"""
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+L2_FLUSH_BYTES = 256 << 20
+METRIC = "advantage-labelled rollout tokens/s & graphs/s; fraction of HBM roofline"
+WORKLOADS = {
+    "tiny": "tiny: 8 prompts x 8 rollouts x 6 steps, fp32 d=256, kappa 0.9",
+    "math": "math RLVR shape: 128 prompts x 16 rollouts, ~16 steps, lognormal lengths (median 2k, cap 8k), "
+            "bf16 d=1024, 32 centroids/prompt, sigma 0.08, rewards Bernoulli(Beta(2,2))",
+    "agentic": "agentic-search shape: 256 prompts x 8 rollouts, 4-10 steps of 64-1024 tokens, bf16 d=1024, "
+               "16 centroids/prompt, rewards Bernoulli(0.3)",
+    "wide": "wide groups: 64 prompts x 64 rollouts x 32 steps (2048 states/group), bf16 d=2048, "
+            "64 centroids/prompt, sigma 0.06",
+    "full": "full batch: 512 prompts x 16 rollouts, ~20 steps, lognormal lengths (median 4k, cap 16k), "
+            "bf16 d=1024, 48 centroids/prompt",
+}
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), float(p["bf16_tflops"]), float(p.get("bf16_tflops_sustained", p["bf16_tflops"])), "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+def algorithmic(b):
+    """Bytes and FLOPs of the path and of each stage (one launch each)."""
+    import numpy as np
+    N = len(b["step_len"])
+    R = len(b["reward"])
+    G = len(b["group_rollout_off"]) - 1
+    T = int(b["rollout_token_off"][-1])
+    d = b["emb"].shape[1]
+    esz = 2 if b["emb_dtype"] == "bf16" else 4
+    zb = N * d * esz
+    so, go = b["rollout_step_off"], b["group_rollout_off"]
+    ng = (so[go[1:]] - so[go[:-1]]).astype(np.float64)
+    flops = float(d * (ng ** 2).sum())  # comparable upper triangle: 2 d n^2 / 2 per group
+    path_bytes = zb + 4 * N + 12 * R + R + 4 * T
+    stages = {
+        "prep": (4 * (G + 1) + 12 * (R + 1) + 4 * N + R + 8 * N + 4 * R, 0.0),
+        "row_stats": (zb + 8 * N + 12 * N, 0.0),
+        "similarity": (zb + 12 * N, flops),
+        "groups": (8 * N + R + 12 * R + 4 * N + 17 * N + 8 * N, 0.0),
+        "tokens": (4 * T + 8 * N + 4 * N + 4 * N, 0.0),
+    }
+    return dict(N=N, R=R, G=G, T=T, path_bytes=path_bytes, flops=flops, stages=stages)
+
+
+class ClockSampler:
+    """nvidia-smi clock and throttle-reason samples during the timed region."""
+    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, bus_id):
+        self.index = None
+        self.proc = None
+        self.path = os.path.join("/tmp", f"gpo_clocks_{os.getpid()}.csv")
+        try:
+            lines = subprocess.run(["nvidia-smi", "--query-gpu=index,pci.bus_id", "--format=csv,noheader"],
+                                   capture_output=True, text=True, timeout=20).stdout.splitlines()
+            for ln in lines:
+                idx, bid = [x.strip() for x in ln.split(",")]
+                if bus_id and bid.lower().endswith(bus_id.lower()[-10:]):
+                    self.index = idx
+            if self.index is None and lines:
+                self.index = lines[0].split(",")[0].strip()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        try:
+            cmd = ["nvidia-smi", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits", "-lms", "200"]
+            if self.index is not None:
+                cmd += ["-i", self.index]
+            self.proc = subprocess.Popen(cmd, stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        rows = []
+        try:
+            rows = [[p.strip() for p in ln.split(",")] for ln in open(self.path) if ln.count(",") >= 7]
+        except Exception:
+            pass
+        num = lambda x: float(x) if x.replace(".", "", 1).isdigit() else None
+        sm = [v for v in (num(r[0]) for r in rows) if v is not None]
+        mx = [v for v in (num(r[1]) for r in rows) if v is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[4:8]) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows), "gpu_index": self.index}
+
+
+def traffic_for(kernel_file):
+    """DRAM bytes per launch from the committed ncu summary, if the kernel is unchanged since."""
+    try:
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+            t = json.load(f)
+        ent = t[kernel_file]
+        src = os.path.join(ROOT, "paper_2606_18954_gb300", "csrc", kernel_file)
+        h = hashlib.sha256(open(src, "rb").read()).hexdigest()
+        if h != ent["source_sha256"]:
+            return None, "kernel changed since the capture"
+        return float(ent["bytes_per_launch"]), ent.get("note", "")
+    except Exception:
+        return None, "no capture"
+
+
+STAGE_SOURCE = {"prep": "gpo_prep.cu", "row_stats": "gpo_prep.cu", "similarity": "gpo_sim_tc.cu",
+                "groups": "gpo_group.cu", "tokens": "gpo_prep.cu"}
+
+
+def cpu_baseline(b, budget_s=6.0, max_groups=None):
+    import numpy as np
+    import oracle
+    from paper_2606_18954_gb300 import workloads as W
+    cores = len(os.sched_getaffinity(0))
+    G = len(b["group_rollout_off"]) - 1
+    sub, sample = b, f"the whole batch ({G} groups)"
+    if max_groups is not None and G > max_groups:
+        sub = W.sub_batch(b, range(max_groups))
+        sample = f"the first {max_groups} of {G} groups"
+    T = int(sub["rollout_token_off"][-1])
+    params = dict(kappa=b["kappa"], w=b["w"], lambda_eff=b["lambda_eff"])
+    oracle.run(W.sub_batch(sub, [0]), params, threads=1)  # build + warm
+    times = []
+    t_start = time.perf_counter()
+    while True:
+        t0 = time.perf_counter()
+        oracle.run(sub, params, threads=cores, want={"adv"})
+        times.append(time.perf_counter() - t0)
+        if time.perf_counter() - t_start > budget_s and len(times) >= 2:
+            break
+    t = statistics.median(times)
+    return {"value": T / t, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": f"{sample}, {len(times)} timed passes, median",
+            "graphs_per_s": (len(sub["group_rollout_off"]) - 1) / t}
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    return ws, int(os.environ.get("RANK", "0")), int(os.environ.get("LOCAL_RANK", "0"))
+
+
+def run_reference(args):
+    ws, rank, _ = dist_env()
+    if rank != 0:
+        return 0
+    from paper_2606_18954_gb300 import workloads as W
+    import oracle
+    b = W.make_batch(W.CONFIGS[args.config])
+    cores = len(os.sched_getaffinity(0))
+    G = len(b["group_rollout_off"]) - 1
+    max_groups = {"wide": 2, "full": 64}.get(args.config)
+    sub, sample = b, f"the whole batch ({G} groups)"
+    if max_groups and G > max_groups:
+        sub = W.sub_batch(b, range(max_groups))
+        sample = f"the first {max_groups} of {G} groups per step"
+    T = int(sub["rollout_token_off"][-1])
+    params = dict(kappa=b["kappa"], w=b["w"], lambda_eff=b["lambda_eff"])
+    for _ in range(args.warmup):
+        oracle.run(sub, params, threads=cores, want={"adv"})
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        oracle.run(sub, params, threads=cores, want={"adv"})
+        times.append(time.perf_counter() - t0)
+    ms = 1e3 * statistics.mean(times)
+    value = T / (ms / 1e3)
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOADS[args.config], "sample": sample},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "graphs_per_s": (len(sub["group_rollout_off"]) - 1) / (ms / 1e3)}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_ours(args):
+    import numpy as np
+    import torch
+    import paper_2606_18954_gb300 as P
+    from paper_2606_18954_gb300 import workloads as W
+
+    ws_n, rank, local = dist_env()
+    if ws_n > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    dev = torch.device("cuda", torch.cuda.current_device())
+    P.build()
+    spec = W.CONFIGS[args.config]
+    b = W.make_batch(spec, seed=W.config_seed(args.config) + rank)
+    alg = algorithmic(b)
+    db = P.Batch.from_arrays(b, device=dev)
+    gp = P.GraphPO(kappa=b["kappa"], w=b["w"], lambda_eff=b["lambda_eff"])
+    out = gp.alloc_outputs(db)
+    wsp = gp.workspace(db)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    gp.enable_timing(True)
+    for _ in range(args.warmup):
+        gp.compute_into(db, out, workspace=wsp)
+    gp.check()
+    torch.cuda.synchronize()
+
+    def barrier():
+        if ws_n > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    bus = None
+    try:
+        bus = torch.cuda.get_device_properties(dev).pci_bus_id
+    except Exception:
+        pass
+    step_ms, stage_acc, nst = [], {}, 0
+    barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(bus) as clk:
+        for _ in range(args.steps):
+            flush.zero_()
+            s = torch.cuda.Event(enable_timing=True)
+            e = torch.cuda.Event(enable_timing=True)
+            s.record(stream)
+            gp.compute_into(db, out, workspace=wsp, stream=stream)
+            e.record(stream)
+            st = gp.stage_times()
+            e.synchronize()
+            step_ms.append(s.elapsed_time(e))
+            nst = len(st)
+            for k, v in st.items():
+                stage_acc[k] = stage_acc.get(k, 0.0) + v
+        torch.cuda.synchronize()
+        barrier()
+    gp.check()
+    gp.enable_timing(False)
+    total_ms = sum(step_ms)
+    if ws_n > 1:
+        import torch.distributed as dist
+        t = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    ms = total_ms / args.steps
+    value = ws_n * alg["T"] / (ms / 1e3)
+
+    # end to end through the public API from pinned host buffers
+    hb = P.Batch.from_arrays(b, device="cpu", pin=True)
+    host_out = torch.empty(alg["T"], dtype=torch.float32, pin_memory=True)
+    h2d = sum(t.numel() * t.element_size() for t in (hb.group_rollout_off, hb.rollout_step_off, hb.step_len,
+                                                      hb.rollout_token_off, hb.emb, hb.reward))
+    for _ in range(max(1, args.warmup // 2)):
+        gp.compute_host(hb, out=host_out)
+    e2e_ms = []
+    for _ in range(args.steps):
+        s = torch.cuda.Event(enable_timing=True)
+        e = torch.cuda.Event(enable_timing=True)
+        s.record(stream)
+        gp.compute_host(hb, out=host_out)
+        e.record(stream)
+        e.synchronize()
+        e2e_ms.append(s.elapsed_time(e))
+    e2e_t = statistics.mean(e2e_ms)
+    if ws_n > 1:
+        import torch.distributed as dist
+        t = torch.tensor([e2e_t], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_t = float(t.item())
+
+    if rank != 0:
+        return 0
+    hbm, tc, tc_sus, peak_src = load_peaks()
+    stage_ms = {k: v / args.steps for k, v in stage_acc.items()}
+    dom = max(stage_ms, key=stage_ms.get)
+    sb, sf = alg["stages"][dom]
+    t_dom = stage_ms[dom] / 1e3
+    if sf and sf / (tc * 1e12) > sb / (hbm * 1e9):
+        roof = {"bound": "tensor", "achieved": sf / t_dom / 1e12, "peak": tc, "unit": "TFLOP/s"}
+    else:
+        roof = {"bound": "hbm", "achieved": sb / t_dom / 1e9, "peak": hbm, "unit": "GB/s"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    traffic, tnote = traffic_for(STAGE_SOURCE.get(dom, ""))
+    roof.update(traffic=traffic, kernel=dom, peak_source=f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured"
+                else "fallback", traffic_note=tnote)
+    path_t = max(alg["path_bytes"] / (hbm * 1e9), alg["flops"] / (tc * 1e12))
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": ws_n, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": WORKLOADS[args.config], "groups": alg["G"], "rollouts": alg["R"],
+                   "states": alg["N"], "tokens": alg["T"], "d": int(b["emb"].shape[1]),
+                   "emb_dtype": b["emb_dtype"], "merge_rule": "noncausal", "kappa": b["kappa"], "w": b["w"],
+                   "lambda_eff": b["lambda_eff"], "l2": "flushed by a 256 MiB write before every timed step",
+                   "seed": W.config_seed(args.config)},
+        "graphs_per_s": ws_n * alg["G"] / (ms / 1e3),
+        "path_roofline": {"bytes": alg["path_bytes"], "flops": alg["flops"], "roofline_us": path_t * 1e6,
+                          "frac": path_t / (ms / 1e3)},
+        "stage_ms": stage_ms,
+        "roofline": roof,
+        "e2e": {"value": ws_n * alg["T"] / (e2e_t / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": int(h2d),
+                "d2h_bytes_per_step": int(4 * alg["T"]), "ms_per_step": e2e_t},
+        "clocks": clk.summary(),
+        "gpu_launches": nst * args.steps,
+    }
+    if not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(b, max_groups={"wide": 2, "full": 64}.get(args.config))
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", choices=list(WORKLOADS), default="math")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -144,6 +144,16 @@ const char* gpo_status_string(gpo_status status);
 /* Last error message recorded on the context (never NULL). */
 const char* gpo_last_error(const gpo_ctx* ctx);
 
+/* Per-stage device timing (instrumentation; the paper has no counterpart).
+ * When enabled, gpo_compute records a CUDA event on the stream before the
+ * first and after every kernel it launches.  gpo_stage_times waits for the
+ * last of those events and writes, for each stage of the last gpo_compute, its
+ * name and its device time in milliseconds (names stay valid for the
+ * context's lifetime).  Stages not launched report 0.  Returns
+ * GPO_ERR_INVALID_ARG if timing was not enabled or capacity is too small. */
+gpo_status gpo_enable_timing(gpo_ctx* ctx, int enable);
+gpo_status gpo_stage_times(gpo_ctx* ctx, float* ms, const char** names, int capacity, int* count);
+
 /* Library version string. */
 const char* gpo_version(void);
 

@@ -54,7 +54,7 @@ class COutputs(ctypes.Structure):
 
 
 EXPORTS = ["gpo_create", "gpo_workspace_size", "gpo_compute", "gpo_sync_status", "gpo_status_string",
-           "gpo_last_error", "gpo_version", "gpo_destroy"]
+           "gpo_last_error", "gpo_version", "gpo_destroy", "gpo_enable_timing", "gpo_stage_times"]
 
 _lib = None
 _lock = threading.Lock()
@@ -93,6 +93,11 @@ def load(build_if_missing: bool = False):
         L.gpo_version.restype = ctypes.c_char_p
         L.gpo_destroy.argtypes = [ctypes.c_void_p]
         L.gpo_destroy.restype = None
+        L.gpo_enable_timing.argtypes = [ctypes.c_void_p, ctypes.c_int]
+        L.gpo_enable_timing.restype = ctypes.c_int
+        L.gpo_stage_times.argtypes = [ctypes.c_void_p, ctypes.POINTER(ctypes.c_float),
+                                      ctypes.POINTER(ctypes.c_char_p), ctypes.c_int, ctypes.POINTER(ctypes.c_int)]
+        L.gpo_stage_times.restype = ctypes.c_int
         _lib = L
         return L
 
@@ -258,6 +263,22 @@ class GraphPO:
         self.compute_into(batch, out, stream=stream)
         return out
 
+    def enable_timing(self, on: bool = True) -> None:
+        code = self._lib.gpo_enable_timing(self._h, int(on))
+        if code != GPO_OK:
+            raise GraphPOError(code, self.last_error())
+
+    def stage_times(self) -> dict:
+        """{stage name: device ms} of the last call (timing must be enabled)."""
+        cap = 16
+        ms = (ctypes.c_float * cap)()
+        names = (ctypes.c_char_p * cap)()
+        n = ctypes.c_int()
+        code = self._lib.gpo_stage_times(self._h, ms, names, cap, ctypes.byref(n))
+        if code != GPO_OK:
+            raise GraphPOError(code, self.last_error())
+        return {names[i].decode(): float(ms[i]) for i in range(n.value)}
+
     def check(self, stream=None) -> None:
         import torch
         if stream is None:
@@ -266,15 +287,32 @@ class GraphPO:
         if code != GPO_OK:
             raise GraphPOError(code, self.last_error())
 
-    def compute_host(self, host_batch: Batch, stream=None) -> "torch.Tensor":
-        """End-to-end call on HOST tensors (ideally pinned): copies the inputs to the
-        current device, runs the path, copies the per-token advantages back."""
+    def compute_host(self, host_batch: Batch, out=None, stream=None) -> "torch.Tensor":
+        """End-to-end call on HOST tensors (pinned for asynchronous copies): copies the
+        inputs into device staging buffers (kept between calls of the same shape),
+        runs the path and copies the per-token advantages back into `out` (a pinned
+        float32 tensor of total_tokens elements, allocated if None).  Waits for the
+        result and raises on a device-side error."""
         import torch
         dev = torch.device("cuda", torch.cuda.current_device())
-        db = host_batch.to(dev, non_blocking=True)
-        out = self.alloc_outputs(db)
-        self.compute_into(db, out, stream=stream)
-        host = torch.empty(out["adv"].shape, dtype=torch.float32, pin_memory=True)
-        host.copy_(out["adv"], non_blocking=True)
+        names = ("group_rollout_off", "rollout_step_off", "step_len", "rollout_token_off", "emb", "reward",
+                 "root_emb")
+        host = [getattr(host_batch, n) for n in names]
+        key = (dev, tuple(None if t is None else (tuple(t.shape), t.dtype) for t in host))
+        if getattr(self, "_stage_key", None) != key:
+            staged = [None if t is None else torch.empty(t.shape, dtype=t.dtype, device=dev) for t in host]
+            self._staged = staged
+            self._stage_key = key
+            self._stage_out = None
+        for h, d in zip(host, self._staged):
+            if h is not None:
+                d.copy_(h, non_blocking=True)
+        db = Batch(*self._staged[:6], host_batch.total_tokens, host_batch.max_states_per_group, self._staged[6])
+        if self._stage_out is None:
+            self._stage_out = self.alloc_outputs(db)
+        self.compute_into(db, self._stage_out, stream=stream)
+        if out is None:
+            out = torch.empty(host_batch.total_tokens, dtype=torch.float32, pin_memory=True)
+        out.copy_(self._stage_out["adv"], non_blocking=True)
         self.check(stream)
-        return host
+        return out

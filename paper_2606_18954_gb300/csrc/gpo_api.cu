@@ -18,6 +18,10 @@ struct gpo_ctx {
   uint32_t* host_status;      // pinned copy of the workspace status words
   const uint32_t* last_status; // device status words of the last gpo_compute
   char msg[512];
+  bool timing;
+  int nstages;                 // stages recorded by the last gpo_compute
+  cudaEvent_t ev[gpo::kMaxStages + 1];
+  const char* stage_name[gpo::kMaxStages];
 };
 
 namespace gpo {
@@ -210,6 +214,15 @@ gpo_status gpo_create(gpo_ctx** out, const gpo_params* params) {
     return GPO_ERR_UNSUPPORTED;
   }
   c->num_sms = prop.multiProcessorCount;
+  c->timing = false;
+  c->nstages = 0;
+  for (int i = 0; i <= kMaxStages; ++i) {
+    if (cudaEventCreate(&c->ev[i]) != cudaSuccess) {
+      cudaGetLastError();
+      delete c;
+      return GPO_ERR_CUDA;
+    }
+  }
   if (setup_sim_tc() != cudaSuccess || setup_groups() != cudaSuccess ||
       cudaMallocHost(&c->host_status, sizeof(uint32_t) * kStatusWords) != cudaSuccess) {
     cudaGetLastError();
@@ -223,6 +236,8 @@ gpo_status gpo_create(gpo_ctx** out, const gpo_params* params) {
 void gpo_destroy(gpo_ctx* ctx) {
   if (!ctx) return;
   if (ctx->host_status) cudaFreeHost(ctx->host_status);
+  for (int i = 0; i <= kMaxStages; ++i)
+    if (ctx->ev[i]) cudaEventDestroy(ctx->ev[i]);
   delete ctx;
 }
 
@@ -290,16 +305,51 @@ gpo_status gpo_compute(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* 
     if (r != CUDA_SUCCESS) return set_msg(ctx, "cuTensorMapEncodeTiled failed (%d)", (int)r), GPO_ERR_UNSUPPORTED;
   }
 
-  cudaError_t e = cudaMemsetAsync(ws.status, 0, sizeof(uint32_t) * kStatusWords, lc.stream);
-  if (e == cudaSuccess) e = launch_prep(lc, b, sz, ws);
+  int ns = 0;
+  auto stage = [&](const char* name, cudaError_t e) {
+    if (ctx->timing && e == cudaSuccess && ns < kMaxStages) {
+      ctx->stage_name[ns] = name;
+      e = cudaEventRecord(ctx->ev[++ns], lc.stream);
+    }
+    return e;
+  };
+  cudaError_t e = cudaSuccess;
+  if (ctx->timing) e = cudaEventRecord(ctx->ev[0], lc.stream);
+  if (e == cudaSuccess) e = cudaMemsetAsync(ws.status, 0, sizeof(uint32_t) * kStatusWords, lc.stream);
+  if (e == cudaSuccess) e = stage("prep", launch_prep(lc, b, sz, ws));
   if (e == cudaSuccess && sz.N > 0) {
-    e = launch_row_stats(lc, b, sz, ws);
-    if (e == cudaSuccess) e = use_tc ? launch_sim_tc(lc, map, sz, ws, pp) : launch_sim_simt(lc, b, sz, ws, pp);
-    if (e == cudaSuccess) e = launch_groups(lc, b, *out, sz, ws, pp);
-    if (e == cudaSuccess) e = launch_tokens(lc, *out, sz, ws);
+    e = stage("row_stats", launch_row_stats(lc, b, sz, ws));
+    if (e == cudaSuccess)
+      e = stage("similarity", use_tc ? launch_sim_tc(lc, map, sz, ws, pp) : launch_sim_simt(lc, b, sz, ws, pp));
+    if (e == cudaSuccess) e = stage("groups", launch_groups(lc, b, *out, sz, ws, pp));
+    if (e == cudaSuccess) e = stage("tokens", launch_tokens(lc, b, *out, sz, ws));
   }
+  ctx->nstages = ns;
   ctx->last_status = ws.status;
   if (e != cudaSuccess) return set_msg(ctx, "launch failed: %s", cudaGetErrorString(e)), GPO_ERR_CUDA;
+  return GPO_OK;
+}
+
+gpo_status gpo_enable_timing(gpo_ctx* ctx, int enable) {
+  if (!ctx) return GPO_ERR_INVALID_ARG;
+  ctx->timing = enable != 0;
+  ctx->nstages = 0;
+  return GPO_OK;
+}
+
+gpo_status gpo_stage_times(gpo_ctx* ctx, float* ms, const char** names, int capacity, int* count) {
+  if (!ctx || !ctx->timing || !count) return GPO_ERR_INVALID_ARG;
+  *count = ctx->nstages;
+  if (capacity < ctx->nstages) return GPO_ERR_INVALID_ARG;
+  if (ctx->nstages == 0) return GPO_OK;
+  cudaError_t e = cudaEventSynchronize(ctx->ev[ctx->nstages]);
+  for (int i = 0; i < ctx->nstages && e == cudaSuccess; ++i) {
+    float t = 0.f;
+    e = cudaEventElapsedTime(&t, ctx->ev[i], ctx->ev[i + 1]);
+    if (ms) ms[i] = t;
+    if (names) names[i] = ctx->stage_name[i];
+  }
+  if (e != cudaSuccess) return set_msg(ctx, "event timing failed: %s", cudaGetErrorString(e)), GPO_ERR_CUDA;
   return GPO_OK;
 }
 

@@ -18,6 +18,7 @@ constexpr int kTileN = 256;          // max columns of one work item (tcgen05 N)
 constexpr int kTileK = 64;           // bf16 elements per 128-byte swizzle row
 constexpr int kEdgeCap = 384;        // spanning-forest edges one item can emit (< rows+cols)
 constexpr int kStatusWords = 16;
+constexpr int kMaxStages = 8;        // timed stages of one gpo_compute
 
 // status words (uint32) at the head of the workspace
 enum : int {
@@ -263,7 +264,8 @@ cudaError_t launch_sim_simt(const LaunchCtx& lc, const gpo_batch& b, const Sizes
                             const Params& p);
 cudaError_t launch_groups(const LaunchCtx& lc, const gpo_batch& b, const gpo_outputs& o, const Sizes& sz,
                           const Ws& ws, const Params& p);
-cudaError_t launch_tokens(const LaunchCtx& lc, const gpo_outputs& o, const Sizes& sz, const Ws& ws);
+cudaError_t launch_tokens(const LaunchCtx& lc, const gpo_batch& b, const gpo_outputs& o, const Sizes& sz,
+                          const Ws& ws);
 
 cudaError_t setup_sim_tc();
 cudaError_t setup_groups();

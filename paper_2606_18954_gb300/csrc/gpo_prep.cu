@@ -5,7 +5,6 @@
 namespace gpo {
 
 constexpr int kPlanThreads = 1024;
-constexpr int kTokChunk = 4096;   // tokens handled by one block of the scatter kernel
 
 // Similarity work items of a group with n states: row blocks of 128 states,
 // each against the columns at or after its own first state, in chunks of 256.
@@ -212,6 +211,7 @@ __global__ void __launch_bounds__(256) row_stats_kernel(gpo_batch b, Sizes sz, W
     }
     const int64_t rb = row * sz.stride, pb = prow * sz.stride;
     float s2 = 0.f, sd = 0.f;
+#pragma unroll 2
     for (int k = lane; k < nvec; k += 32) {
       float x[8];
       load8<kBf16>(rowp, rb + 8 * k, x);
@@ -261,76 +261,67 @@ cudaError_t launch_row_stats(const LaunchCtx& lc, const gpo_batch& b, const Size
 }
 
 // ---------------------------------------------------------------------------
-// K3: every token of edge e receives e's advantage (Sec. 4.5).  Block c owns
-// tokens [c*kTokChunk, (c+1)*kTokChunk); the edges that overlap it are found
-// by a short binary search over the edges' first tokens.  Each thread writes
-// four consecutive tokens with one 16-byte store per output.
+// K3: every token of edge e receives e's advantage (Sec. 4.5).  One warp
+// writes whole edge spans: the metadata of 32 consecutive edges is fetched in
+// one coalesced round trip and broadcast by shuffles; each span is written
+// with 16-byte stores in its aligned middle and scalar stores at the ends.
 
-__global__ void __launch_bounds__(256) tokens_kernel(gpo_outputs o, Sizes sz, Ws ws) {
+__device__ __forceinline__ void write_span(float* dst, int64_t ts, int64_t te, float v, int lane) {
+  const int64_t a = min(te, (ts + 3) & ~int64_t(3));
+  const int64_t z = max(a, te & ~int64_t(3));
+  if (lane < a - ts) dst[ts + lane] = v;
+  const float4 v4 = make_float4(v, v, v, v);
+  for (int64_t q = (a >> 2) + lane; q < (z >> 2); q += 32) reinterpret_cast<float4*>(dst)[q] = v4;
+  if (lane < te - z) dst[z + lane] = v;
+}
+
+__device__ __forceinline__ void write_span_u8(uint8_t* dst, int64_t ts, int64_t te, uint8_t v, int lane) {
+  const int64_t a = min(te, (ts + 3) & ~int64_t(3));
+  const int64_t z = max(a, te & ~int64_t(3));
+  if (lane < a - ts) dst[ts + lane] = v;
+  const uint32_t v4 = 0x01010101u * v;
+  for (int64_t q = (a >> 2) + lane; q < (z >> 2); q += 32) reinterpret_cast<uint32_t*>(dst)[q] = v4;
+  if (lane < te - z) dst[z + lane] = v;
+}
+
+__global__ void __launch_bounds__(256) tokens_kernel(gpo_batch b, gpo_outputs o, Sizes sz, Ws ws) {
   if (aborted(ws.status)) return;
-  const int64_t t0 = (int64_t)blockIdx.x * kTokChunk;
-  const int64_t t1 = min(sz.T, t0 + kTokChunk);
-  // first edge of the chunk: last v with tok_start[v] <= t0
-  __shared__ int s_lo, s_hi;
-  if (threadIdx.x == 0) {
-    int lo = 0, hi = sz.N - 1;
-    while (lo < hi) {
-      const int mid = (lo + hi + 1) >> 1;
-      if (ws.tok_start[mid] <= t0) lo = mid; else hi = mid - 1;
+  const int lane = threadIdx.x & 31;
+  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t base = warp * 32; base < sz.N; base += nwarps * 32) {
+    const int64_t v = base + lane;
+    int64_t ts = 0;
+    int L = 0;
+    float va = 0.f, vc = 0.f, ve = 0.f;
+    uint32_t vm = 0;
+    if (v < sz.N) {
+      ts = ws.tok_start[v];
+      L = b.step_len[v];
+      va = ws.e_adv[v];
+      if (o.adv_cor) vc = ws.e_cor[v];
+      if (o.adv_eff) ve = ws.e_eff[v];
+      if (o.eff_mask) vm = ws.e_mask[v];
     }
-    s_lo = lo;
-    int lo2 = lo, hi2 = sz.N - 1;
-    while (lo2 < hi2) {
-      const int mid = (lo2 + hi2 + 1) >> 1;
-      if (ws.tok_start[mid] <= t1 - 1) lo2 = mid; else hi2 = mid - 1;
-    }
-    s_hi = lo2;
-  }
-  __syncthreads();
-  const int vlo = s_lo, vhi = s_hi;
-  for (int64_t t = t0 + 4 * (int64_t)threadIdx.x; t < t1; t += 4 * (int64_t)blockDim.x) {
-    // edge of token t
-    int lo = vlo, hi = vhi;
-    while (lo < hi) {
-      const int mid = (lo + hi + 1) >> 1;
-      if (ws.tok_start[mid] <= t) lo = mid; else hi = mid - 1;
-    }
-    int v[4];
-    v[0] = lo;
-#pragma unroll
-    for (int j = 1; j < 4; ++j) {
-      int u = v[j - 1];
-      while (u < vhi && ws.tok_start[u + 1] <= t + j) ++u;
-      v[j] = u;
-    }
-    if (t + 4 <= sz.T) {
-      *reinterpret_cast<float4*>(o.adv + t) =
-          make_float4(ws.e_adv[v[0]], ws.e_adv[v[1]], ws.e_adv[v[2]], ws.e_adv[v[3]]);
-      if (o.adv_cor)
-        *reinterpret_cast<float4*>(o.adv_cor + t) =
-            make_float4(ws.e_cor[v[0]], ws.e_cor[v[1]], ws.e_cor[v[2]], ws.e_cor[v[3]]);
-      if (o.adv_eff)
-        *reinterpret_cast<float4*>(o.adv_eff + t) =
-            make_float4(ws.e_eff[v[0]], ws.e_eff[v[1]], ws.e_eff[v[2]], ws.e_eff[v[3]]);
-      if (o.eff_mask)
-        *reinterpret_cast<uint32_t*>(o.eff_mask + t) =
-            (uint32_t)ws.e_mask[v[0]] | ((uint32_t)ws.e_mask[v[1]] << 8) | ((uint32_t)ws.e_mask[v[2]] << 16) |
-            ((uint32_t)ws.e_mask[v[3]] << 24);
-    } else {
-      for (int j = 0; j < 4 && t + j < sz.T; ++j) {
-        o.adv[t + j] = ws.e_adv[v[j]];
-        if (o.adv_cor) o.adv_cor[t + j] = ws.e_cor[v[j]];
-        if (o.adv_eff) o.adv_eff[t + j] = ws.e_eff[v[j]];
-        if (o.eff_mask) o.eff_mask[t + j] = ws.e_mask[v[j]];
-      }
+    const int cnt = (int)(sz.N - base < 32 ? sz.N - base : 32);
+    for (int j = 0; j < cnt; ++j) {
+      const int64_t s = __shfl_sync(0xffffffffu, ts, j);
+      const int64_t e = s + __shfl_sync(0xffffffffu, L, j);
+      write_span(o.adv, s, e, __shfl_sync(0xffffffffu, va, j), lane);
+      if (o.adv_cor) write_span(o.adv_cor, s, e, __shfl_sync(0xffffffffu, vc, j), lane);
+      if (o.adv_eff) write_span(o.adv_eff, s, e, __shfl_sync(0xffffffffu, ve, j), lane);
+      if (o.eff_mask) write_span_u8(o.eff_mask, s, e, (uint8_t)__shfl_sync(0xffffffffu, vm, j), lane);
     }
   }
 }
 
-cudaError_t launch_tokens(const LaunchCtx& lc, const gpo_outputs& o, const Sizes& sz, const Ws& ws) {
+cudaError_t launch_tokens(const LaunchCtx& lc, const gpo_batch& b, const gpo_outputs& o, const Sizes& sz,
+                          const Ws& ws) {
   if (sz.T == 0 || sz.N == 0) return cudaSuccess;
-  const int64_t blocks = (sz.T + kTokChunk - 1) / kTokChunk;
-  tokens_kernel<<<(unsigned)blocks, 256, 0, lc.stream>>>(o, sz, ws);
+  int64_t blocks = (sz.N + 255) / 256;  // one warp per 32 edges
+  const int64_t cap = (int64_t)lc.num_sms * 8;
+  if (blocks > cap) blocks = cap;
+  tokens_kernel<<<(unsigned)blocks, 256, 0, lc.stream>>>(b, o, sz, ws);
   return cudaGetLastError();
 }
 

@@ -227,31 +227,44 @@ __global__ void __launch_bounds__(kThreads, 1)
       const bool got = mbar_wait(&ctl->tfull[buf], (uint32_t)(m >> 1) & 1u, st, 15);
       if (epi_any(!got)) break;
       tc_fence_after();
-      const int slot_row = t;
+      // pass masks first (branch-free), unions afterwards over the few set bits
       const int nchunks = (item.ncols + 31) >> 5;
-      for (int ch = 0; ch < nchunks; ++ch) {
+      uint32_t masks[kTileN / 32];
+#pragma unroll
+      for (int ch = 0; ch < kTileN / 32; ++ch) masks[ch] = 0u;
+#pragma unroll
+      for (int ch = 0; ch < kTileN / 32; ++ch) {
+        if (ch >= nchunks) break;
+        // a chunk whose last column is at or above no row of this warp holds no pair col > row
+        if (item.col0 + ch * 32 + 31 <= item.row0 + q * 32) continue;
         uint32_t r[32];
         tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * kTileN + ch * 32), r);
         tmem_wait_ld();
-        if (!vrow) continue;
+        uint32_t mk = 0u;
 #pragma unroll
         for (int j = 0; j < 32; ++j) {
           const int c = ch * 32 + j;
-          if (c >= item.ncols) break;
-          const int col = item.col0 + c;
-          if (col <= row) continue;
-          if (ctl->cm_roll[c] == rmeta.x) continue;              // same rollout: ancestor-related
-          if (rule == GPO_MERGE_SAME_DEPTH && ctl->cm_depth[c] != rmeta.y) continue;
-          const float cosv = __uint_as_float(r[j]) * rn_i * ctl->cm_rn[c];
-          if (cosv >= kappa) {
-            const int slot_col = (col < item.row0 + kTileM) ? col - item.row0 : kTileM + (col - item.col0);
-            lunion(ctl->lp, slot_row, slot_col);
-          }
+          const bool ok = (c < item.ncols) & (item.col0 + c > row) & (ctl->cm_roll[c] != rmeta.x) &
+                          ((rule != GPO_MERGE_SAME_DEPTH) | (ctl->cm_depth[c] == rmeta.y)) &
+                          (__uint_as_float(r[j]) * rn_i * ctl->cm_rn[c] >= kappa);
+          mk |= (uint32_t)ok << j;
         }
+        masks[ch] = vrow ? mk : 0u;
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&ctl->tempty[buf]);
+      if (lane == 0) mbar_arrive(&ctl->tempty[buf]);  // accumulator free for the next item
+#pragma unroll
+      for (int ch = 0; ch < kTileN / 32; ++ch) {
+        uint32_t mk = masks[ch];
+        while (mk) {
+          const int j = __ffs(mk) - 1;
+          mk &= mk - 1u;
+          const int col = item.col0 + ch * 32 + j;
+          const int slot_col = (col < item.row0 + kTileM) ? col - item.row0 : kTileM + (col - item.col0);
+          lunion(ctl->lp, t, slot_col);
+        }
+      }
       epi_sync();
       // spanning forest of this item: one edge per non-root slot
       int2* out = ws.edges + (size_t)it * kEdgeCap;
