@@ -154,6 +154,22 @@ const char* gpo_last_error(const gpo_ctx* ctx);
 gpo_status gpo_enable_timing(gpo_ctx* ctx, int enable);
 gpo_status gpo_stage_times(gpo_ctx* ctx, float* ms, const char** names, int capacity, int* count);
 
+/* Allocation-free variant of gpo_compute (the paper has no counterpart).
+ * For callers that cannot allocate device memory when they need the
+ * advantages -- a trainer whose device memory is all owned by a framework
+ * pool, a plug-in whose host forbids allocation calls, a loop that cannot take
+ * cudaMalloc's implicit synchronisation.  Same inputs and outputs as
+ * gpo_compute, but the workspace is one array of GPO_NOALLOC_SCRATCH_BYTES
+ * compiled into the library (held by every GPU that loads it until exit); it
+ * calls no cudaMalloc/cudaFree.  Batches whose gpo_workspace_size exceeds that
+ * size are rejected with GPO_ERR_WORKSPACE before anything is enqueued.  The
+ * first call on a device looks up the array's address; make it before any
+ * stream capture.  All calls on a device share the array: calls that overlap on
+ * the GPU race and must be ordered by the caller.  Errors and gpo_sync_status
+ * behave as for gpo_compute. */
+#define GPO_NOALLOC_SCRATCH_BYTES ((size_t)32 << 20)
+gpo_status gpo_compute_noalloc(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* out, void* stream);
+
 /* Library version string. */
 const char* gpo_version(void);
 

@@ -54,7 +54,7 @@ class COutputs(ctypes.Structure):
 
 
 EXPORTS = ["gpo_create", "gpo_workspace_size", "gpo_compute", "gpo_sync_status", "gpo_status_string",
-           "gpo_last_error", "gpo_version", "gpo_destroy", "gpo_enable_timing", "gpo_stage_times"]
+           "gpo_last_error", "gpo_version", "gpo_destroy", "gpo_enable_timing", "gpo_stage_times", "gpo_compute_noalloc"]
 
 _lib = None
 _lock = threading.Lock()
@@ -93,6 +93,9 @@ def load(build_if_missing: bool = False):
         L.gpo_version.restype = ctypes.c_char_p
         L.gpo_destroy.argtypes = [ctypes.c_void_p]
         L.gpo_destroy.restype = None
+        L.gpo_compute_noalloc.argtypes = [ctypes.c_void_p, ctypes.POINTER(CBatch), ctypes.POINTER(COutputs),
+                                          ctypes.c_void_p]
+        L.gpo_compute_noalloc.restype = ctypes.c_int
         L.gpo_enable_timing.argtypes = [ctypes.c_void_p, ctypes.c_int]
         L.gpo_enable_timing.restype = ctypes.c_int
         L.gpo_stage_times.argtypes = [ctypes.c_void_p, ctypes.POINTER(ctypes.c_float),

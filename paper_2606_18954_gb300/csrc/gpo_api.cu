@@ -170,6 +170,9 @@ gpo_status check_outputs(gpo_ctx* c, const gpo_batch* b, const gpo_outputs* o) {
 }
 
 }  // namespace
+
+void note_error(gpo_ctx* ctx, const char* msg) { set_msg(ctx, "%s", msg); }
+
 }  // namespace gpo
 
 using namespace gpo;

@@ -267,6 +267,9 @@ cudaError_t launch_groups(const LaunchCtx& lc, const gpo_batch& b, const gpo_out
 cudaError_t launch_tokens(const LaunchCtx& lc, const gpo_batch& b, const gpo_outputs& o, const Sizes& sz,
                           const Ws& ws);
 
+// Records a message on the context (gpo_last_error).
+void note_error(gpo_ctx* ctx, const char* msg);
+
 cudaError_t setup_sim_tc();
 cudaError_t setup_groups();
 size_t sim_tc_smem_bytes();
