@@ -88,6 +88,10 @@ typedef struct {
 /* Compute the pairwise similarities of bf16 embeddings on the CUDA cores (fp32
  * FMA) instead of the tcgen05 tensor cores; fp32 embeddings always use them. */
 #define GPO_FLAG_SIMT_SIMILARITY 1
+/* Use the multi-kernel tiled path even when every group fits the fused
+ * group-resident kernel (bf16 embeddings, max_states_per_group <= 384);
+ * for comparisons and tests. */
+#define GPO_FLAG_TILED 2
 
 typedef struct {
   int32_t num_groups;     /* G >= 0 */

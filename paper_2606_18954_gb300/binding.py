@@ -22,6 +22,7 @@ STATUS_NAMES = {0: "ok", 1: "invalid argument", 2: "shape", 3: "bad reward", 4: 
                 5: "unsupported", 6: "cuda", 7: "timeout", 8: "workspace"}
 MERGE_RULES = {"noncausal": 0, "same_depth": 1}
 FLAG_SIMT_SIMILARITY = 1
+FLAG_TILED = 2
 EMB_BF16, EMB_F32 = 0, 1
 
 

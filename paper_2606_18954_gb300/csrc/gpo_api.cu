@@ -126,7 +126,7 @@ Ws workspace_views(void* base, const Layout& L) {
 gpo_status check_params(const gpo_params& p) {
   if (!std::isfinite(p.kappa) || !(p.w >= 0.0 && p.w <= 1.0) || !(p.lambda_eff >= 0.0) ||
       !std::isfinite(p.lambda_eff) || !(p.std_eps >= 0.0) || !std::isfinite(p.std_eps) || p.std_ddof < 0 ||
-      p.std_ddof > 1 || p.merge_rule < 0 || p.merge_rule > 1 || (p.flags & ~GPO_FLAG_SIMT_SIMILARITY))
+      p.std_ddof > 1 || p.merge_rule < 0 || p.merge_rule > 1 || (p.flags & ~(GPO_FLAG_SIMT_SIMILARITY | GPO_FLAG_TILED)))
     return GPO_ERR_INVALID_ARG;
   return GPO_OK;
 }
@@ -226,7 +226,7 @@ gpo_status gpo_create(gpo_ctx** out, const gpo_params* params) {
       return GPO_ERR_CUDA;
     }
   }
-  if (setup_sim_tc() != cudaSuccess || setup_groups() != cudaSuccess ||
+  if (setup_sim_tc() != cudaSuccess || setup_groups() != cudaSuccess || setup_fused() != cudaSuccess ||
       cudaMallocHost(&c->host_status, sizeof(uint32_t) * kStatusWords) != cudaSuccess) {
     cudaGetLastError();
     delete c;
@@ -319,6 +319,10 @@ gpo_status gpo_compute(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* 
   cudaError_t e = cudaSuccess;
   if (ctx->timing) e = cudaEventRecord(ctx->ev[0], lc.stream);
   if (e == cudaSuccess) e = cudaMemsetAsync(ws.status, 0, sizeof(uint32_t) * kStatusWords, lc.stream);
+  const bool fused = use_tc && !(p.flags & GPO_FLAG_TILED) && sz.G > 0 && sz.maxn <= kFusedMaxStates;
+  if (fused) {
+    if (e == cudaSuccess) e = stage("fused", launch_fused(lc, map, b, *out, sz, ws, pp));
+  } else {
   if (e == cudaSuccess) e = stage("prep", launch_prep(lc, b, sz, ws));
   if (e == cudaSuccess && sz.N > 0) {
     e = stage("row_stats", launch_row_stats(lc, b, sz, ws));
@@ -326,6 +330,7 @@ gpo_status gpo_compute(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* 
       e = stage("similarity", use_tc ? launch_sim_tc(lc, map, sz, ws, pp) : launch_sim_simt(lc, b, sz, ws, pp));
     if (e == cudaSuccess) e = stage("groups", launch_groups(lc, b, *out, sz, ws, pp));
     if (e == cudaSuccess) e = stage("tokens", launch_tokens(lc, b, *out, sz, ws));
+  }
   }
   ctx->nstages = ns;
   ctx->last_status = ws.status;

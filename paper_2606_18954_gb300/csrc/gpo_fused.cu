@@ -1,0 +1,524 @@
+// Fused group-resident path: the whole advantage construction for bf16
+// prompt groups of at most 384 states, one persistent CTA per SM working
+// through its groups.
+//
+// Per group g (states [s0, s0+n), rollouts [r0, r0+nr)):
+//   producer warp   TMA: per k-slice of 64 embedding elements, the group's
+//                   rows as ceil(n/128) boxes of 128 rows x 128 B (128B swizzle)
+//   MMA warp        tcgen05.mma kind::f16 (bf16 -> fp32 in TMEM) of the upper
+//                   triangle in 128-row blocks: block b against columns
+//                   [128 b, n), at most 512 accumulator columns per pass;
+//                   if a group needs more, blocks >= 1 go first, block 0 second
+//                   (Sec. 4.2: sim of every comparable pair)
+//   warps 4..7      TMEM drain of each pass: the diagonal and super-diagonal
+//                   entries give |z_i|^2 and <z_i, z_{i+1}> (the norms of the
+//                   cosine and eta(p(v), v)); then cos = acc / (|z_i||z_j|),
+//                   pair mask (different rollout; optionally same depth) and
+//                   threshold sim >= kappa into pass masks, then shared-memory
+//                   union-find (Alg. S.1); the accumulator is released before
+//                   the unions so the next pass / group can start
+//   warps 2..7      per-group validation, graph reward and dual-group advantage
+//                   (gpo_group_math.cuh, fp64) and the token scatter (Sec. 4.5),
+//                   overlapping the next group's loads and MMAs
+// Group ranges are assigned round-robin to CTAs.  Every wait is bounded.
+#include "gpo_group_math.cuh"
+
+namespace gpo {
+
+namespace {
+
+constexpr int kStages = 3;
+constexpr int kThreads = 256;
+constexpr int kMaxN = kFusedMaxStates;          // 384
+constexpr int kBoxBytes = kTileM * 128;         // 128 rows x 128 bytes
+constexpr int kStageBytes = 3 * kBoxBytes;      // up to 384 rows
+constexpr int kTmemCols = 512;
+constexpr int kGThreads = 192;                  // warps 2..7
+constexpr int kBarGroup = 1;                    // named barrier of warps 2..7
+constexpr int kBarEpi = 2;                      // named barrier of warps 4..7
+
+struct Seg {
+  int b, c0, len, tcol;  // row block, first column (local), columns, TMEM column
+};
+
+struct Plan {
+  int npass;
+  int nseg[2];
+  Seg seg[2][4];
+};
+
+__device__ __forceinline__ int r16(int x) { return (x + 15) & ~15; }
+__device__ __forceinline__ int r32(int x) { return (x + 31) & ~31; }
+
+// Segments of the upper triangle: row block b against columns [128 b, n) in
+// chunks of at most 256 (one MMA each).  Each segment owns a multiple of 32
+// TMEM columns (the epilogue reads 32 columns at a time).  One pass if they
+// fit 512 TMEM columns, else pass 0 = blocks >= 1 (at most 256 + 128 columns)
+// and pass 1 = block 0 (at most 256 + 128), so that the norms of every column
+// a pass needs come from its own or an earlier pass.
+__device__ __forceinline__ void make_plan(int n, Plan& pl) {
+  Seg all[4];
+  int na = 0, tot = 0;
+  for (int b = 0; b * kTileM < n; ++b)
+    for (int c0 = b * kTileM; c0 < n && na < 4; c0 += kTileN) {
+      all[na].b = b;
+      all[na].c0 = c0;
+      all[na].len = min(kTileN, n - c0);
+      tot += r32(all[na].len);
+      ++na;
+    }
+  pl.nseg[0] = pl.nseg[1] = 0;
+  if (tot <= kTmemCols) {
+    pl.npass = 1;
+    int col = 0;
+    for (int i = 0; i < na; ++i) {
+      Seg s = all[i];
+      s.tcol = col;
+      col += r32(s.len);
+      pl.seg[0][pl.nseg[0]++] = s;
+    }
+  } else {
+    pl.npass = 2;
+    int col0 = 0, col1 = 0;
+    for (int i = 0; i < na; ++i) {
+      Seg s = all[i];
+      if (s.b >= 1) {
+        s.tcol = col0;
+        col0 += r32(s.len);
+        pl.seg[0][pl.nseg[0]++] = s;
+      } else {
+        s.tcol = col1;
+        col1 += r32(s.len);
+        pl.seg[1][pl.nseg[1]++] = s;
+      }
+    }
+  }
+}
+
+// The group's rollout and state ranges; false if they are out of range.
+__device__ __forceinline__ bool group_range(const gpo_batch& b, const Sizes& sz, int g, int& r0, int& nr, int& s0,
+                                            int& n) {
+  const int a = b.group_rollout_off[g], c = b.group_rollout_off[g + 1];
+  if (a < 0 || c < a || c > sz.R) return false;
+  const int x = b.rollout_step_off[a], y = b.rollout_step_off[c];
+  if (x < 0 || y < x || y > sz.N) return false;
+  r0 = a;
+  nr = c - a;
+  s0 = x;
+  n = y - x;
+  return true;
+}
+
+// Group handled here (all roles agree, they read the same inputs).
+__device__ __forceinline__ bool group_active(const gpo_batch& b, const Sizes& sz, int g, int& r0, int& nr, int& s0,
+                                             int& n) {
+  return group_range(b, sz, g, r0, nr, s0, n) && n > 0 && n <= kMaxN && nr > 0 && nr <= n;
+}
+
+struct __align__(16) GroupSmem {
+  int lab[kMaxN];
+  int roll[kMaxN];
+  int dep[kMaxN];
+  int slen[kMaxN];
+  int rstart[kMaxN + 1];
+  float n2[kMaxN];
+  float dn[kMaxN];       // <z_i, z_{i+1}>
+  float rn[kMaxN];
+  float root_dot[kMaxN]; // <root, z of the first state of rollout r>
+  float eadv[kMaxN], ecor[kMaxN], eeff[kMaxN];
+  int64_t tok0[kMaxN + 1];
+  int64_t tstart[kMaxN];
+  uint8_t rew[kMaxN];
+  uint8_t emask[kMaxN];
+  int flags;             // bit 0: group invalid
+  float root_n2;
+  unsigned char X[group_scratch_bytes(kMaxN)];
+};
+
+struct __align__(8) Ctl {
+  uint64_t full[kStages];
+  uint64_t empty[kStages];
+  uint64_t tfull;
+  uint64_t tempty;
+  uint64_t drain;
+  uint32_t tmem_base;
+};
+
+__device__ __forceinline__ void bar_group() { asm volatile("bar.sync %0, %1;" ::"n"(kBarGroup), "n"(kGThreads) : "memory"); }
+__device__ __forceinline__ void bar_epi() { asm volatile("bar.sync %0, 128;" ::"n"(kBarEpi) : "memory"); }
+
+template <int kBar, int kCount>
+__device__ __forceinline__ bool bar_any(bool flag) {
+  uint32_t out;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.or.pred q, %2, %3, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(out)
+      : "r"((uint32_t)flag), "n"(kBar), "n"(kCount)
+      : "memory");
+  return out != 0;
+}
+
+__device__ __forceinline__ float pick(const uint32_t (&r)[32], int j) {
+  float v = 0.f;
+#pragma unroll
+  for (int k = 0; k < 32; ++k)
+    if (k == j) v = __uint_as_float(r[k]);
+  return v;
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    fused_kernel(const __grid_constant__ CUtensorMap zmap, gpo_batch b, gpo_outputs o, Sizes sz, Ws ws, Params p) {
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  unsigned char* tiles =
+      reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  Ctl* ctl = reinterpret_cast<Ctl*>(tiles + kStages * kStageBytes);
+  GroupSmem* gs = reinterpret_cast<GroupSmem*>(reinterpret_cast<unsigned char*>(ctl) + 256);
+  uint32_t* st = ws.status;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int KT = (sz.d + kTileK - 1) / kTileK;
+  const float kappa = (float)p.kappa;
+
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    if (b.group_rollout_off[0] != 0 || b.group_rollout_off[sz.G] != sz.R) report(st, GPO_ERR_SHAPE, 2, 0);
+    if (b.rollout_step_off[0] != 0 || b.rollout_step_off[sz.R] != sz.N) report(st, GPO_ERR_SHAPE, 2, 1);
+    if (b.rollout_token_off[0] != 0 || b.rollout_token_off[sz.R] != sz.T) report(st, GPO_ERR_SHAPE, 2, 2);
+  }
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&ctl->full[s], 1);
+      mbar_init(&ctl->empty[s], 1);
+    }
+    mbar_init(&ctl->tfull, 1);
+    mbar_init(&ctl->tempty, 4);
+    mbar_init(&ctl->drain, 1);
+    fence_mbar_init();
+    tma_prefetch_desc(&zmap);
+  }
+  if (warp == 1) {
+    tmem_alloc(&ctl->tmem_base, kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = ctl->tmem_base;
+
+  if (warp == 0 && lane == 0) {
+    // ---------------------------------------------------------------- TMA producer
+    int stage = 0;
+    uint32_t phase = 0;
+    int last_parity[kStages];
+    for (int s = 0; s < kStages; ++s) last_parity[s] = -1;
+    bool ok = true;
+    for (int g = blockIdx.x; g < sz.G && ok; g += gridDim.x) {
+      int r0, nr, s0, n;
+      if (!group_active(b, sz, g, r0, nr, s0, n)) continue;
+      Plan pl;
+      make_plan(n, pl);
+      const int nbox = (n + kTileM - 1) / kTileM;
+      for (int pass = 0; pass < pl.npass && ok; ++pass)
+        for (int k = 0; k < KT; ++k) {
+          if (!mbar_wait(&ctl->empty[stage], phase ^ 1u, st, 20)) {
+            ok = false;
+            break;
+          }
+          unsigned char* t = tiles + stage * kStageBytes;
+          mbar_arrive_expect_tx(&ctl->full[stage], (uint32_t)(nbox * kBoxBytes));
+          last_parity[stage] = (int)phase;
+          for (int bx = 0; bx < nbox; ++bx)
+            tma_load_2d(t + bx * kBoxBytes, &zmap, &ctl->full[stage], k * kTileK, s0 + bx * kTileM);
+          if (++stage == kStages) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+    }
+    for (int s = 0; s < kStages; ++s)
+      if (last_parity[s] >= 0) mbar_wait(&ctl->full[s], (uint32_t)last_parity[s], st, 21, 200000000ull, false);
+  } else if (warp == 1 && lane == 0) {
+    // ---------------------------------------------------------------- MMA issuer
+    int stage = 0;
+    uint32_t phase = 0;
+    int u = 0;  // accumulator uses (passes) so far
+    bool ok = true;
+    for (int g = blockIdx.x; g < sz.G && ok; g += gridDim.x) {
+      int r0, nr, s0, n;
+      if (!group_active(b, sz, g, r0, nr, s0, n)) continue;
+      Plan pl;
+      make_plan(n, pl);
+      for (int pass = 0; pass < pl.npass && ok; ++pass, ++u) {
+        if (!mbar_wait(&ctl->tempty, ((uint32_t)u & 1u) ^ 1u, st, 22)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        for (int k = 0; k < KT; ++k) {
+          if (!mbar_wait(&ctl->full[stage], phase, st, 23)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t t = smem_u32(tiles + stage * kStageBytes);
+          for (int si = 0; si < pl.nseg[pass]; ++si) {
+            const Seg s = pl.seg[pass][si];
+            const uint64_t ad = smem_desc_k128(t + (uint32_t)(s.b * kBoxBytes));
+            const uint64_t bd = smem_desc_k128(t + (uint32_t)(s.c0 * 128));
+            const uint32_t idesc = idesc_bf16_f32(kTileM, r16(s.len));
+#pragma unroll
+            for (int kk = 0; kk < kTileK / 16; ++kk)
+              mma_bf16_ss(tmem + (uint32_t)s.tcol, ad + 2u * kk, bd + 2u * kk, idesc, (k | kk) != 0);
+          }
+          mma_commit(&ctl->empty[stage]);
+          if (++stage == kStages) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (ok) mma_commit(&ctl->tfull);
+      }
+    }
+    mma_commit(&ctl->drain);
+    mbar_wait(&ctl->drain, 0, st, 24, 200000000ull, false);
+  } else if (warp >= 2) {
+    // ---------------------------------------------------------------- group warps
+    const int gt = threadIdx.x - 64;  // 0..191
+    const bool epi = warp >= 4;
+    const int q = warp & 3;           // TMEM lane quarter of an epilogue warp
+    const int wg = warp - 2;          // 0..5
+    int u = 0;
+    for (int g = blockIdx.x; g < sz.G; g += gridDim.x) {
+      int r0 = 0, nr = 0, s0 = 0, n = 0;
+      const bool in_range = group_range(b, sz, g, r0, nr, s0, n);
+      if (!(in_range && n > 0 && n <= kMaxN && nr > 0 && nr <= n)) {
+        if (gt == 0) {
+          if (!in_range || nr > n || (nr > 0 && n == 0)) report(st, GPO_ERR_SHAPE, 2, g);
+          else if (n > kMaxN || n > sz.maxn) report(st, GPO_ERR_UNSUPPORTED, 2, g);
+        }
+        continue;
+      }
+      Plan pl;
+      make_plan(n, pl);
+
+      // ---- validate the group and lay out its states (Sec. 4.2 chain layout)
+      if (gt == 0) gs->flags = (n > sz.maxn) ? 1 : 0;
+      for (int r = gt; r <= nr; r += kGThreads) {
+        gs->rstart[r] = b.rollout_step_off[r0 + r] - s0;
+        gs->tok0[r] = b.rollout_token_off[r0 + r];
+      }
+      for (int r = gt; r < nr; r += kGThreads) gs->rew[r] = b.reward[r0 + r];
+      for (int i = gt; i < n; i += kGThreads) {
+        gs->lab[i] = i;
+        gs->slen[i] = b.step_len[s0 + i];
+        gs->roll[i] = 0;
+        gs->dep[i] = 1;
+      }
+      bar_group();
+      for (int r = gt; r < nr; r += kGThreads) {
+        const int a = gs->rstart[r], e = gs->rstart[r + 1];
+        bool bad = !(a >= 0 && e > a && e <= n) || gs->rew[r] > 1;
+        if (gs->rew[r] > 1) report(st, GPO_ERR_BAD_REWARD, 2, r0 + r);
+        int64_t t = gs->tok0[r];
+        if (!bad) {
+          for (int i = a; i < e; ++i) {
+            gs->roll[i] = r;
+            gs->dep[i] = i - a + 1;
+            gs->tstart[i] = t;
+            if (gs->slen[i] < 1) bad = true;
+            t += gs->slen[i];
+          }
+          if (t != gs->tok0[r + 1] || gs->tok0[r] < 0 || gs->tok0[r + 1] > sz.T) bad = true;
+        }
+        if (bad) {
+          if (gs->rew[r] <= 1) report(st, GPO_ERR_SHAPE, 2, r0 + r);
+          atomicOr(&gs->flags, 1);
+        }
+      }
+      bar_group();
+      const bool valid = (gs->flags & 1) == 0;
+
+      // ---- drain the accumulator pass by pass (warps 4..7); warps 2..3 fetch
+      //      the prompt-embedding dots when a root embedding is given
+      bool fail = false;
+      if (!epi) {
+        if (b.root_emb && valid) {
+          const int64_t rb = (int64_t)g * sz.stride;
+          const uint16_t* Rz = reinterpret_cast<const uint16_t*>(b.root_emb);
+          const uint16_t* Z = reinterpret_cast<const uint16_t*>(b.emb);
+          for (int r = wg; r < nr + 1; r += 2) {  // r == nr: |root|^2
+            const int64_t zb = (int64_t)(s0 + gs->rstart[r < nr ? r : 0]) * sz.stride;
+            float acc = 0.f;
+            for (int k = lane; k < sz.d; k += 32) {
+              const float x = __uint_as_float((uint32_t)Rz[rb + k] << 16);
+              const float y = r < nr ? __uint_as_float((uint32_t)Z[zb + k] << 16) : x;
+              acc = fmaf(x, y, acc);
+            }
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+            if (lane == 0) {
+              if (r < nr) gs->root_dot[r] = acc;
+              else gs->root_n2 = acc;
+            }
+          }
+        }
+      } else {
+        for (int pass = 0; pass < pl.npass; ++pass, ++u) {
+          const bool got = mbar_wait(&ctl->tfull, (uint32_t)u & 1u, st, 25);
+          if (bar_any<kBarEpi, 128>(!got)) {
+            fail = true;
+            break;
+          }
+          tc_fence_after();
+          // norms and super-diagonal dots from the diagonal segments of this pass
+          for (int si = 0; si < pl.nseg[pass]; ++si) {
+            const Seg s = pl.seg[pass][si];
+            if (s.c0 != s.b * kTileM || q * 32 >= s.len) continue;  // no row of this warp in the block
+            const int i = s.b * kTileM + q * 32 + lane;
+            const uint32_t base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)s.tcol;
+            uint32_t r[32];
+            tmem_ld_32x32b_x32(base + (uint32_t)(q * 32), r);
+            tmem_wait_ld();
+            const float dg = pick(r, lane);
+            float up = pick(r, lane + 1);
+            if (q * 32 + 32 < s.len) {
+              uint32_t r2[32];
+              tmem_ld_32x32b_x32(base + (uint32_t)(q * 32 + 32), r2);
+              tmem_wait_ld();
+              if (lane == 31) up = __uint_as_float(r2[0]);
+            }
+            if (i < n) {
+              gs->n2[i] = dg;
+              if (i + 1 < n) gs->dn[i] = up;
+              if (!isfinite(dg)) report(st, GPO_ERR_NONFINITE, 2, s0 + i);
+            }
+          }
+          bar_epi();
+          for (int si = 0; si < pl.nseg[pass]; ++si) {
+            const Seg s = pl.seg[pass][si];
+            if (s.c0 != s.b * kTileM) continue;
+            const int i = s.b * kTileM + (threadIdx.x - 128);
+            if (i < n) gs->rn[i] = gs->n2[i] > 0.f ? 1.0f / sqrtf(gs->n2[i]) : 0.f;
+          }
+          bar_epi();
+          // pass masks: comparable pairs (different rollout [, same depth]) with sim >= kappa
+          uint32_t masks[4][kTileN / 32];
+#pragma unroll
+          for (int si = 0; si < 4; ++si)
+#pragma unroll
+            for (int ch = 0; ch < kTileN / 32; ++ch) masks[si][ch] = 0u;
+#pragma unroll
+          for (int si = 0; si < 4; ++si) {
+            if (si >= pl.nseg[pass]) break;
+            const Seg s = pl.seg[pass][si];
+            const int i = s.b * kTileM + q * 32 + lane;
+            const bool vrow = valid && i < n;
+            const int ri = vrow ? gs->roll[i] : -1, di = vrow ? gs->dep[i] : 0;
+            const float rni = vrow ? gs->rn[i] : 0.f;
+            const int nch = (s.len + 31) >> 5;
+#pragma unroll
+            for (int ch = 0; ch < kTileN / 32; ++ch) {
+              if (ch >= nch) break;
+              if (s.c0 + ch * 32 + 31 <= s.b * kTileM + q * 32) continue;  // no col > row in this warp
+              uint32_t r[32];
+              tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(s.tcol + ch * 32), r);
+              tmem_wait_ld();
+              uint32_t mk = 0u;
+#pragma unroll
+              for (int j = 0; j < 32; ++j) {
+                const int c = s.c0 + ch * 32 + j;  // local column
+                const int cc = c < n ? c : n - 1;
+                const bool okp = (ch * 32 + j < s.len) & (c > i) & (gs->roll[cc] != ri) &
+                                 ((p.rule != GPO_MERGE_SAME_DEPTH) | (gs->dep[cc] == di)) &
+                                 (__uint_as_float(r[j]) * rni * gs->rn[cc] >= kappa);
+                mk |= (uint32_t)okp << j;
+              }
+              masks[si][ch] = vrow ? mk : 0u;
+            }
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&ctl->tempty);  // accumulator free for the next pass
+#pragma unroll
+          for (int si = 0; si < 4; ++si) {
+            if (si >= pl.nseg[pass]) break;
+            const Seg s = pl.seg[pass][si];
+            const int i = s.b * kTileM + q * 32 + lane;
+#pragma unroll
+            for (int ch = 0; ch < kTileN / 32; ++ch) {
+              uint32_t mk = masks[si][ch];
+              while (mk) {
+                const int j = __ffs(mk) - 1;
+                mk &= mk - 1u;
+                uf_union(gs->lab, i, s.c0 + ch * 32 + j);
+              }
+            }
+          }
+        }
+      }
+      if (bar_any<kBarGroup, kGThreads>(fail)) break;
+
+      // ---- graph reward and dual-group advantage of every edge (fp64)
+      if (valid) {
+        auto eta = [&](int i) -> double {
+          double e = 0.0;
+          if (gs->dep[i] == 1) {
+            if (b.root_emb) {
+              const double n1 = gs->root_n2, n2v = gs->n2[i];
+              if (n1 > 0.0 && n2v > 0.0) e = (double)gs->root_dot[gs->roll[i]] / sqrt(n1 * n2v);
+            }
+          } else {
+            const double n1 = gs->n2[i - 1], n2v = gs->n2[i];
+            if (n1 > 0.0 && n2v > 0.0) e = (double)gs->dn[i - 1] / sqrt(n1 * n2v);
+          }
+          return e > 0.0 ? e : 0.0;
+        };
+        auto out = [&](int i, int label, double S, double acor, double E, double dual, unsigned char mask) {
+          gs->eadv[i] = (float)dual;
+          gs->ecor[i] = (float)acor;
+          gs->eeff[i] = (float)E;
+          gs->emask[i] = mask;
+          const int v = s0 + i;
+          if (o.edge_adv) o.edge_adv[v] = (float)dual;
+          if (o.class_id) o.class_id[v] = s0 + label;
+          if (o.node_score) o.node_score[v] = (float)S;
+        };
+        group_advantages<2>(n, nr, gs->lab, gs->roll, gs->dep, gs->rstart, gs->rew, gs->X, p, gt, kGThreads,
+                            [] { bar_group(); }, eta, out);
+        // ---- every token of an edge carries the edge's advantage (Sec. 4.5)
+        for (int i = wg; i < n; i += kGThreads / 32) {
+          const int64_t ts = gs->tstart[i], te = ts + gs->slen[i];
+          write_span(o.adv, ts, te, gs->eadv[i], lane);
+          if (o.adv_cor) write_span(o.adv_cor, ts, te, gs->ecor[i], lane);
+          if (o.adv_eff) write_span(o.adv_eff, ts, te, gs->eeff[i], lane);
+          if (o.eff_mask) write_span_u8(o.eff_mask, ts, te, gs->emask[i], lane);
+        }
+      }
+      bar_group();
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, kTmemCols);
+}
+
+size_t fused_smem() { return (size_t)kStages * kStageBytes + 256 + sizeof(GroupSmem) + 1024; }
+
+}  // namespace
+
+cudaError_t setup_fused() {
+  return cudaFuncSetAttribute(fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)fused_smem());
+}
+
+cudaError_t launch_fused(const LaunchCtx& lc, const CUtensorMap& map, const gpo_batch& b, const gpo_outputs& o,
+                         const Sizes& sz, const Ws& ws, const Params& p) {
+  if (sz.G == 0) return cudaSuccess;
+  const int grid = sz.G < lc.num_sms ? sz.G : lc.num_sms;
+  fused_kernel<<<grid, kThreads, fused_smem(), lc.stream>>>(map, b, o, sz, ws, p);
+  return cudaGetLastError();
+}
+
+}  // namespace gpo

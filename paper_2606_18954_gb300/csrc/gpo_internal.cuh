@@ -19,6 +19,7 @@ constexpr int kTileK = 64;           // bf16 elements per 128-byte swizzle row
 constexpr int kEdgeCap = 384;        // spanning-forest edges one item can emit (< rows+cols)
 constexpr int kStatusWords = 16;
 constexpr int kMaxStages = 8;        // timed stages of one gpo_compute
+constexpr int kFusedMaxStates = 384; // largest group of the fused group-resident kernel
 
 // status words (uint32) at the head of the workspace
 enum : int {
@@ -249,6 +250,28 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
 }
 
+// ------------------------------------------------------------------ token spans
+
+// One warp writes value v to dst[ts, te): 16-byte stores in the aligned middle,
+// scalar stores for the unaligned ends (dst must be 16-byte aligned).
+__device__ __forceinline__ void write_span(float* dst, int64_t ts, int64_t te, float v, int lane) {
+  const int64_t a = min(te, (ts + 3) & ~int64_t(3));
+  const int64_t z = max(a, te & ~int64_t(3));
+  if (lane < a - ts) dst[ts + lane] = v;
+  const float4 v4 = make_float4(v, v, v, v);
+  for (int64_t q = (a >> 2) + lane; q < (z >> 2); q += 32) reinterpret_cast<float4*>(dst)[q] = v4;
+  if (lane < te - z) dst[z + lane] = v;
+}
+
+__device__ __forceinline__ void write_span_u8(uint8_t* dst, int64_t ts, int64_t te, uint8_t v, int lane) {
+  const int64_t a = min(te, (ts + 3) & ~int64_t(3));
+  const int64_t z = max(a, te & ~int64_t(3));
+  if (lane < a - ts) dst[ts + lane] = v;
+  const uint32_t v4 = 0x01010101u * v;
+  for (int64_t q = (a >> 2) + lane; q < (z >> 2); q += 32) reinterpret_cast<uint32_t*>(dst)[q] = v4;
+  if (lane < te - z) dst[z + lane] = v;
+}
+
 // ------------------------------------------------------------------ launchers (host)
 
 struct LaunchCtx {
@@ -270,6 +293,9 @@ cudaError_t launch_tokens(const LaunchCtx& lc, const gpo_batch& b, const gpo_out
 // Records a message on the context (gpo_last_error).
 void note_error(gpo_ctx* ctx, const char* msg);
 
+cudaError_t launch_fused(const LaunchCtx& lc, const CUtensorMap& map, const gpo_batch& b, const gpo_outputs& o,
+                         const Sizes& sz, const Ws& ws, const Params& p);
+cudaError_t setup_fused();
 cudaError_t setup_sim_tc();
 cudaError_t setup_groups();
 size_t sim_tc_smem_bytes();

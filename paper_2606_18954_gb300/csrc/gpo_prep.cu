@@ -266,24 +266,6 @@ cudaError_t launch_row_stats(const LaunchCtx& lc, const gpo_batch& b, const Size
 // one coalesced round trip and broadcast by shuffles; each span is written
 // with 16-byte stores in its aligned middle and scalar stores at the ends.
 
-__device__ __forceinline__ void write_span(float* dst, int64_t ts, int64_t te, float v, int lane) {
-  const int64_t a = min(te, (ts + 3) & ~int64_t(3));
-  const int64_t z = max(a, te & ~int64_t(3));
-  if (lane < a - ts) dst[ts + lane] = v;
-  const float4 v4 = make_float4(v, v, v, v);
-  for (int64_t q = (a >> 2) + lane; q < (z >> 2); q += 32) reinterpret_cast<float4*>(dst)[q] = v4;
-  if (lane < te - z) dst[z + lane] = v;
-}
-
-__device__ __forceinline__ void write_span_u8(uint8_t* dst, int64_t ts, int64_t te, uint8_t v, int lane) {
-  const int64_t a = min(te, (ts + 3) & ~int64_t(3));
-  const int64_t z = max(a, te & ~int64_t(3));
-  if (lane < a - ts) dst[ts + lane] = v;
-  const uint32_t v4 = 0x01010101u * v;
-  for (int64_t q = (a >> 2) + lane; q < (z >> 2); q += 32) reinterpret_cast<uint32_t*>(dst)[q] = v4;
-  if (lane < te - z) dst[z + lane] = v;
-}
-
 __global__ void __launch_bounds__(256) tokens_kernel(gpo_batch b, gpo_outputs o, Sizes sz, Ws ws) {
   if (aborted(ws.status)) return;
   const int lane = threadIdx.x & 31;

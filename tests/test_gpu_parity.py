@@ -93,24 +93,30 @@ def oracle_run(b, params, threads=8):
 SCALED = [("tiny", 8), ("math", 4), ("agentic", 24), ("full", 3), ("wide", 1)]
 
 
+# fused: the group-resident kernel (bf16, groups <= 384 states); tiled: the
+# multi-kernel tensor-core path; simt: the multi-kernel CUDA-core path
+PATH_FLAGS = {"fused": 0, "tiled": 2, "simt": 1}
+
+
 @pytest.mark.parametrize("name,groups", SCALED)
 @pytest.mark.parametrize("rule", [0, 1])
-@pytest.mark.parametrize("path", ["tc", "simt"])
+@pytest.mark.parametrize("path", ["fused", "tiled", "simt"])
 def test_parity_scaled(gp_mod, name, groups, rule, path):
     b = batch_of(name, groups)
-    if path == "tc" and b["emb_dtype"] != "bf16":
+    if path != "simt" and b["emb_dtype"] != "bf16":
         pytest.skip("fp32 embeddings always use the CUDA-core similarity kernel")
     params = oracle_params(b, merge_rule=rule)
     ref = oracle_run(b, params)
-    gpu = run_gpu(gp_mod, b, params, flags=1 if path == "simt" else 0)
+    gpu = run_gpu(gp_mod, b, params, flags=PATH_FLAGS[path])
     compare(gpu, ref, f"{name}/{rule}/{path}")
 
 
 @pytest.mark.parametrize("lam", [0.0, 0.5])
-def test_parity_lambda(gp_mod, lam):
+@pytest.mark.parametrize("path", ["fused", "tiled"])
+def test_parity_lambda(gp_mod, lam, path):
     b = batch_of("math", 3)
     params = oracle_params(b, lambda_eff=lam)
-    compare(run_gpu(gp_mod, b, params), oracle_run(b, params), f"lambda={lam}")
+    compare(run_gpu(gp_mod, b, params, flags=PATH_FLAGS[path]), oracle_run(b, params), f"lambda={lam}")
 
 
 def test_parity_root_embedding(gp_mod):
@@ -126,14 +132,16 @@ def test_parity_root_embedding(gp_mod):
     params = oracle_params(b)
     ref = oracle_run(b, params)
     assert np.any(ref["eta"][first] > 0)
-    compare(run_gpu(gp_mod, b, params), ref, "root_emb")
+    for path in ("fused", "tiled"):
+        compare(run_gpu(gp_mod, b, params, flags=PATH_FLAGS[path]), ref, f"root_emb/{path}")
 
 
-def test_deterministic(gp_mod):
+@pytest.mark.parametrize("path", ["fused", "tiled"])
+def test_deterministic(gp_mod, path):
     b = batch_of("math", 4)
     params = oracle_params(b)
-    a1 = run_gpu(gp_mod, b, params)
-    a2 = run_gpu(gp_mod, b, params)
+    a1 = run_gpu(gp_mod, b, params, flags=PATH_FLAGS[path])
+    a2 = run_gpu(gp_mod, b, params, flags=PATH_FLAGS[path])
     for k in a1:
         np.testing.assert_array_equal(a1[k], a2[k], err_msg=k)
 
@@ -181,13 +189,13 @@ EDGE_CASES = {
 
 
 @pytest.mark.parametrize("case", sorted(EDGE_CASES))
-@pytest.mark.parametrize("path", ["tc", "simt"])
+@pytest.mark.parametrize("path", ["fused", "tiled", "simt"])
 def test_edge_cases(gp_mod, case, path):
-    rng = np.random.default_rng(abs(hash(case)) % 2**32)
+    rng = np.random.default_rng(sum(map(ord, case)))
     b = from_rollouts(EDGE_CASES[case](rng), dtype="bf16", kappa=0.9, w=0.7, lambda_eff=1.0)
     assert _margin_ok(b, 0.9)
     params = oracle_params(b)
-    compare(run_gpu(gp_mod, b, params, flags=1 if path == "simt" else 0), oracle_run(b, params), case)
+    compare(run_gpu(gp_mod, b, params, flags=PATH_FLAGS[path]), oracle_run(b, params), case)
 
 
 def test_zero_rows_and_f32(gp_mod):
@@ -212,9 +220,9 @@ def test_largest_group(gp_mod):
 # --------------------------------------------------------------------- errors
 
 
-def _expect_status(P, b, code, host=False):
+def _expect_status(P, b, code, host=False, flags=0):
     import torch
-    gp = P.GraphPO()
+    gp = P.GraphPO(flags=flags)
     db = P.Batch.from_arrays(b, device="cuda")
     if host:
         with pytest.raises(P.GraphPOError) as e:
@@ -233,39 +241,47 @@ def _expect_status(P, b, code, host=False):
     torch.cuda.synchronize()
 
 
-def test_error_bad_reward(gp_mod):
+ERR_PATHS = pytest.mark.parametrize("flags", [0, 2], ids=["fused", "tiled"])
+
+
+@ERR_PATHS
+def test_error_bad_reward(gp_mod, flags):
     b = dict(batch_of("math", 2))
     b["reward"] = b["reward"].copy()
     b["reward"][5] = 2
-    _expect_status(gp_mod, b, 3)
+    _expect_status(gp_mod, b, 3, flags=flags)
 
 
-def test_error_bad_step_len(gp_mod):
+@ERR_PATHS
+def test_error_bad_step_len(gp_mod, flags):
     b = dict(batch_of("math", 2))
     b["step_len"] = b["step_len"].copy()
     b["step_len"][7] = 0
-    _expect_status(gp_mod, b, 2)
+    _expect_status(gp_mod, b, 2, flags=flags)
 
 
-def test_error_token_spans(gp_mod):
+@ERR_PATHS
+def test_error_token_spans(gp_mod, flags):
     b = dict(batch_of("math", 2))
     b["rollout_token_off"] = b["rollout_token_off"].copy()
     b["rollout_token_off"][3] += 1
-    _expect_status(gp_mod, b, 2)
+    _expect_status(gp_mod, b, 2, flags=flags)
 
 
-def test_error_offsets_out_of_range(gp_mod):
+@ERR_PATHS
+def test_error_offsets_out_of_range(gp_mod, flags):
     b = dict(batch_of("math", 2))
     b["rollout_step_off"] = b["rollout_step_off"].copy()
     b["rollout_step_off"][4] = 10 ** 6
-    _expect_status(gp_mod, b, 2)
+    _expect_status(gp_mod, b, 2, flags=flags)
 
 
-def test_error_nonfinite(gp_mod):
+@ERR_PATHS
+def test_error_nonfinite(gp_mod, flags):
     b = dict(batch_of("math", 2))
     b["emb"] = b["emb"].copy()
     b["emb"][9, 17] = 0x7FC0  # bf16 quiet NaN
-    _expect_status(gp_mod, b, 4)
+    _expect_status(gp_mod, b, 4, flags=flags)
 
 
 def test_error_group_too_large(gp_mod):
