@@ -72,6 +72,7 @@ def algorithmic(b):
         "similarity": (zb + 12 * N, flops),
         "groups": (8 * N + R + 12 * R + 4 * N + 17 * N + 8 * N, 0.0),
         "tokens": (4 * T + 8 * N + 4 * N + 4 * N, 0.0),
+        "fused": (path_bytes, flops),  # the group-resident kernel does the whole path
     }
     return dict(N=N, R=R, G=G, T=T, path_bytes=path_bytes, flops=flops, stages=stages)
 
@@ -150,7 +151,7 @@ def traffic_for(kernel_file):
 
 
 STAGE_SOURCE = {"prep": "gpo_prep.cu", "row_stats": "gpo_prep.cu", "similarity": "gpo_sim_tc.cu",
-                "groups": "gpo_group.cu", "tokens": "gpo_prep.cu"}
+                "groups": "gpo_group.cu", "tokens": "gpo_prep.cu", "fused": "gpo_fused.cu"}
 
 
 def cpu_baseline(b, budget_s=6.0, max_groups=None):

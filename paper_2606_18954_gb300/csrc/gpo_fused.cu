@@ -132,7 +132,10 @@ struct __align__(16) GroupSmem {
   uint8_t emask[kMaxN];
   int flags;             // bit 0: group invalid
   float root_n2;
-  unsigned char X[group_scratch_bytes(kMaxN)];
+  Plan plan;
+  int ckey[kMaxN];       // rollout << 12 | depth (same-depth rule), rollout << 12 (non-causal rule)
+  uint32_t masks[4 * (kTileN / 32)][128];  // pass masks: [segment*8 + chunk][epilogue thread]
+  alignas(16) unsigned char X[group_scratch_bytes(kMaxN)];  // holds int64 and fp64 arrays
 };
 
 struct __align__(8) Ctl {
@@ -299,11 +302,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         continue;
       }
-      Plan pl;
-      make_plan(n, pl);
+      if (gt == 0) {
+        make_plan(n, gs->plan);
+        gs->flags = (n > sz.maxn) ? 1 : 0;
+      }
 
       // ---- validate the group and lay out its states (Sec. 4.2 chain layout)
-      if (gt == 0) gs->flags = (n > sz.maxn) ? 1 : 0;
       for (int r = gt; r <= nr; r += kGThreads) {
         gs->rstart[r] = b.rollout_step_off[r0 + r] - s0;
         gs->tok0[r] = b.rollout_token_off[r0 + r];
@@ -325,6 +329,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int i = a; i < e; ++i) {
             gs->roll[i] = r;
             gs->dep[i] = i - a + 1;
+            gs->ckey[i] = (r << 12) | (p.rule == GPO_MERGE_SAME_DEPTH ? (i - a + 1) & 0xFFF : 0);
             gs->tstart[i] = t;
             if (gs->slen[i] < 1) bad = true;
             t += gs->slen[i];
@@ -364,6 +369,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       } else {
+        const Plan& pl = gs->plan;
+        const int t128 = threadIdx.x - 128;
         for (int pass = 0; pass < pl.npass; ++pass, ++u) {
           const bool got = mbar_wait(&ctl->tfull, (uint32_t)u & 1u, st, 25);
           if (bar_any<kBarEpi, 128>(!got)) {
@@ -371,22 +378,23 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           }
           tc_fence_after();
+          const int nseg = pl.nseg[pass];
           // norms and super-diagonal dots from the diagonal segments of this pass
-          for (int si = 0; si < pl.nseg[pass]; ++si) {
-            const Seg s = pl.seg[pass][si];
-            if (s.c0 != s.b * kTileM || q * 32 >= s.len) continue;  // no row of this warp in the block
-            const int i = s.b * kTileM + q * 32 + lane;
-            const uint32_t base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)s.tcol;
+#pragma unroll 1
+          for (int si = 0; si < nseg; ++si) {
+            const Seg sg = pl.seg[pass][si];
+            if (sg.c0 != sg.b * kTileM || q * 32 >= sg.len) continue;  // no row of this warp here
+            const int i = sg.b * kTileM + q * 32 + lane;
+            const uint32_t base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)sg.tcol;
             uint32_t r[32];
             tmem_ld_32x32b_x32(base + (uint32_t)(q * 32), r);
             tmem_wait_ld();
             const float dg = pick(r, lane);
             float up = pick(r, lane + 1);
-            if (q * 32 + 32 < s.len) {
-              uint32_t r2[32];
-              tmem_ld_32x32b_x32(base + (uint32_t)(q * 32 + 32), r2);
+            if (q * 32 + 32 < sg.len) {
+              tmem_ld_32x32b_x32(base + (uint32_t)(q * 32 + 32), r);
               tmem_wait_ld();
-              if (lane == 31) up = __uint_as_float(r2[0]);
+              if (lane == 31) up = __uint_as_float(r[0]);
             }
             if (i < n) {
               gs->n2[i] = dg;
@@ -395,63 +403,62 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
           bar_epi();
-          for (int si = 0; si < pl.nseg[pass]; ++si) {
-            const Seg s = pl.seg[pass][si];
-            if (s.c0 != s.b * kTileM) continue;
-            const int i = s.b * kTileM + (threadIdx.x - 128);
+#pragma unroll 1
+          for (int si = 0; si < nseg; ++si) {
+            const Seg sg = pl.seg[pass][si];
+            if (sg.c0 != sg.b * kTileM) continue;
+            const int i = sg.b * kTileM + t128;
             if (i < n) gs->rn[i] = gs->n2[i] > 0.f ? 1.0f / sqrtf(gs->n2[i]) : 0.f;
           }
           bar_epi();
           // pass masks: comparable pairs (different rollout [, same depth]) with sim >= kappa
-          uint32_t masks[4][kTileN / 32];
-#pragma unroll
-          for (int si = 0; si < 4; ++si)
-#pragma unroll
-            for (int ch = 0; ch < kTileN / 32; ++ch) masks[si][ch] = 0u;
-#pragma unroll
-          for (int si = 0; si < 4; ++si) {
-            if (si >= pl.nseg[pass]) break;
-            const Seg s = pl.seg[pass][si];
-            const int i = s.b * kTileM + q * 32 + lane;
+#pragma unroll 1
+          for (int si = 0; si < nseg; ++si) {
+            const Seg sg = pl.seg[pass][si];
+            const int i = sg.b * kTileM + q * 32 + lane;
             const bool vrow = valid && i < n;
-            const int ri = vrow ? gs->roll[i] : -1, di = vrow ? gs->dep[i] : 0;
+            const int ki = vrow ? gs->ckey[i] : -1;
             const float rni = vrow ? gs->rn[i] : 0.f;
-            const int nch = (s.len + 31) >> 5;
-#pragma unroll
-            for (int ch = 0; ch < kTileN / 32; ++ch) {
-              if (ch >= nch) break;
-              if (s.c0 + ch * 32 + 31 <= s.b * kTileM + q * 32) continue;  // no col > row in this warp
-              uint32_t r[32];
-              tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(s.tcol + ch * 32), r);
-              tmem_wait_ld();
+            const int nch = (sg.len + 31) >> 5;
+#pragma unroll 1
+            for (int ch = 0; ch < nch; ++ch) {
               uint32_t mk = 0u;
+              if (sg.c0 + ch * 32 + 31 > sg.b * kTileM + q * 32) {  // some col > row in this warp
+                uint32_t r[32];
+                tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(sg.tcol + ch * 32), r);
+                tmem_wait_ld();
+                const int cbase = sg.c0 + ch * 32;
+                const int cend = min(32, sg.len - ch * 32);
 #pragma unroll
-              for (int j = 0; j < 32; ++j) {
-                const int c = s.c0 + ch * 32 + j;  // local column
-                const int cc = c < n ? c : n - 1;
-                const bool okp = (ch * 32 + j < s.len) & (c > i) & (gs->roll[cc] != ri) &
-                                 ((p.rule != GPO_MERGE_SAME_DEPTH) | (gs->dep[cc] == di)) &
-                                 (__uint_as_float(r[j]) * rni * gs->rn[cc] >= kappa);
-                mk |= (uint32_t)okp << j;
+                for (int j = 0; j < 32; ++j) {
+                  const int c = min(cbase + j, n - 1);
+                  // comparable: different rollout, and equal depth bits (always equal under the
+                  // non-causal rule, whose keys carry no depth)
+                  const int x = gs->ckey[c] ^ ki;
+                  const bool okp = (j < cend) & (cbase + j > i) & ((x >> 12) != 0) & ((x & 0xFFF) == 0) &
+                                   (__uint_as_float(r[j]) * rni * gs->rn[c] >= kappa);
+                  mk |= (uint32_t)okp << j;
+                }
+                if (!vrow) mk = 0u;
               }
-              masks[si][ch] = vrow ? mk : 0u;
+              gs->masks[si * 8 + ch][t128] = mk;
             }
           }
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&ctl->tempty);  // accumulator free for the next pass
-#pragma unroll
-          for (int si = 0; si < 4; ++si) {
-            if (si >= pl.nseg[pass]) break;
-            const Seg s = pl.seg[pass][si];
-            const int i = s.b * kTileM + q * 32 + lane;
-#pragma unroll
-            for (int ch = 0; ch < kTileN / 32; ++ch) {
-              uint32_t mk = masks[si][ch];
+#pragma unroll 1
+          for (int si = 0; si < nseg; ++si) {
+            const Seg sg = pl.seg[pass][si];
+            const int i = sg.b * kTileM + q * 32 + lane;
+            const int nch = (sg.len + 31) >> 5;
+#pragma unroll 1
+            for (int ch = 0; ch < nch; ++ch) {
+              uint32_t mk = gs->masks[si * 8 + ch][t128];
               while (mk) {
                 const int j = __ffs(mk) - 1;
                 mk &= mk - 1u;
-                uf_union(gs->lab, i, s.c0 + ch * 32 + j);
+                uf_union(gs->lab, i, sg.c0 + ch * 32 + j);
               }
             }
           }
@@ -461,28 +468,30 @@ __global__ void __launch_bounds__(kThreads, 1)
 
       // ---- graph reward and dual-group advantage of every edge (fp64)
       if (valid) {
-        auto eta = [&](int i) -> double {
-          double e = 0.0;
+        auto eta = [&](int i) -> float {
+          float e = 0.f, n1 = 0.f, dot = 0.f;
           if (gs->dep[i] == 1) {
             if (b.root_emb) {
-              const double n1 = gs->root_n2, n2v = gs->n2[i];
-              if (n1 > 0.0 && n2v > 0.0) e = (double)gs->root_dot[gs->roll[i]] / sqrt(n1 * n2v);
+              n1 = gs->root_n2;
+              dot = gs->root_dot[gs->roll[i]];
             }
           } else {
-            const double n1 = gs->n2[i - 1], n2v = gs->n2[i];
-            if (n1 > 0.0 && n2v > 0.0) e = (double)gs->dn[i - 1] / sqrt(n1 * n2v);
+            n1 = gs->n2[i - 1];
+            dot = gs->dn[i - 1];
           }
-          return e > 0.0 ? e : 0.0;
+          const float n2v = gs->n2[i];
+          if (n1 > 0.f && n2v > 0.f) e = dot / sqrtf(n1 * n2v);
+          return e > 0.f ? e : 0.f;
         };
-        auto out = [&](int i, int label, double S, double acor, double E, double dual, unsigned char mask) {
-          gs->eadv[i] = (float)dual;
-          gs->ecor[i] = (float)acor;
-          gs->eeff[i] = (float)E;
+        auto out = [&](int i, int label, float S, float acor, float E, float dual, unsigned char mask) {
+          gs->eadv[i] = dual;
+          gs->ecor[i] = acor;
+          gs->eeff[i] = E;
           gs->emask[i] = mask;
           const int v = s0 + i;
-          if (o.edge_adv) o.edge_adv[v] = (float)dual;
+          if (o.edge_adv) o.edge_adv[v] = dual;
           if (o.class_id) o.class_id[v] = s0 + label;
-          if (o.node_score) o.node_score[v] = (float)S;
+          if (o.node_score) o.node_score[v] = S;
         };
         group_advantages<2>(n, nr, gs->lab, gs->roll, gs->dep, gs->rstart, gs->rew, gs->X, p, gt, kGThreads,
                             [] { bar_group(); }, eta, out);

@@ -57,29 +57,31 @@ __global__ void __launch_bounds__(1024) groups_kernel(gpo_batch b, gpo_outputs o
   __syncthreads();
 
   // eta(p(v), v) from the fp32 row statistics; zero rows give 0
-  auto eta = [&](int i) -> double {
+  auto eta = [&](int i) -> float {
     const int v = s0 + i;
-    double e = 0.0;
+    float e = 0.f, n1 = 0.f, dot = 0.f;
     if (dep[i] == 1) {
       if (b.root_emb) {
-        const float n1 = ws.root_n2[g], n2 = ws.nrm2[v];
-        if (n1 > 0.f && n2 > 0.f) e = (double)ws.dotp[v] / sqrt((double)n1 * (double)n2);
+        n1 = ws.root_n2[g];
+        dot = ws.dotp[v];
       }
     } else {
-      const float n1 = ws.nrm2[v - 1], n2 = ws.nrm2[v];
-      if (n1 > 0.f && n2 > 0.f) e = (double)ws.dotp[v] / sqrt((double)n1 * (double)n2);
+      n1 = ws.nrm2[v - 1];
+      dot = ws.dotp[v];
     }
-    return e > 0.0 ? e : 0.0;
+    const float n2 = ws.nrm2[v];
+    if (n1 > 0.f && n2 > 0.f) e = dot / sqrtf(n1 * n2);
+    return e > 0.f ? e : 0.f;
   };
-  auto out = [&](int i, int label, double S, double acor, double E, double dual, unsigned char mask) {
+  auto out = [&](int i, int label, float S, float acor, float E, float dual, unsigned char mask) {
     const int v = s0 + i;
-    ws.e_adv[v] = (float)dual;
-    ws.e_cor[v] = (float)acor;
-    ws.e_eff[v] = (float)E;
+    ws.e_adv[v] = dual;
+    ws.e_cor[v] = acor;
+    ws.e_eff[v] = E;
     ws.e_mask[v] = mask;
-    if (o.edge_adv) o.edge_adv[v] = (float)dual;
+    if (o.edge_adv) o.edge_adv[v] = dual;
     if (o.class_id) o.class_id[v] = s0 + label;
-    if (o.node_score) o.node_score[v] = (float)S;
+    if (o.node_score) o.node_score[v] = S;
   };
   group_advantages<kPer>(n, nr, lab, roll, dep, rstart, rew, X, p, tid, nt, [] { __syncthreads(); }, eta, out);
 
