@@ -76,7 +76,8 @@ typedef enum {
 typedef enum { GPO_EMB_BF16 = 0, GPO_EMB_F32 = 1 } gpo_emb_dtype;
 
 typedef struct {
-  double kappa;      /* merge threshold: linked when sim >= kappa (Sec. 4.2; paper uses 0.92) */
+  double kappa;      /* merge threshold, > 0: linked when sim >= kappa (Sec. 4.2; the paper
+                        takes kappa in (0,1) and uses 0.92; kappa > 1 disables merging) */
   double w;          /* pooling coefficient in [0,1], Eq. (combain) (paper uses 0.7) */
   double lambda_eff; /* >= 0, weight of A_eff in A_dual (Sec. 4.5; paper gives no value) */
   double std_eps;    /* >= 0, added to every standard deviation (GRPO convention 1e-6) */

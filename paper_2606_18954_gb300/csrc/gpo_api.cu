@@ -124,7 +124,7 @@ Ws workspace_views(void* base, const Layout& L) {
 }
 
 gpo_status check_params(const gpo_params& p) {
-  if (!std::isfinite(p.kappa) || !(p.w >= 0.0 && p.w <= 1.0) || !(p.lambda_eff >= 0.0) ||
+  if (!std::isfinite(p.kappa) || !(p.kappa > 0.0) || !(p.w >= 0.0 && p.w <= 1.0) || !(p.lambda_eff >= 0.0) ||
       !std::isfinite(p.lambda_eff) || !(p.std_eps >= 0.0) || !std::isfinite(p.std_eps) || p.std_ddof < 0 ||
       p.std_ddof > 1 || p.merge_rule < 0 || p.merge_rule > 1 || (p.flags & ~(GPO_FLAG_SIMT_SIMILARITY | GPO_FLAG_TILED)))
     return GPO_ERR_INVALID_ARG;
@@ -293,19 +293,25 @@ gpo_status gpo_compute(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* 
   lc.num_sms = ctx->num_sms;
 
   const bool use_tc = b.emb_dtype == GPO_EMB_BF16 && !(p.flags & GPO_FLAG_SIMT_SIMILARITY) && sz.N > 0;
-  CUtensorMap map;
+  // embedding tensor maps: boxes of 64 elements x 128 rows and x 32 rows, 128B swizzle
+  CUtensorMap map, map32;
   memset(&map, 0, sizeof map);
+  memset(&map32, 0, sizeof map32);
   if (use_tc) {
     EncodeTiledFn enc = encode_fn();
     if (!enc) return set_msg(ctx, "cuTensorMapEncodeTiled unavailable"), GPO_ERR_CUDA;
     const cuuint64_t dims[2] = {(cuuint64_t)sz.d, (cuuint64_t)sz.N};
     const cuuint64_t strides[1] = {(cuuint64_t)(sz.stride * 2)};
-    const cuuint32_t box[2] = {(cuuint32_t)kTileK, (cuuint32_t)kTileM};
     const cuuint32_t estr[2] = {1, 1};
-    const CUresult r = enc(&map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(b.emb), dims, strides, box,
-                           estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    if (r != CUDA_SUCCESS) return set_msg(ctx, "cuTensorMapEncodeTiled failed (%d)", (int)r), GPO_ERR_UNSUPPORTED;
+    CUtensorMap* maps[2] = {&map, &map32};
+    const cuuint32_t rows[2] = {(cuuint32_t)kTileM, 32};
+    for (int m = 0; m < 2; ++m) {
+      const cuuint32_t box[2] = {(cuuint32_t)kTileK, rows[m]};
+      const CUresult r = enc(maps[m], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(b.emb), dims, strides, box,
+                             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+      if (r != CUDA_SUCCESS) return set_msg(ctx, "cuTensorMapEncodeTiled failed (%d)", (int)r), GPO_ERR_UNSUPPORTED;
+    }
   }
 
   int ns = 0;
@@ -321,7 +327,7 @@ gpo_status gpo_compute(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* 
   if (e == cudaSuccess) e = cudaMemsetAsync(ws.status, 0, sizeof(uint32_t) * kStatusWords, lc.stream);
   const bool fused = use_tc && !(p.flags & GPO_FLAG_TILED) && sz.G > 0 && sz.maxn <= kFusedMaxStates;
   if (fused) {
-    if (e == cudaSuccess) e = stage("fused", launch_fused(lc, map, b, *out, sz, ws, pp));
+    if (e == cudaSuccess) e = stage("fused", launch_fused(lc, map, map32, b, *out, sz, ws, pp));
   } else {
   if (e == cudaSuccess) e = stage("prep", launch_prep(lc, b, sz, ws));
   if (e == cudaSuccess && sz.N > 0) {

@@ -10,15 +10,16 @@
 //                   [128 b, n), at most 512 accumulator columns per pass;
 //                   if a group needs more, blocks >= 1 go first, block 0 second
 //                   (Sec. 4.2: sim of every comparable pair)
-//   warps 4..7      TMEM drain of each pass: the diagonal and super-diagonal
-//                   entries give |z_i|^2 and <z_i, z_{i+1}> (the norms of the
-//                   cosine and eta(p(v), v)); then cos = acc / (|z_i||z_j|),
-//                   pair mask (different rollout; optionally same depth) and
-//                   threshold sim >= kappa into pass masks, then shared-memory
-//                   union-find (Alg. S.1); the accumulator is released before
-//                   the unions so the next pass / group can start
-//   warps 2..7      per-group validation, graph reward and dual-group advantage
-//                   (gpo_group_math.cuh, fp64) and the token scatter (Sec. 4.5),
+//   warps 4..15     TMEM drain of each pass (three warps per accumulator lane
+//                   quarter, splitting the 32-column chunks): the diagonal and
+//                   super-diagonal entries give |z_i|^2 and <z_i, z_{i+1}> (the
+//                   norms of the cosine and eta(p(v), v)); then every comparable
+//                   pair (different rollout; optionally same depth) with
+//                   cos = acc / (|z_i||z_j|) >= kappa goes to an edge list; the
+//                   accumulator is released and the listed pairs are united in a
+//                   shared-memory union-find forest (Alg. S.1)
+//   warps 2..15     per-group validation, graph reward and dual-group advantage
+//                   (gpo_group_math.cuh) and the token scatter (Sec. 4.5),
 //                   overlapping the next group's loads and MMAs
 // Group ranges are assigned round-robin to CTAs.  Every wait is bounded.
 #include "gpo_group_math.cuh"
@@ -27,15 +28,18 @@ namespace gpo {
 
 namespace {
 
-constexpr int kStages = 3;
-constexpr int kThreads = 256;
+constexpr int kMaxSlots = 8;                    // pipeline stages at most
+constexpr int kRingBytes = 160 * 1024;          // tile ring: slots of r32(max states) rows x 128 bytes
+constexpr int kThreads = 512;
 constexpr int kMaxN = kFusedMaxStates;          // 384
 constexpr int kBoxBytes = kTileM * 128;         // 128 rows x 128 bytes
-constexpr int kStageBytes = 3 * kBoxBytes;      // up to 384 rows
+constexpr int kTailRows = 32;                   // rows of the second tensor map's box
 constexpr int kTmemCols = 512;
-constexpr int kGThreads = 192;                  // warps 2..7
-constexpr int kBarGroup = 1;                    // named barrier of warps 2..7
-constexpr int kBarEpi = 2;                      // named barrier of warps 4..7
+constexpr int kGThreads = 448;                  // warps 2..15
+constexpr int kEpiThreads = 384;                // warps 4..15: three per accumulator lane quarter
+constexpr int kEdgeList = 4096;                 // linked pairs listed per pass
+constexpr int kBarGroup = 1;                    // named barrier of warps 2..15
+constexpr int kBarEpi = 2;                      // named barrier of warps 4..15
 
 struct Seg {
   int b, c0, len, tcol;  // row block, first column (local), columns, TMEM column
@@ -112,7 +116,7 @@ __device__ __forceinline__ bool group_range(const gpo_batch& b, const Sizes& sz,
 // Group handled here (all roles agree, they read the same inputs).
 __device__ __forceinline__ bool group_active(const gpo_batch& b, const Sizes& sz, int g, int& r0, int& nr, int& s0,
                                              int& n) {
-  return group_range(b, sz, g, r0, nr, s0, n) && n > 0 && n <= kMaxN && nr > 0 && nr <= n;
+  return group_range(b, sz, g, r0, nr, s0, n) && n > 0 && n <= kMaxN && n <= sz.maxn && nr > 0 && nr <= n;
 }
 
 struct __align__(16) GroupSmem {
@@ -131,24 +135,31 @@ struct __align__(16) GroupSmem {
   uint8_t rew[kMaxN];
   uint8_t emask[kMaxN];
   int flags;             // bit 0: group invalid
+  int ecount;            // linked pairs of the current pass (edge list in X)
   float root_n2;
   Plan plan;
-  int ckey[kMaxN];       // rollout << 12 | depth (same-depth rule), rollout << 12 (non-causal rule)
-  uint32_t masks[4 * (kTileN / 32)][128];  // pass masks: [segment*8 + chunk][epilogue thread]
-  alignas(16) unsigned char X[group_scratch_bytes(kMaxN)];  // holds int64 and fp64 arrays
+  int2 col[kMaxN];       // {depth, bits of 1/|z|} of every state, read per column by the pair loop
+  uint32_t elist[kEdgeList];  // linked pairs of the pass: i | j << 16
+  alignas(16) unsigned char X[group_scratch_sep_bytes(kMaxN)];  // group-math sums (separate layout)
 };
 
 struct __align__(8) Ctl {
-  uint64_t full[kStages];
-  uint64_t empty[kStages];
+  uint64_t full[kMaxSlots];
+  uint64_t empty[kMaxSlots];
   uint64_t tfull;
   uint64_t tempty;
   uint64_t drain;
   uint32_t tmem_base;
 };
 
+constexpr uint32_t kCtlOff = (sizeof(GroupSmem) + 15) & ~15u;
+constexpr uint32_t kTilesOff = kCtlOff + ((sizeof(Ctl) + 15) & ~15u);
+
 __device__ __forceinline__ void bar_group() { asm volatile("bar.sync %0, %1;" ::"n"(kBarGroup), "n"(kGThreads) : "memory"); }
-__device__ __forceinline__ void bar_epi() { asm volatile("bar.sync %0, 128;" ::"n"(kBarEpi) : "memory"); }
+__device__ __forceinline__ void bar_epi() { asm volatile("bar.sync %0, %1;" ::"n"(kBarEpi), "n"(kEpiThreads) : "memory"); }
+
+// Bits a..31 of a word (all for a <= 0, none for a >= 32).
+__device__ __forceinline__ uint32_t bits_from(int a) { return a <= 0 ? 0xFFFFFFFFu : (a >= 32 ? 0u : 0xFFFFFFFFu << a); }
 
 template <int kBar, int kCount>
 __device__ __forceinline__ bool bar_any(bool flag) {
@@ -173,15 +184,26 @@ __device__ __forceinline__ float pick(const uint32_t (&r)[32], int j) {
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
-    fused_kernel(const __grid_constant__ CUtensorMap zmap, gpo_batch b, gpo_outputs o, Sizes sz, Ws ws, Params p) {
+    fused_kernel(const __grid_constant__ CUtensorMap zmap, const __grid_constant__ CUtensorMap zmap32, gpo_batch b,
+                 gpo_outputs o, Sizes sz, Ws ws, Params p) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
-  unsigned char* tiles =
-      reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  Ctl* ctl = reinterpret_cast<Ctl*>(tiles + kStages * kStageBytes);
-  GroupSmem* gs = reinterpret_cast<GroupSmem*>(reinterpret_cast<unsigned char*>(ctl) + 256);
+  // group state, barriers, then the tiles on a 1024-byte boundary (128B swizzle).  Every
+  // pointer is smem_raw plus an offset, so the compiler keeps the shared address space
+  // (plain shared loads, stores and atomics rather than generic ones).
+  GroupSmem* gs = reinterpret_cast<GroupSmem*>(smem_raw);
+  Ctl* ctl = reinterpret_cast<Ctl*>(smem_raw + kCtlOff);
+  const uint32_t sbase = smem_u32(smem_raw);
+  unsigned char* tiles = smem_raw + (((sbase + kTilesOff + 1023u) & ~1023u) - sbase);
   uint32_t* st = ws.status;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int KT = (sz.d + kTileK - 1) / kTileK;
+  // pipeline geometry of this launch: one slot holds a k-slice of r32(max states) rows.  The
+  // MMA of the last 128-row block reads its A operand up to the next multiple of 128 rows
+  // (rows past the group only feed accumulator lanes that are never read), so the ring
+  // keeps that much room behind the last slot.
+  const int maxr = min(max(sz.maxn, 1), kMaxN);
+  const int slot_bytes = r32(maxr) * 128;
+  const int nslots = min(kMaxSlots, (kRingBytes - (((maxr + kTileM - 1) & ~(kTileM - 1)) - r32(maxr)) * 128) / slot_bytes);
   const float kappa = (float)p.kappa;
 
   if (blockIdx.x == 0 && threadIdx.x == 0) {
@@ -190,15 +212,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (b.rollout_token_off[0] != 0 || b.rollout_token_off[sz.R] != sz.T) report(st, GPO_ERR_SHAPE, 2, 2);
   }
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < kMaxSlots; ++s) {
       mbar_init(&ctl->full[s], 1);
       mbar_init(&ctl->empty[s], 1);
     }
     mbar_init(&ctl->tfull, 1);
-    mbar_init(&ctl->tempty, 4);
+    mbar_init(&ctl->tempty, kEpiThreads / 32);
     mbar_init(&ctl->drain, 1);
     fence_mbar_init();
     tma_prefetch_desc(&zmap);
+    tma_prefetch_desc(&zmap32);
   }
   if (warp == 1) {
     tmem_alloc(&ctl->tmem_base, kTmemCols);
@@ -209,40 +232,49 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = ctl->tmem_base;
 
-  if (warp == 0 && lane == 0) {
-    // ---------------------------------------------------------------- TMA producer
+  if (warp == 0) {
+    // ---------------------------------------------------------------- TMA producer (lane 0)
+    if (lane == 0) {
     int stage = 0;
     uint32_t phase = 0;
-    int last_parity[kStages];
-    for (int s = 0; s < kStages; ++s) last_parity[s] = -1;
+    int last_parity[kMaxSlots];
+    for (int s = 0; s < kMaxSlots; ++s) last_parity[s] = -1;
     bool ok = true;
     for (int g = blockIdx.x; g < sz.G && ok; g += gridDim.x) {
       int r0, nr, s0, n;
       if (!group_active(b, sz, g, r0, nr, s0, n)) continue;
       Plan pl;
       make_plan(n, pl);
-      const int nbox = (n + kTileM - 1) / kTileM;
-      for (int pass = 0; pass < pl.npass && ok; ++pass)
+      const int rows = r32(n);  // rows [0, r32(n)) of the group; the MMAs read no further
+      for (int pass = 0; pass < pl.npass && ok; ++pass) {
+        const int row0 = pl.npass == 2 && pass == 0 ? kTileM : 0;  // pass 0 of two never reads block 0
         for (int k = 0; k < KT; ++k) {
           if (!mbar_wait(&ctl->empty[stage], phase ^ 1u, st, 20)) {
             ok = false;
             break;
           }
-          unsigned char* t = tiles + stage * kStageBytes;
-          mbar_arrive_expect_tx(&ctl->full[stage], (uint32_t)(nbox * kBoxBytes));
+          unsigned char* t = tiles + stage * slot_bytes;
+          mbar_arrive_expect_tx(&ctl->full[stage], (uint32_t)((rows - row0) * 128));
           last_parity[stage] = (int)phase;
-          for (int bx = 0; bx < nbox; ++bx)
-            tma_load_2d(t + bx * kBoxBytes, &zmap, &ctl->full[stage], k * kTileK, s0 + bx * kTileM);
-          if (++stage == kStages) {
+          for (int r = row0; r < rows;) {  // 128-row boxes, then 32-row boxes for the tail
+            const bool big = rows - r >= kTileM;
+            tma_load_2d(t + r * 128, big ? &zmap : &zmap32, &ctl->full[stage], k * kTileK, s0 + r);
+            r += big ? kTileM : kTailRows;
+          }
+          if (++stage == nslots) {
             stage = 0;
             phase ^= 1u;
           }
         }
+      }
     }
-    for (int s = 0; s < kStages; ++s)
+    for (int s = 0; s < kMaxSlots; ++s)
       if (last_parity[s] >= 0) mbar_wait(&ctl->full[s], (uint32_t)last_parity[s], st, 21, 200000000ull, false);
-  } else if (warp == 1 && lane == 0) {
-    // ---------------------------------------------------------------- MMA issuer
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer (lane 0)
+    if (lane == 0) {
     int stage = 0;
     uint32_t phase = 0;
     int u = 0;  // accumulator uses (passes) so far
@@ -264,7 +296,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           }
           tc_fence_after();
-          const uint32_t t = smem_u32(tiles + stage * kStageBytes);
+          const uint32_t t = smem_u32(tiles + stage * slot_bytes);
           for (int si = 0; si < pl.nseg[pass]; ++si) {
             const Seg s = pl.seg[pass][si];
             const uint64_t ad = smem_desc_k128(t + (uint32_t)(s.b * kBoxBytes));
@@ -275,7 +307,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               mma_bf16_ss(tmem + (uint32_t)s.tcol, ad + 2u * kk, bd + 2u * kk, idesc, (k | kk) != 0);
           }
           mma_commit(&ctl->empty[stage]);
-          if (++stage == kStages) {
+          if (++stage == nslots) {
             stage = 0;
             phase ^= 1u;
           }
@@ -285,17 +317,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     mma_commit(&ctl->drain);
     mbar_wait(&ctl->drain, 0, st, 24, 200000000ull, false);
+    }
+    __syncwarp();
   } else if (warp >= 2) {
     // ---------------------------------------------------------------- group warps
-    const int gt = threadIdx.x - 64;  // 0..191
+    const int gt = threadIdx.x - 64;  // 0..447
     const bool epi = warp >= 4;
     const int q = warp & 3;           // TMEM lane quarter of an epilogue warp
-    const int wg = warp - 2;          // 0..5
+    const int wg = warp - 2;          // 0..13
     int u = 0;
     for (int g = blockIdx.x; g < sz.G; g += gridDim.x) {
       int r0 = 0, nr = 0, s0 = 0, n = 0;
       const bool in_range = group_range(b, sz, g, r0, nr, s0, n);
-      if (!(in_range && n > 0 && n <= kMaxN && nr > 0 && nr <= n)) {
+      if (!(in_range && n > 0 && n <= kMaxN && n <= sz.maxn && nr > 0 && nr <= n)) {
         if (gt == 0) {
           if (!in_range || nr > n || (nr > 0 && n == 0)) report(st, GPO_ERR_SHAPE, 2, g);
           else if (n > kMaxN || n > sz.maxn) report(st, GPO_ERR_UNSUPPORTED, 2, g);
@@ -304,7 +338,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (gt == 0) {
         make_plan(n, gs->plan);
-        gs->flags = (n > sz.maxn) ? 1 : 0;
+        gs->flags = 0;
       }
 
       // ---- validate the group and lay out its states (Sec. 4.2 chain layout)
@@ -313,6 +347,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         gs->tok0[r] = b.rollout_token_off[r0 + r];
       }
       for (int r = gt; r < nr; r += kGThreads) gs->rew[r] = b.reward[r0 + r];
+      group_scratch_zero(group_scratch_sep(gs->X, n), n, gt, kGThreads);  // read after the drain
       for (int i = gt; i < n; i += kGThreads) {
         gs->lab[i] = i;
         gs->slen[i] = b.step_len[s0 + i];
@@ -329,7 +364,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int i = a; i < e; ++i) {
             gs->roll[i] = r;
             gs->dep[i] = i - a + 1;
-            gs->ckey[i] = (r << 12) | (p.rule == GPO_MERGE_SAME_DEPTH ? (i - a + 1) & 0xFFF : 0);
             gs->tstart[i] = t;
             if (gs->slen[i] < 1) bad = true;
             t += gs->slen[i];
@@ -344,7 +378,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       bar_group();
       const bool valid = (gs->flags & 1) == 0;
 
-      // ---- drain the accumulator pass by pass (warps 4..7); warps 2..3 fetch
+      // ---- drain the accumulator pass by pass (warps 4..15); warps 2..3 fetch
       //      the prompt-embedding dots when a root embedding is given
       bool fail = false;
       if (!epi) {
@@ -370,21 +404,25 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       } else {
         const Plan& pl = gs->plan;
-        const int t128 = threadIdx.x - 128;
+        const int te = threadIdx.x - 128;     // 0..383
+        const int t128 = q * 32 + lane;       // accumulator lane = row within a 128-row block
+        const int rep = (warp - 4) >> 2;      // 0..2: which of the quarter's three warps
         for (int pass = 0; pass < pl.npass; ++pass, ++u) {
           const bool got = mbar_wait(&ctl->tfull, (uint32_t)u & 1u, st, 25);
-          if (bar_any<kBarEpi, 128>(!got)) {
+          if (bar_any<kBarEpi, kEpiThreads>(!got)) {
             fail = true;
             break;
           }
           tc_fence_after();
           const int nseg = pl.nseg[pass];
-          // norms and super-diagonal dots from the diagonal segments of this pass
+          // norms and super-diagonal dots from the diagonal segments of this pass (row
+          // block b is read by the quarter's warp b % 3)
+          if (te == 0) gs->ecount = 0;
 #pragma unroll 1
           for (int si = 0; si < nseg; ++si) {
             const Seg sg = pl.seg[pass][si];
-            if (sg.c0 != sg.b * kTileM || q * 32 >= sg.len) continue;  // no row of this warp here
-            const int i = sg.b * kTileM + q * 32 + lane;
+            if (sg.c0 != sg.b * kTileM || sg.b % 3 != rep || q * 32 >= sg.len) continue;
+            const int i = sg.b * kTileM + t128;
             const uint32_t base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)sg.tcol;
             uint32_t r[32];
             tmem_ld_32x32b_x32(base + (uint32_t)(q * 32), r);
@@ -406,67 +444,87 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll 1
           for (int si = 0; si < nseg; ++si) {
             const Seg sg = pl.seg[pass][si];
-            if (sg.c0 != sg.b * kTileM) continue;
+            if (sg.c0 != sg.b * kTileM || sg.b % 3 != rep) continue;
             const int i = sg.b * kTileM + t128;
-            if (i < n) gs->rn[i] = gs->n2[i] > 0.f ? 1.0f / sqrtf(gs->n2[i]) : 0.f;
+            if (i < n) {
+              const float rni = gs->n2[i] > 0.f ? 1.0f / sqrtf(gs->n2[i]) : 0.f;
+              gs->rn[i] = rni;
+              gs->col[i] = make_int2(gs->dep[i], __float_as_int(rni));
+            }
           }
           bar_epi();
-          // pass masks: comparable pairs (different rollout [, same depth]) with sim >= kappa
+          // linked pairs: comparable (different rollout [, same depth]) with sim >= kappa,
+          // tested as acc / |z_j| >= kappa |z_i| (one multiply per pair).  Columns of the row's
+          // own rollout, columns j <= i and columns past the group leave through one bit mask
+          // per 32-column chunk.  Each pair found goes to the edge list (or, past its capacity,
+          // straight into the forest).
 #pragma unroll 1
           for (int si = 0; si < nseg; ++si) {
             const Seg sg = pl.seg[pass][si];
-            const int i = sg.b * kTileM + q * 32 + lane;
+            const int rowbase = sg.b * kTileM + q * 32;
+            const int i = rowbase + lane;
             const bool vrow = valid && i < n;
-            const int ki = vrow ? gs->ckey[i] : -1;
-            const float rni = vrow ? gs->rn[i] : 0.f;
+            const float thr = vrow && gs->n2[i] > 0.f ? kappa * sqrtf(gs->n2[i]) : __int_as_float(0x7f800000);
+            const int ri = vrow ? gs->roll[i] : 0;
+            const int ra = vrow ? gs->rstart[ri] : 0, re = vrow ? gs->rstart[ri + 1] : 0;
+            const int di = vrow ? gs->dep[i] : -1;
             const int nch = (sg.len + 31) >> 5;
 #pragma unroll 1
-            for (int ch = 0; ch < nch; ++ch) {
-              uint32_t mk = 0u;
-              if (sg.c0 + ch * 32 + 31 > sg.b * kTileM + q * 32) {  // some col > row in this warp
-                uint32_t r[32];
-                tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(sg.tcol + ch * 32), r);
-                tmem_wait_ld();
-                const int cbase = sg.c0 + ch * 32;
-                const int cend = min(32, sg.len - ch * 32);
+            for (int ch = rep; ch < nch; ch += 3) {
+              const int cbase = sg.c0 + ch * 32;
+              if (cbase + 31 <= rowbase) continue;  // no column right of any row of this warp
+              uint32_t r[32];
+              tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(sg.tcol + ch * 32), r);
+              tmem_wait_ld();
+              uint32_t hit = 0u;
+              if (p.rule == GPO_MERGE_SAME_DEPTH) {
 #pragma unroll
                 for (int j = 0; j < 32; ++j) {
-                  const int c = min(cbase + j, n - 1);
-                  // comparable: different rollout, and equal depth bits (always equal under the
-                  // non-causal rule, whose keys carry no depth)
-                  const int x = gs->ckey[c] ^ ki;
-                  const bool okp = (j < cend) & (cbase + j > i) & ((x >> 12) != 0) & ((x & 0xFFF) == 0) &
-                                   (__uint_as_float(r[j]) * rni * gs->rn[c] >= kappa);
-                  mk |= (uint32_t)okp << j;
+                  const int2 cj = gs->col[cbase + j];
+                  hit |= (uint32_t)((cj.x == di) & (__uint_as_float(r[j]) * __int_as_float(cj.y) >= thr)) << j;
                 }
-                if (!vrow) mk = 0u;
+              } else {
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                  hit |= (uint32_t)(__uint_as_float(r[j]) * gs->rn[cbase + j] >= thr) << j;
               }
-              gs->masks[si * 8 + ch][t128] = mk;
+              const uint32_t own = bits_from(ra - cbase) & ~bits_from(re - cbase);
+              uint32_t mk = vrow ? hit & bits_from(i - cbase + 1) & ~bits_from(n - cbase) & ~own : 0u;
+              if (mk) {
+                int slot = atomicAdd(&gs->ecount, __popc(mk));
+                do {
+                  const int j = cbase + __ffs(mk) - 1;
+                  mk &= mk - 1u;
+                  if (slot < kEdgeList) gs->elist[slot] = (uint32_t)i | ((uint32_t)j << 16);
+                  else uf_union(gs->lab, i, j);
+                  ++slot;
+                } while (mk);
+              }
             }
           }
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&ctl->tempty);  // accumulator free for the next pass
+          // classes = connected components of the linked pairs (Alg. S.1): every thread
+          // unites one listed pair at a time into the shared forest (lock-free; the larger
+          // root is hooked under the smaller, so a class's root is its smallest member).
+          // Lanes stay converged, one union per lane per step.
+          bar_epi();
+          const int ne = min(gs->ecount, kEdgeList);
 #pragma unroll 1
-          for (int si = 0; si < nseg; ++si) {
-            const Seg sg = pl.seg[pass][si];
-            const int i = sg.b * kTileM + q * 32 + lane;
-            const int nch = (sg.len + 31) >> 5;
-#pragma unroll 1
-            for (int ch = 0; ch < nch; ++ch) {
-              uint32_t mk = gs->masks[si * 8 + ch][t128];
-              while (mk) {
-                const int j = __ffs(mk) - 1;
-                mk &= mk - 1u;
-                uf_union(gs->lab, i, sg.c0 + ch * 32 + j);
-              }
+          for (int e0 = 0; e0 < ne; e0 += kEpiThreads) {
+            const int e = e0 + te;
+            if (e < ne) {
+              const uint32_t ij = gs->elist[e];
+              uf_union(gs->lab, (int)(ij & 0xFFFFu), (int)(ij >> 16));
             }
+            __syncwarp();
           }
         }
       }
       if (bar_any<kBarGroup, kGThreads>(fail)) break;
 
-      // ---- graph reward and dual-group advantage of every edge (fp64)
+      // ---- graph reward and dual-group advantage of every edge
       if (valid) {
         auto eta = [&](int i) -> float {
           float e = 0.f, n1 = 0.f, dot = 0.f;
@@ -493,15 +551,48 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (o.class_id) o.class_id[v] = s0 + label;
           if (o.node_score) o.node_score[v] = S;
         };
-        group_advantages<2>(n, nr, gs->lab, gs->roll, gs->dep, gs->rstart, gs->rew, gs->X, p, gt, kGThreads,
-                            [] { bar_group(); }, eta, out);
-        // ---- every token of an edge carries the edge's advantage (Sec. 4.5)
-        for (int i = wg; i < n; i += kGThreads / 32) {
+        group_advantages<1, true>(n, nr, gs->lab, gs->roll, gs->dep, gs->rstart, gs->rew, group_scratch_sep(gs->X, n),
+                                  p, gt, kGThreads, [] { bar_group(); }, eta, out);
+        // ---- every token of an edge carries the edge's advantage (Sec. 4.5).  State-major:
+        //      each half-warp takes a state, its 16 lanes write the whole 16-byte chunks of the
+        //      state's token span, then the at most 3 + 3 tokens of its partial first and last
+        //      chunk (which neighbour other states' tokens) with scalar stores.
+        const bool more = o.adv_cor || o.adv_eff || o.eff_mask;
+        const int hl = gt & 15;
+#pragma unroll 1
+        for (int i = gt >> 4; i < n; i += kGThreads / 16) {
           const int64_t ts = gs->tstart[i], te = ts + gs->slen[i];
-          write_span(o.adv, ts, te, gs->eadv[i], lane);
-          if (o.adv_cor) write_span(o.adv_cor, ts, te, gs->ecor[i], lane);
-          if (o.adv_eff) write_span(o.adv_eff, ts, te, gs->eeff[i], lane);
-          if (o.eff_mask) write_span_u8(o.eff_mask, ts, te, gs->emask[i], lane);
+          const float x = gs->eadv[i];
+          const int64_t qa = (ts + 3) >> 2, qb = te >> 2;
+          const int64_t h1 = qa <= qb ? 4 * qa : te;  // head [ts, h1)
+          const int64_t t0 = qa <= qb ? 4 * qb : te;  // tail [t0, te)
+          const int64_t tp = hl < 4 ? ts + hl : t0 + (hl - 4);
+          const bool scal = hl < 4 ? tp < h1 : (hl < 8 && tp < te);
+          {
+            const float4 v = make_float4(x, x, x, x);
+            for (int64_t c = qa + hl; c < qb; c += 16) reinterpret_cast<float4*>(o.adv)[c] = v;
+            if (scal) o.adv[tp] = x;
+          }
+          if (more) {
+            if (o.adv_cor) {
+              const float y = gs->ecor[i];
+              const float4 v = make_float4(y, y, y, y);
+              for (int64_t c = qa + hl; c < qb; c += 16) reinterpret_cast<float4*>(o.adv_cor)[c] = v;
+              if (scal) o.adv_cor[tp] = y;
+            }
+            if (o.adv_eff) {
+              const float y = gs->eeff[i];
+              const float4 v = make_float4(y, y, y, y);
+              for (int64_t c = qa + hl; c < qb; c += 16) reinterpret_cast<float4*>(o.adv_eff)[c] = v;
+              if (scal) o.adv_eff[tp] = y;
+            }
+            if (o.eff_mask) {
+              const uint8_t m = gs->emask[i];
+              const uint32_t v = 0x01010101u * m;
+              for (int64_t c = qa + hl; c < qb; c += 16) reinterpret_cast<uint32_t*>(o.eff_mask)[c] = v;
+              if (scal) o.eff_mask[tp] = m;
+            }
+          }
         }
       }
       bar_group();
@@ -514,7 +605,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 1) tmem_dealloc(tmem, kTmemCols);
 }
 
-size_t fused_smem() { return (size_t)kStages * kStageBytes + 256 + sizeof(GroupSmem) + 1024; }
+size_t fused_smem() { return (size_t)kTilesOff + 1023 + (size_t)kRingBytes; }
 
 }  // namespace
 
@@ -522,11 +613,11 @@ cudaError_t setup_fused() {
   return cudaFuncSetAttribute(fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)fused_smem());
 }
 
-cudaError_t launch_fused(const LaunchCtx& lc, const CUtensorMap& map, const gpo_batch& b, const gpo_outputs& o,
-                         const Sizes& sz, const Ws& ws, const Params& p) {
+cudaError_t launch_fused(const LaunchCtx& lc, const CUtensorMap& map, const CUtensorMap& map32, const gpo_batch& b,
+                         const gpo_outputs& o, const Sizes& sz, const Ws& ws, const Params& p) {
   if (sz.G == 0) return cudaSuccess;
   const int grid = sz.G < lc.num_sms ? sz.G : lc.num_sms;
-  fused_kernel<<<grid, kThreads, fused_smem(), lc.stream>>>(map, b, o, sz, ws, p);
+  fused_kernel<<<grid, kThreads, fused_smem(), lc.stream>>>(map, map32, b, o, sz, ws, p);
   return cudaGetLastError();
 }
 

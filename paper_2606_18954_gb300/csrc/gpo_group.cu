@@ -83,7 +83,9 @@ __global__ void __launch_bounds__(1024) groups_kernel(gpo_batch b, gpo_outputs o
     if (o.class_id) o.class_id[v] = s0 + label;
     if (o.node_score) o.node_score[v] = S;
   };
-  group_advantages<kPer>(n, nr, lab, roll, dep, rstart, rew, X, p, tid, nt, [] { __syncthreads(); }, eta, out);
+  __shared__ int s_rootc;
+  group_advantages<kPer, false>(n, nr, lab, roll, dep, rstart, rew, group_scratch_shared(X, n, &s_rootc), p, tid, nt,
+                                [] { __syncthreads(); }, eta, out);
 
   // first token of every edge
   for (int rr = tid; rr < nr; rr += nt) {

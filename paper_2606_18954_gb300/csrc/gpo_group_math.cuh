@@ -14,9 +14,6 @@
 //             l_v = depth (a_Q is the root), routed onto every edge of
 //             root -> v, summed over routes                           (Sec. 4.4)
 //   A_dual    A_cor + lambda_eff * routed A_eff                        (Sec. 4.5)
-// in fp64.  Group sums go through exact two-word fixed-point accumulators
-// (resolution 2^-76) in shared-memory int64 atomics, so the results do not
-// depend on the order in which threads add.
 #pragma once
 
 #include "gpo_internal.cuh"
@@ -69,11 +66,84 @@ __device__ __forceinline__ long long div_round(long long a, int k) {
 
 __host__ __device__ constexpr size_t al16(size_t x) { return (x + 15) & ~size_t(15); }
 
-// Scratch bytes group_advantages needs for a group of n states: the largest of
-// its three phases (class sums 24 B/class, correctness-group sums 28 B/group,
-// route sums 9 B/state).
+// Scratch arrays of group_advantages.  Class sums are indexed by the class root
+// (a local state index), correctness-group sums by the key (the class of the
+// parent, or n for the prompt root); the route sums reuse the class arrays.
+struct GroupScratch {
+  int* ccnt;            // [n]   |Q|
+  int* csum;            // [n]   C_Q = sum of the members' rewards
+  int* lsum;            // [n]   sum of the members' depths
+  long long* l2;        // [n]   sum of the squared depths
+  int* kcnt;            // [n+1] edges per correctness group
+  long long* ksum;      // [n+1] sum of r on the 2^-50 grid
+  long long* kq_hi;     // [n+1] sum of (r - mean)^2, 2^-36 grid part
+  long long* kq_lo;     // [n+1] and 2^-76 grid remainder
+  float* aeff;          // [n]   A_eff of each route end (over ccnt / csum)
+  float* E;             // [n]   routed A_eff (over lsum)
+  unsigned char* cov;   // [n]   covered by a route (over l2)
+  int* rootc;           // [1]   sum of the group's rewards
+};
+
+// Separate layout: class and key arrays side by side, for callers that zero
+// them ahead of time (group_scratch_zero); bytes for a group of up to n states.
+__host__ __device__ constexpr size_t group_scratch_sep_bytes(int n) {
+  return al16(12 * (size_t)n) + al16(8 * (size_t)n) + al16(4 * (size_t)(n + 1)) + 3 * al16(8 * (size_t)(n + 1)) + 16;
+}
+
+__device__ __forceinline__ GroupScratch group_scratch_sep(unsigned char* X, int n) {
+  GroupScratch g;
+  g.ccnt = reinterpret_cast<int*>(X);
+  g.csum = g.ccnt + n;
+  g.lsum = g.csum + n;
+  g.l2 = reinterpret_cast<long long*>(X + al16(12 * (size_t)n));
+  unsigned char* k = X + al16(12 * (size_t)n) + al16(8 * (size_t)n);
+  g.kcnt = reinterpret_cast<int*>(k);
+  g.ksum = reinterpret_cast<long long*>(k + al16(4 * (size_t)(n + 1)));
+  g.kq_hi = g.ksum + (n + 1);
+  g.kq_lo = g.kq_hi + (n + 1);
+  g.rootc = reinterpret_cast<int*>(k + al16(4 * (size_t)(n + 1)) + 3 * al16(8 * (size_t)(n + 1)));
+  g.aeff = reinterpret_cast<float*>(g.ccnt);
+  g.E = reinterpret_cast<float*>(g.lsum);
+  g.cov = reinterpret_cast<unsigned char*>(g.l2);
+  return g;
+}
+
+// Zero the sums of a separate-layout scratch (before the barrier that precedes
+// group_advantages<kPer, true>).
+__device__ __forceinline__ void group_scratch_zero(const GroupScratch& g, int n, int tid, int nt) {
+  for (int i = tid; i < n; i += nt) {
+    g.ccnt[i] = g.csum[i] = g.lsum[i] = 0;
+    g.l2[i] = 0;
+  }
+  for (int i = tid; i <= n; i += nt) {
+    g.kcnt[i] = 0;
+    g.ksum[i] = g.kq_hi[i] = g.kq_lo[i] = 0;
+  }
+  if (tid == 0) *g.rootc = 0;
+}
+
+// Shared layout: the class, key and route arrays overlay one region (the
+// largest is the key sums, 28 B per key), for large groups; group_advantages
+// zeroes each in turn, at the cost of extra barriers.
 __host__ __device__ constexpr size_t group_scratch_bytes(int n) {
   return al16(28 * (size_t)(n + 1) + 32);
+}
+
+__device__ __forceinline__ GroupScratch group_scratch_shared(unsigned char* X, int n, int* rootc) {
+  GroupScratch g;
+  g.ccnt = reinterpret_cast<int*>(X);
+  g.csum = g.ccnt + n;
+  g.lsum = g.csum + n;
+  g.l2 = reinterpret_cast<long long*>(X + al16(12 * (size_t)n));
+  g.kcnt = reinterpret_cast<int*>(X);
+  g.ksum = reinterpret_cast<long long*>(X + al16(4 * (size_t)(n + 1)));
+  g.kq_hi = g.ksum + (n + 1);
+  g.kq_lo = g.kq_hi + (n + 1);
+  g.aeff = reinterpret_cast<float*>(X);
+  g.E = g.aeff + n;
+  g.cov = reinterpret_cast<unsigned char*>(g.E + n);
+  g.rootc = rootc;
+  return g;
 }
 
 // One group, `nt` cooperating threads (thread index tid), kPer * nt >= n.
@@ -83,72 +153,51 @@ __host__ __device__ constexpr size_t group_scratch_bytes(int n) {
 //   dep     [n] depth of each state (1 = first step)
 //   rstart  [nr+1] local state offsets of the rollouts
 //   rew     [nr] rewards
-//   X       shared scratch of group_scratch_bytes(n), 16-byte aligned
+//   sc      scratch: separate layout zeroed by the caller (kZeroed), or the
+//           shared layout (!kZeroed)
 //   eta(i)  eta(p(v), v) of local state i (fp32, already clamped at 0)
 //   out(i, label, S, acor, E, dual, mask) is called once per state by its owner
 //   sync()  barrier over the nt threads
 //
 // Precision: fp32 arithmetic with exact integer class sums and an exact
 // fixed-point group mean (the one quantity whose rounding the standardisation
-// amplifies).  Per-class and per-group constants are computed once by one
-// thread.  Sums go through integer atomics, so results do not depend on the
-// order in which threads add.
-template <int kPer, class Sync, class Eta, class Out>
+// amplifies).  Per-class and per-group constants are recomputed by every state
+// that needs them (same operands, same operations, so the same value), which
+// saves a barrier per constant.  Sums go through integer atomics, so results do
+// not depend on the order in which threads add.
+template <int kPer, bool kZeroed, class Sync, class Eta, class Out>
 __device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const int* roll, const int* dep,
-                                                 const int* rstart, const uint8_t* rew, unsigned char* X,
+                                                 const int* rstart, const uint8_t* rew, const GroupScratch& sc,
                                                  const Params& p, int tid, int nt, Sync sync, Eta eta, Out out) {
   const float w = (float)p.w, eps = (float)p.eps;
   // ---- phase A: class sums C_Q (rewards), |Q|, sum l, sum l^2
-  int* ccnt = reinterpret_cast<int*>(X);
-  int* csum = ccnt + n;
-  int* lsum = csum + n;
-  long long* l2 = reinterpret_cast<long long*>(X + al16(12 * (size_t)n));
-  float* cg = reinterpret_cast<float*>(l2 + n);    // efficiency factor of the class
-  __shared__ int s_rootc;
-
-  for (int i = tid; i < n; i += nt) {
-    ccnt[i] = csum[i] = lsum[i] = 0;
-    l2[i] = 0;
+  if (!kZeroed) {
+    for (int i = tid; i < n; i += nt) {
+      sc.ccnt[i] = sc.csum[i] = sc.lsum[i] = 0;
+      sc.l2[i] = 0;
+    }
+    if (tid == 0) *sc.rootc = 0;
+    sync();
   }
-  if (tid == 0) s_rootc = 0;
   int lb[kPer];
 #pragma unroll
   for (int k = 0; k < kPer; ++k) {
     const int i = tid + k * nt;
-    lb[k] = i < n ? uf_find(lab, i) : 0;
-  }
-  sync();
-#pragma unroll
-  for (int k = 0; k < kPer; ++k) {
-    const int i = tid + k * nt;
+    lb[k] = 0;
     if (i < n) {
+      // writing the root over the parent keeps every concurrent find on the same root
+      lb[k] = uf_find(lab, i);
       lab[i] = lb[k];
       const int d = dep[i];
-      atomicAdd(&ccnt[lb[k]], 1);
-      atomicAdd(&csum[lb[k]], (int)rew[roll[i]]);
-      atomicAdd(&lsum[lb[k]], d);
-      atomicAdd(reinterpret_cast<unsigned long long*>(&l2[lb[k]]), (unsigned long long)((long long)d * d));
+      atomicAdd(&sc.ccnt[lb[k]], 1);
+      atomicAdd(&sc.csum[lb[k]], (int)rew[roll[i]]);
+      atomicAdd(&sc.lsum[lb[k]], d);
+      atomicAdd(reinterpret_cast<unsigned long long*>(&sc.l2[lb[k]]), (unsigned long long)((long long)d * d));
     }
   }
-  for (int r = tid; r < nr; r += nt) atomicAdd(&s_rootc, (int)rew[r]);
+  for (int r = tid; r < nr; r += nt) atomicAdd(sc.rootc, (int)rew[r]);
   sync();
-  for (int L = tid; L < n; L += nt) {  // class constants, once per class
-    const int Q = ccnt[L];
-    if (Q == 0) continue;
-    float g = 0.f;
-    if (Q >= 2) {
-      // Sbar_Q = mean of S over Q = C_Q / |Q| (every member has t_own = 1);
-      // sum (l - mean)^2 = (Q sum l^2 - (sum l)^2) / Q with an exact integer numerator;
-      // A_eff(v) = Sbar (mean l - l_v) / (sd + eps) = g (sum l - Q l_v)
-      const long long ls = lsum[L];
-      const float ss = (float)((long long)Q * l2[L] - ls * ls) / (float)Q;
-      const float sd = sqrtf(ss / (float)(Q - p.ddof));
-      g = ((float)csum[L] / (float)Q) / ((sd + eps) * (float)Q);
-    }
-    cg[L] = g;
-  }
-  sync();
-  const float S_root = (float)s_rootc / (float)nr;
+  const float S_root = (float)*sc.rootc / (float)nr;
   float S[kPer], aeff[kPer], r[kPer];
   int key[kPer];
   bool route_end[kPer];
@@ -159,38 +208,42 @@ __device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const 
     key[k] = n;
     route_end[k] = false;
     if (i >= n) continue;
-    const int L = lb[k], Q = ccnt[L], d = dep[i], c = rew[roll[i]];
+    const int L = lb[k], Q = sc.ccnt[L], d = dep[i], c = rew[roll[i]];
     // Eq. (combain): (c_own + w sum_{q != v} c_own(q)) / (t_own + w sum_{q != v} t_own(q)), t_own = 1.
     // Correctly rounded, with numerator and denominator formed by the same fma, so that a
     // class whose members share one reward gets S exactly 0 or 1 (as the exact formula).
-    S[k] = fmaf(w, (float)(csum[L] - c), (float)c) / fmaf(w, (float)(Q - 1), 1.0f);
+    S[k] = fmaf(w, (float)(sc.csum[L] - c), (float)c) / fmaf(w, (float)(Q - 1), 1.0f);
     if (Q >= 2) {
+      // Sbar_Q = mean of S over Q = C_Q / |Q| (every member has t_own = 1);
+      // sum (l - mean)^2 = (Q sum l^2 - (sum l)^2) / Q with an exact integer numerator;
+      // A_eff(v) = Sbar (mean l - l_v) / (sd + eps) = g (sum l - Q l_v)
+      const long long ls = sc.lsum[L];
+      const float ss = (float)((long long)Q * sc.l2[L] - ls * ls) / (float)Q;
+      const float sd = sqrtf(ss / (float)(Q - p.ddof));
+      const float g = ((float)sc.csum[L] / (float)Q) / ((sd + eps) * (float)Q);
       route_end[k] = true;
-      aeff[k] = cg[L] * (float)(lsum[L] - Q * d);
+      aeff[k] = g * (float)(sc.lsum[L] - Q * d);
     }
     float Sp;
     if (d == 1) {
       Sp = S_root;
     } else {
       const int Lp = lab[i - 1];  // parent: the previous state of the same rollout (same reward c)
-      Sp = fmaf(w, (float)(csum[Lp] - c), (float)c) / fmaf(w, (float)(ccnt[Lp] - 1), 1.0f);
+      Sp = fmaf(w, (float)(sc.csum[Lp] - c), (float)c) / fmaf(w, (float)(sc.ccnt[Lp] - 1), 1.0f);
       key[k] = Lp;
     }
     r[k] = (S[k] - Sp) * (1.0f - eta(i));
   }
-  sync();  // phase A scratch no longer read
 
   // ---- phase B: correctness groups, key = class of p(v), n = the prompt root
-  int* kcnt = reinterpret_cast<int*>(X);
-  long long* ksum = reinterpret_cast<long long*>(X + al16(4 * (size_t)(n + 1)));  // becomes the mean
-  long long* kq_hi = ksum + (n + 1);
-  long long* kq_lo = kq_hi + (n + 1);
-  float* kinv = reinterpret_cast<float*>(kq_hi);  // 1 / (sd + eps), written over kq_hi after use
-  for (int i = tid; i <= n; i += nt) {
-    kcnt[i] = 0;
-    ksum[i] = kq_hi[i] = kq_lo[i] = 0;
+  if (!kZeroed) {
+    sync();  // class sums no longer read
+    for (int i = tid; i <= n; i += nt) {
+      sc.kcnt[i] = 0;
+      sc.ksum[i] = sc.kq_hi[i] = sc.kq_lo[i] = 0;
+    }
+    sync();
   }
-  sync();
   long long rf[kPer];
 #pragma unroll
   for (int k = 0; k < kPer; ++k) {
@@ -198,49 +251,41 @@ __device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const 
     if (tid + k * nt < n) {
       // |r| <= 1 and a group holds at most 4096 edges: a 2^50 fixed point cannot overflow
       rf[k] = __float2ll_rn(r[k] * 0x1p50f);
-      atomicAdd(&kcnt[key[k]], 1);
-      atomicAdd(reinterpret_cast<unsigned long long*>(&ksum[key[k]]), (unsigned long long)rf[k]);
+      atomicAdd(&sc.kcnt[key[k]], 1);
+      atomicAdd(reinterpret_cast<unsigned long long*>(&sc.ksum[key[k]]), (unsigned long long)rf[k]);
     }
   }
-  sync();
-  for (int K = tid; K <= n; K += nt)
-    if (kcnt[K] > 0) ksum[K] = div_round(ksum[K], kcnt[K]);  // exact mean on the 2^-50 grid
   sync();
   float dv[kPer];
 #pragma unroll
   for (int k = 0; k < kPer; ++k) {
     dv[k] = 0.f;
     if (tid + k * nt < n) {
-      dv[k] = (float)(rf[k] - ksum[key[k]]) * 0x1p-50f;
-      fx_add32(&kq_hi[key[k]], &kq_lo[key[k]], dv[k] * dv[k]);
+      const long long mean = div_round(sc.ksum[key[k]], sc.kcnt[key[k]]);  // exact mean on the 2^-50 grid
+      dv[k] = (float)(rf[k] - mean) * 0x1p-50f;
+      fx_add32(&sc.kq_hi[key[k]], &sc.kq_lo[key[k]], dv[k] * dv[k]);
     }
-  }
-  sync();
-  for (int K = tid; K <= n; K += nt) {
-    const int cnt = kcnt[K];
-    float inv = 0.f;  // groups of one edge get no advantage
-    if (cnt >= 2) {
-      const float ss = (float)kq_hi[K] * 0x1p-36f + (float)kq_lo[K] * 0x1p-76f;  // sum (r - mean)^2
-      inv = 1.0f / (sqrtf(ss / (float)(cnt - p.ddof)) + eps);
-    }
-    kinv[2 * K] = inv;  // kq_hi[K]'s first word; only this thread touches kq_*[K]
   }
   sync();
   float acor[kPer];
 #pragma unroll
-  for (int k = 0; k < kPer; ++k) acor[k] = (tid + k * nt < n) ? dv[k] * kinv[2 * key[k]] : 0.f;
-  sync();  // phase B scratch no longer read
+  for (int k = 0; k < kPer; ++k) {
+    acor[k] = 0.f;
+    const int K = key[k], cnt = sc.kcnt[K];
+    if (tid + k * nt < n && cnt >= 2) {  // groups of one edge get no advantage
+      const float ss = (float)sc.kq_hi[K] * 0x1p-36f + (float)sc.kq_lo[K] * 0x1p-76f;  // sum (r - mean)^2
+      acor[k] = dv[k] * (1.0f / (sqrtf(ss / (float)(cnt - p.ddof)) + eps));
+    }
+  }
 
   // ---- phase C: every edge on root -> v receives A_eff(v) (suffix sums per rollout)
-  float* s_aeff = reinterpret_cast<float*>(X);
-  float* s_E = s_aeff + n;
-  unsigned char* s_cov = reinterpret_cast<unsigned char*>(s_E + n);
+  if (!kZeroed) sync();  // key sums no longer read (the route arrays overlay them)
 #pragma unroll
   for (int k = 0; k < kPer; ++k) {
     const int i = tid + k * nt;
     if (i < n) {
-      s_aeff[i] = aeff[k];
-      s_cov[i] = route_end[k] ? 1 : 0;
+      sc.aeff[i] = aeff[k];
+      sc.cov[i] = route_end[k] ? 1 : 0;
     }
   }
   sync();
@@ -248,10 +293,10 @@ __device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const 
     float acc = 0.f;
     unsigned char cov = 0;
     for (int i = rstart[rr + 1] - 1; i >= rstart[rr]; --i) {
-      acc += s_aeff[i];
-      cov |= s_cov[i];
-      s_E[i] = acc;
-      s_cov[i] = cov;
+      acc += sc.aeff[i];
+      cov |= sc.cov[i];
+      sc.E[i] = acc;
+      sc.cov[i] = cov;
     }
   }
   sync();
@@ -259,7 +304,7 @@ __device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const 
 #pragma unroll
   for (int k = 0; k < kPer; ++k) {
     const int i = tid + k * nt;
-    if (i < n) out(i, lb[k], S[k], acor[k], s_E[i], fmaf(lam, s_E[i], acor[k]), s_cov[i]);
+    if (i < n) out(i, lb[k], S[k], acor[k], sc.E[i], fmaf(lam, sc.E[i], acor[k]), sc.cov[i]);
   }
   sync();
 }

@@ -293,8 +293,8 @@ cudaError_t launch_tokens(const LaunchCtx& lc, const gpo_batch& b, const gpo_out
 // Records a message on the context (gpo_last_error).
 void note_error(gpo_ctx* ctx, const char* msg);
 
-cudaError_t launch_fused(const LaunchCtx& lc, const CUtensorMap& map, const gpo_batch& b, const gpo_outputs& o,
-                         const Sizes& sz, const Ws& ws, const Params& p);
+cudaError_t launch_fused(const LaunchCtx& lc, const CUtensorMap& map, const CUtensorMap& map32, const gpo_batch& b,
+                         const gpo_outputs& o, const Sizes& sz, const Ws& ws, const Params& p);
 cudaError_t setup_fused();
 cudaError_t setup_sim_tc();
 cudaError_t setup_groups();

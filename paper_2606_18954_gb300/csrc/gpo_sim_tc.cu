@@ -88,10 +88,12 @@ __device__ __forceinline__ void lunion(int* p, int a, int b) {
 __global__ void __launch_bounds__(kThreads, 1)
     sim_tc_kernel(const __grid_constant__ CUtensorMap zmap, Sizes sz, Ws ws, float kappa, int rule) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
-  // 1024-byte alignment for the swizzled tiles
-  unsigned char* tiles =
-      reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  SmemCtl* ctl = reinterpret_cast<SmemCtl*>(tiles + kStages * kStageBytes);
+  // control block first, then the tiles on a 1024-byte boundary (128B swizzle); both are
+  // smem_raw plus an offset, so the compiler keeps the shared address space
+  SmemCtl* ctl = reinterpret_cast<SmemCtl*>(smem_raw);
+  const uint32_t sbase = smem_u32(smem_raw);
+  constexpr uint32_t kCtlBytes = (sizeof(SmemCtl) + 15) & ~15u;
+  unsigned char* tiles = smem_raw + (((sbase + kCtlBytes + 1023u) & ~1023u) - sbase);
   uint32_t* st = ws.status;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -122,8 +124,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = ctl->tmem_base;
 
-  if (warp == 0 && lane == 0) {
-    // ------------------------------------------------------------ TMA producer
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer (lane 0)
+    if (lane == 0) {
     int stage = 0;
     uint32_t phase = 0;
     int last_parity[kStages];
@@ -159,8 +162,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     // wind-down: every issued copy must land before the CTA may exit
     for (int s = 0; s < kStages; ++s)
       if (last_parity[s] >= 0) mbar_wait(&ctl->full[s], (uint32_t)last_parity[s], st, 11, 200000000ull, false);
-  } else if (warp == 1 && lane == 0) {
-    // ------------------------------------------------------------ MMA issuer
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer (lane 0)
+    if (lane == 0) {
     int stage = 0;
     uint32_t phase = 0;
     int m = 0;
@@ -197,6 +203,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     // wind-down: all issued MMAs complete before TMEM is released
     mma_commit(&ctl->drain);
     mbar_wait(&ctl->drain, 0, st, 14, 200000000ull, false);
+    }
+    __syncwarp();
   } else if (warp >= 4) {
     // ------------------------------------------------------------ epilogue
     const int q = warp & 3;
@@ -291,7 +299,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 }  // namespace
 
-size_t sim_tc_smem_bytes() { return (size_t)kStages * kStageBytes + sizeof(SmemCtl) + 1024; }
+size_t sim_tc_smem_bytes() { return ((sizeof(SmemCtl) + 15) & ~size_t(15)) + 1023 + (size_t)kStages * kStageBytes; }
 
 cudaError_t setup_sim_tc() {
   return cudaFuncSetAttribute(sim_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,

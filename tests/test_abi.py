@@ -73,6 +73,8 @@ def test_argument_checks_without_device(lib):
     assert lib.gpo_create(ctypes.byref(h), ctypes.byref(bad)) == 1
     bad = B.Params(0.92, 0.7, -1.0, 1e-6, 1, 0, 0)  # negative lambda
     assert lib.gpo_create(ctypes.byref(h), ctypes.byref(bad)) == 1
+    bad = B.Params(0.0, 0.7, 1.0, 1e-6, 1, 0, 0)    # kappa must be positive
+    assert lib.gpo_create(ctypes.byref(h), ctypes.byref(bad)) == 1
     assert lib.gpo_create(None, None) == 1
     assert lib.gpo_sync_status(None, None) == 1
     assert lib.gpo_compute(None, None, None, None, 0, None) == 1

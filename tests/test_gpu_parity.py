@@ -290,6 +290,22 @@ def test_error_group_too_large(gp_mod):
     _expect_status(gp_mod, b, 5, host=True)
 
 
+@ERR_PATHS
+def test_error_group_above_declared_max(gp_mod, flags):
+    """A group larger than the batch's declared max_states_per_group is refused on the device."""
+    import dataclasses
+    import torch
+    P = gp_mod
+    db = P.Batch.from_arrays(batch_of("math", 2), device="cuda")
+    db = dataclasses.replace(db, max_states_per_group=db.max_states_per_group - 40)
+    gp = P.GraphPO(flags=flags)
+    gp(db)
+    with pytest.raises(P.GraphPOError) as e:
+        gp.check()
+    assert e.value.code == 5, gp.last_error()
+    torch.cuda.synchronize()
+
+
 def test_error_workspace_too_small(gp_mod):
     import torch
     P = gp_mod
