@@ -37,7 +37,8 @@ constexpr int kTailRows = 32;                   // rows of the second tensor map
 constexpr int kTmemCols = 512;
 constexpr int kGThreads = 448;                  // warps 2..15
 constexpr int kEpiThreads = 384;                // warps 4..15: three per accumulator lane quarter
-constexpr int kEdgeList = 4096;                 // linked pairs listed per pass
+constexpr int kWarpEdges = 256;                 // linked pairs listed per epilogue warp and group
+constexpr int kEdgeList = kWarpEdges * (kEpiThreads / 32);
 constexpr int kBarGroup = 1;                    // named barrier of warps 2..15
 constexpr int kBarEpi = 2;                      // named barrier of warps 4..15
 
@@ -127,7 +128,9 @@ struct __align__(16) GroupSmem {
   int rstart[kMaxN + 1];
   float n2[kMaxN];
   float dn[kMaxN];       // <z_i, z_{i+1}>
-  float rn[kMaxN];
+  alignas(16) float rn[kMaxN];  // 1 / |z_i| (0 for a zero row), read four at a time
+  float thr[kMaxN];      // kappa |z_i| (+inf for a zero row or a row that is not tested)
+  int rend[kMaxN];       // end (local, exclusive) of the rollout of state i
   float root_dot[kMaxN]; // <root, z of the first state of rollout r>
   float eadv[kMaxN], ecor[kMaxN], eeff[kMaxN];
   int64_t tok0[kMaxN + 1];
@@ -135,11 +138,10 @@ struct __align__(16) GroupSmem {
   uint8_t rew[kMaxN];
   uint8_t emask[kMaxN];
   int flags;             // bit 0: group invalid
-  int ecount;            // linked pairs of the current pass (edge list in X)
+  int overflow;          // some warp found more pairs than its part of elist holds
   float root_n2;
   Plan plan;
-  int2 col[kMaxN];       // {depth, bits of 1/|z|} of every state, read per column by the pair loop
-  uint32_t elist[kEdgeList];  // linked pairs of the pass: i | j << 16
+  uint32_t elist[kEdgeList];  // linked pairs of the group, kWarpEdges per epilogue warp: i | j << 16
   alignas(16) unsigned char X[group_scratch_sep_bytes(kMaxN)];  // group-math sums (separate layout)
 };
 
@@ -339,6 +341,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (gt == 0) {
         make_plan(n, gs->plan);
         gs->flags = 0;
+        gs->overflow = 0;
       }
 
       // ---- validate the group and lay out its states (Sec. 4.2 chain layout)
@@ -347,7 +350,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         gs->tok0[r] = b.rollout_token_off[r0 + r];
       }
       for (int r = gt; r < nr; r += kGThreads) gs->rew[r] = b.reward[r0 + r];
-      group_scratch_zero(group_scratch_sep(gs->X, n), n, gt, kGThreads);  // read after the drain
+      group_scratch_zero(gs->X, n, gt, kGThreads);  // read after the drain
       for (int i = gt; i < n; i += kGThreads) {
         gs->lab[i] = i;
         gs->slen[i] = b.step_len[s0 + i];
@@ -364,6 +367,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int i = a; i < e; ++i) {
             gs->roll[i] = r;
             gs->dep[i] = i - a + 1;
+            gs->rend[i] = e;
             gs->tstart[i] = t;
             if (gs->slen[i] < 1) bad = true;
             t += gs->slen[i];
@@ -407,6 +411,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int te = threadIdx.x - 128;     // 0..383
         const int t128 = q * 32 + lane;       // accumulator lane = row within a 128-row block
         const int rep = (warp - 4) >> 2;      // 0..2: which of the quarter's three warps
+        const int ew = warp - 4;              // epilogue warp 0..11: owns elist[ew * kWarpEdges, ...)
+        uint32_t* wlist = gs->elist + ew * kWarpEdges;
+        int wcount = 0;                       // pairs this warp found in the group (warp-uniform)
         for (int pass = 0; pass < pl.npass; ++pass, ++u) {
           const bool got = mbar_wait(&ctl->tfull, (uint32_t)u & 1u, st, 25);
           if (bar_any<kBarEpi, kEpiThreads>(!got)) {
@@ -417,7 +424,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int nseg = pl.nseg[pass];
           // norms and super-diagonal dots from the diagonal segments of this pass (row
           // block b is read by the quarter's warp b % 3)
-          if (te == 0) gs->ecount = 0;
 #pragma unroll 1
           for (int si = 0; si < nseg; ++si) {
             const Seg sg = pl.seg[pass][si];
@@ -447,78 +453,130 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (sg.c0 != sg.b * kTileM || sg.b % 3 != rep) continue;
             const int i = sg.b * kTileM + t128;
             if (i < n) {
-              const float rni = gs->n2[i] > 0.f ? 1.0f / sqrtf(gs->n2[i]) : 0.f;
-              gs->rn[i] = rni;
-              gs->col[i] = make_int2(gs->dep[i], __float_as_int(rni));
+              const float n2i = gs->n2[i];
+              gs->rn[i] = n2i > 0.f ? 1.0f / sqrtf(n2i) : 0.f;
+              gs->thr[i] = n2i > 0.f && valid ? kappa * sqrtf(n2i) : __int_as_float(0x7f800000);
             }
           }
           bar_epi();
           // linked pairs: comparable (different rollout [, same depth]) with sim >= kappa,
-          // tested as acc / |z_j| >= kappa |z_i| (one multiply per pair).  Columns of the row's
-          // own rollout, columns j <= i and columns past the group leave through one bit mask
-          // per 32-column chunk.  Each pair found goes to the edge list (or, past its capacity,
-          // straight into the forest).
+          // tested as acc / |z_j| - kappa |z_i| >= 0 (one fma per pair).  In the chain layout
+          // the columns j > i outside i's rollout are exactly j >= rend(i), so one bit mask per
+          // 32-column chunk keeps j in [rend(i), n).  The quarter's chunks that hold a column
+          // right of some row of the warp are dealt round-robin to its three warps.  Each pair
+          // found goes to the edge list (or, past its capacity, straight into the forest).
+          {
+            int dealt = 0;
 #pragma unroll 1
-          for (int si = 0; si < nseg; ++si) {
-            const Seg sg = pl.seg[pass][si];
-            const int rowbase = sg.b * kTileM + q * 32;
-            const int i = rowbase + lane;
-            const bool vrow = valid && i < n;
-            const float thr = vrow && gs->n2[i] > 0.f ? kappa * sqrtf(gs->n2[i]) : __int_as_float(0x7f800000);
-            const int ri = vrow ? gs->roll[i] : 0;
-            const int ra = vrow ? gs->rstart[ri] : 0, re = vrow ? gs->rstart[ri + 1] : 0;
-            const int di = vrow ? gs->dep[i] : -1;
-            const int nch = (sg.len + 31) >> 5;
+            for (int si = 0; si < nseg; ++si) {
+              const Seg sg = pl.seg[pass][si];
+              const int rowbase = sg.b * kTileM + q * 32;
+              const int i = rowbase + lane;
+              const bool vrow = i < n;
+              const float thr = vrow ? gs->thr[i] : __int_as_float(0x7f800000);
+              const int re = vrow ? gs->rend[i] : n;
+              const int di = vrow ? gs->dep[i] : -1;
+              const int nch = (sg.len + 31) >> 5;
 #pragma unroll 1
-            for (int ch = rep; ch < nch; ch += 3) {
-              const int cbase = sg.c0 + ch * 32;
-              if (cbase + 31 <= rowbase) continue;  // no column right of any row of this warp
-              uint32_t r[32];
-              tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(sg.tcol + ch * 32), r);
-              tmem_wait_ld();
-              uint32_t hit = 0u;
-              if (p.rule == GPO_MERGE_SAME_DEPTH) {
+              for (int ch = 0; ch < nch; ++ch) {
+                const int cbase = sg.c0 + ch * 32;
+                if (cbase + 31 <= rowbase) continue;  // no column right of any row of this warp
+                if (dealt++ % 3 != rep) continue;
+                uint32_t r[32];
+                tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(sg.tcol + ch * 32), r);
+                tmem_wait_ld();
+                // bit j of `miss` = sign of acc_j / |z_j| - kappa |z_i| (one fma, exact product):
+                // set when the pair is below the threshold
+                uint32_t miss = 0u;
+                const float4* rn4 = reinterpret_cast<const float4*>(gs->rn + cbase);
 #pragma unroll
-                for (int j = 0; j < 32; ++j) {
-                  const int2 cj = gs->col[cbase + j];
-                  hit |= (uint32_t)((cj.x == di) & (__uint_as_float(r[j]) * __int_as_float(cj.y) >= thr)) << j;
+                for (int j4 = 0; j4 < 8; ++j4) {
+                  const float4 c = rn4[j4];
+                  const float cc[4] = {c.x, c.y, c.z, c.w};
+#pragma unroll
+                  for (int t = 0; t < 4; ++t) {
+                    const int j = 4 * j4 + t;
+                    const uint32_t sgn = __float_as_uint(fmaf(__uint_as_float(r[j]), cc[t], -thr)) >> 31;
+                    miss |= sgn << j;
+                  }
                 }
-              } else {
-#pragma unroll
-                for (int j = 0; j < 32; ++j)
-                  hit |= (uint32_t)(__uint_as_float(r[j]) * gs->rn[cbase + j] >= thr) << j;
-              }
-              const uint32_t own = bits_from(ra - cbase) & ~bits_from(re - cbase);
-              uint32_t mk = vrow ? hit & bits_from(i - cbase + 1) & ~bits_from(n - cbase) & ~own : 0u;
-              if (mk) {
-                int slot = atomicAdd(&gs->ecount, __popc(mk));
-                do {
-                  const int j = cbase + __ffs(mk) - 1;
-                  mk &= mk - 1u;
-                  if (slot < kEdgeList) gs->elist[slot] = (uint32_t)i | ((uint32_t)j << 16);
-                  else uf_union(gs->lab, i, j);
-                  ++slot;
-                } while (mk);
+                uint32_t mk = vrow ? ~miss & bits_from(re - cbase) & ~bits_from(n - cbase) : 0u;
+                if (p.rule == GPO_MERGE_SAME_DEPTH && mk) {
+                  uint32_t m2 = 0u;
+                  for (uint32_t t = mk; t; t &= t - 1u) {
+                    const int j = __ffs(t) - 1;
+                    if (gs->dep[cbase + j] == di) m2 |= 1u << j;
+                  }
+                  mk = m2;
+                }
+                // this warp's part of the edge list: one pair per lane per step, slots by ballot
+                for (uint32_t act = __ballot_sync(0xffffffffu, mk != 0); act;
+                     act = __ballot_sync(0xffffffffu, mk != 0)) {
+                  const int slot = wcount + __popc(act & ((1u << lane) - 1u));
+                  if (mk) {
+                    const int j = cbase + __ffs(mk) - 1;
+                    mk &= mk - 1u;
+                    if (slot < kWarpEdges) wlist[slot] = (uint32_t)i | ((uint32_t)j << 16);
+                    else uf_union(gs->lab, i, j);
+                  }
+                  wcount += __popc(act);
+                }
               }
             }
           }
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&ctl->tempty);  // accumulator free for the next pass
-          // classes = connected components of the linked pairs (Alg. S.1): every thread
-          // unites one listed pair at a time into the shared forest (lock-free; the larger
-          // root is hooked under the smaller, so a class's root is its smallest member).
-          // Lanes stay converged, one union per lane per step.
+          // classes = connected components of the linked pairs (Alg. S.1) in the label forest
+          // lab (lab[x] <= x, within x's class).  Rounds of hooking over every listed pair of
+          // the group (the larger of the two current labels is pointed at the smaller) and
+          // shortcutting (lab[x] = lab[lab[x]]) until no pair has unequal labels and every
+          // label is a root: then each class's label is its smallest member.  The rounds
+          // revisit the pairs of earlier passes, whose links a hook may re-point.  If the list
+          // overflowed (pairs united directly), the listed pairs are united the same way
+          // instead (root-to-root links, which never re-point a link).
+          if (lane == 0 && wcount > kWarpEdges) gs->overflow = 1;
           bar_epi();
-          const int ne = min(gs->ecount, kEdgeList);
+          const int nw = min(wcount, kWarpEdges);  // this warp's listed pairs
+          if (!gs->overflow) {
+            bool conv = false;
 #pragma unroll 1
-          for (int e0 = 0; e0 < ne; e0 += kEpiThreads) {
-            const int e = e0 + te;
-            if (e < ne) {
-              const uint32_t ij = gs->elist[e];
-              uf_union(gs->lab, (int)(ij & 0xFFFFu), (int)(ij >> 16));
+            for (int round = 0; round <= kMaxN && !conv; ++round) {
+              bool ch = false;
+              for (int e = lane; e < nw; e += 32) {
+                const uint32_t ij = wlist[e];
+                const int lu = gs->lab[ij & 0xFFFFu], lv = gs->lab[ij >> 16];
+                if (lu != lv) {
+                  atomicMin(&gs->lab[max(lu, lv)], min(lu, lv));
+                  ch = true;
+                }
+              }
+              for (int x = te; x < n; x += kEpiThreads) {
+                const int l = gs->lab[x], ll = gs->lab[l];
+                if (ll != l) {
+                  gs->lab[x] = ll;
+                  ch = true;
+                }
+              }
+              conv = !bar_any<kBarEpi, kEpiThreads>(ch);
             }
-            __syncwarp();
+            if (!conv) {  // not reached in practice; the unions below are correct from any state
+              for (int e0 = 0; e0 < nw; e0 += 32) {
+                if (e0 + lane < nw) {
+                  const uint32_t ij = wlist[e0 + lane];
+                  uf_union(gs->lab, (int)(ij & 0xFFFFu), (int)(ij >> 16));
+                }
+                __syncwarp();
+              }
+            }
+          } else {
+            for (int e0 = 0; e0 < nw; e0 += 32) {
+              if (e0 + lane < nw) {
+                const uint32_t ij = wlist[e0 + lane];
+                uf_union(gs->lab, (int)(ij & 0xFFFFu), (int)(ij >> 16));
+              }
+              __syncwarp();
+            }
           }
         }
       }

@@ -10,11 +10,11 @@ namespace {
 
 constexpr int kPer = 4;  // states per thread (blockDim >= n / kPer)
 
-// Shared memory: labels, rollout/depth per state, rollout offsets, rewards,
-// then the scratch of group_advantages.
+// Shared memory: labels, rollout/depth per state (16-bit: a group holds at most
+// 4096 states), rollout offsets, rewards, then the scratch of group_advantages.
 __host__ __device__ inline size_t group_smem(int n) {
-  return al16(sizeof(int) * (size_t)n) * 3 + al16(sizeof(int) * (size_t)(n + 1)) + al16((size_t)n) +
-         group_scratch_bytes(n) + 64;
+  return al16(sizeof(int) * (size_t)n) + 2 * al16(sizeof(int16_t) * (size_t)n) + al16(sizeof(int) * (size_t)(n + 1)) +
+         al16((size_t)n) + group_scratch_bytes(n) + 64;
 }
 
 __global__ void __launch_bounds__(1024) groups_kernel(gpo_batch b, gpo_outputs o, Sizes sz, Ws ws, Params p) {
@@ -27,17 +27,17 @@ __global__ void __launch_bounds__(1024) groups_kernel(gpo_batch b, gpo_outputs o
   if (nr == 0 || n == 0 || n > sz.maxn) return;
 
   int* lab = reinterpret_cast<int*>(sm);
-  int* roll = reinterpret_cast<int*>(sm + al16(sizeof(int) * (size_t)n));
-  int* dep = reinterpret_cast<int*>(sm + 2 * al16(sizeof(int) * (size_t)n));
-  int* rstart = reinterpret_cast<int*>(sm + 3 * al16(sizeof(int) * (size_t)n));
-  uint8_t* rew = sm + 3 * al16(sizeof(int) * (size_t)n) + al16(sizeof(int) * (size_t)(n + 1));
+  int16_t* roll = reinterpret_cast<int16_t*>(sm + al16(sizeof(int) * (size_t)n));
+  int16_t* dep = roll + al16(sizeof(int16_t) * (size_t)n) / sizeof(int16_t);
+  int* rstart = reinterpret_cast<int*>(reinterpret_cast<unsigned char*>(dep) + al16(sizeof(int16_t) * (size_t)n));
+  uint8_t* rew = reinterpret_cast<uint8_t*>(rstart) + al16(sizeof(int) * (size_t)(n + 1));
   unsigned char* X = rew + al16((size_t)n);
 
   for (int i = tid; i < n; i += nt) {
     lab[i] = i;
     const int2 m = ws.state_meta[s0 + i];
-    roll[i] = m.x - gi.r0;
-    dep[i] = m.y;
+    roll[i] = (int16_t)(m.x - gi.r0);
+    dep[i] = (int16_t)m.y;
   }
   for (int r = tid; r <= nr; r += nt) rstart[r] = b.rollout_step_off[gi.r0 + r] - s0;
   for (int r = tid; r < nr; r += nt) rew[r] = b.reward[gi.r0 + r];
@@ -84,8 +84,8 @@ __global__ void __launch_bounds__(1024) groups_kernel(gpo_batch b, gpo_outputs o
     if (o.node_score) o.node_score[v] = S;
   };
   __shared__ int s_rootc;
-  group_advantages<kPer, false>(n, nr, lab, roll, dep, rstart, rew, group_scratch_shared(X, n, &s_rootc), p, tid, nt,
-                                [] { __syncthreads(); }, eta, out);
+  group_advantages<kPer, false, int16_t>(n, nr, lab, roll, dep, rstart, rew, group_scratch_shared(X, n, &s_rootc), p,
+                                         tid, nt, [] { __syncthreads(); }, eta, out);
 
   // first token of every edge
   for (int rr = tid; rr < nr; rr += nt) {

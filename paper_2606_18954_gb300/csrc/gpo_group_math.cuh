@@ -45,16 +45,36 @@ __device__ __forceinline__ void uf_union(int* p, int a, int b) {
   }
 }
 
-// Exact, order-independent sum of non-negative fp32 values below 2^26: each value
-// is split into a 2^-36-grid part and a 2^-76-grid remainder (both exact in
-// fp32) that go into two int64 accumulators.
-__device__ __forceinline__ void fx_add32(long long* hi, long long* lo, float x) {
+// Exact, order-independent integer sums through 32-bit shared-memory atomics (64-bit
+// ones are compare-and-swap loops that serialise under contention): a non-negative
+// value below 2^(kChunks * kBits) is added as kChunks chunks of kBits bits, one counter
+// each.  With kBits <= 19 and at most 4096 terms no counter can overflow.
+template <int kChunks, int kBits>
+__device__ __forceinline__ void red_chunks(unsigned* acc, unsigned long long v) {
+#pragma unroll
+  for (int c = 0; c < kChunks; ++c) atomicAdd(&acc[c], (unsigned)((v >> (c * kBits)) & ((1ull << kBits) - 1)));
+}
+
+template <int kChunks, int kBits>
+__device__ __forceinline__ unsigned long long sum_chunks(const unsigned* acc) {
+  unsigned long long s = 0;
+#pragma unroll
+  for (int c = 0; c < kChunks; ++c) s += (unsigned long long)acc[c] << (c * kBits);
+  return s;
+}
+
+// Chunk counters of the sums below (per key).
+constexpr int kSumWords = 3;   // sum of r on the 2^-50 grid: r * 2^50 + 2^50 in [0, 2^51], 3 x 18 bits
+constexpr int kSqhWords = 3;   // sum of (r - mean)^2 on the 2^-36 grid: in [0, 2^38] (|r - mean| <= 2), 3 x 13 bits
+constexpr int kSqlWords = 3;   // and its 2^-76 grid remainder + 2^39, in [0, 2^40], 3 x 14 bits
+
+// Exact sum of x = (r - mean)^2 <= 4: each x splits into a 2^-36-grid part and a
+// 2^-76-grid remainder (both exact in fp32), summed as chunked integers.
+__device__ __forceinline__ void sq_add(unsigned* hi, unsigned* lo, float x) {
   const float X = x * 0x1p36f;
   const float h = rintf(X);
-  const long long hl = __float2ll_rn(h);
-  const long long ll = __float2ll_rn((X - h) * 0x1p40f);
-  atomicAdd(reinterpret_cast<unsigned long long*>(hi), (unsigned long long)hl);
-  atomicAdd(reinterpret_cast<unsigned long long*>(lo), (unsigned long long)ll);
+  red_chunks<kSqhWords, 13>(hi, (unsigned long long)__float2ll_rn(h));
+  red_chunks<kSqlWords, 14>(lo, (unsigned long long)(__float2ll_rn((X - h) * 0x1p40f) + (1ll << 39)));
 }
 
 // Rounded quotient of an int64 by a positive int.
@@ -73,75 +93,65 @@ struct GroupScratch {
   int* ccnt;            // [n]   |Q|
   int* csum;            // [n]   C_Q = sum of the members' rewards
   int* lsum;            // [n]   sum of the members' depths
-  long long* l2;        // [n]   sum of the squared depths
+  unsigned* l2;         // [n][2] sum of the squared depths, 2 x 13-bit chunks
   int* kcnt;            // [n+1] edges per correctness group
-  long long* ksum;      // [n+1] sum of r on the 2^-50 grid
-  long long* kq_hi;     // [n+1] sum of (r - mean)^2, 2^-36 grid part
-  long long* kq_lo;     // [n+1] and 2^-76 grid remainder
-  float* aeff;          // [n]   A_eff of each route end (over ccnt / csum)
+  unsigned* ksum;       // [n+1][kSumWords] sum of r (chunked, see above)
+  unsigned* kqh;        // [n+1][kSqhWords] sum of (r - mean)^2, 2^-36 grid part
+  unsigned* kql;        // [n+1][kSqlWords] and its 2^-76 grid remainder
+  float* aeff;          // [n]   A_eff of each route end (over ccnt)
   float* E;             // [n]   routed A_eff (over lsum)
   unsigned char* cov;   // [n]   covered by a route (over l2)
   int* rootc;           // [1]   sum of the group's rewards
 };
 
+constexpr int kClassWords = 5;                                   // 4-byte words per class
+constexpr int kKeyWords = 1 + kSumWords + kSqhWords + kSqlWords;  // per key
+
 // Separate layout: class and key arrays side by side, for callers that zero
 // them ahead of time (group_scratch_zero); bytes for a group of up to n states.
 __host__ __device__ constexpr size_t group_scratch_sep_bytes(int n) {
-  return al16(12 * (size_t)n) + al16(8 * (size_t)n) + al16(4 * (size_t)(n + 1)) + 3 * al16(8 * (size_t)(n + 1)) + 16;
+  return 4 * (kClassWords * (size_t)n + kKeyWords * (size_t)(n + 1)) + 16;
+}
+
+__device__ __forceinline__ void group_scratch_carve(GroupScratch& g, unsigned char* cls, unsigned char* key, int n) {
+  g.ccnt = reinterpret_cast<int*>(cls);
+  g.csum = g.ccnt + n;
+  g.lsum = g.csum + n;
+  g.l2 = reinterpret_cast<unsigned*>(g.lsum + n);
+  g.kcnt = reinterpret_cast<int*>(key);
+  g.ksum = reinterpret_cast<unsigned*>(g.kcnt + (n + 1));
+  g.kqh = g.ksum + kSumWords * (n + 1);
+  g.kql = g.kqh + kSqhWords * (n + 1);
+  g.aeff = reinterpret_cast<float*>(g.ccnt);
+  g.E = reinterpret_cast<float*>(g.lsum);
+  g.cov = reinterpret_cast<unsigned char*>(g.l2);
 }
 
 __device__ __forceinline__ GroupScratch group_scratch_sep(unsigned char* X, int n) {
   GroupScratch g;
-  g.ccnt = reinterpret_cast<int*>(X);
-  g.csum = g.ccnt + n;
-  g.lsum = g.csum + n;
-  g.l2 = reinterpret_cast<long long*>(X + al16(12 * (size_t)n));
-  unsigned char* k = X + al16(12 * (size_t)n) + al16(8 * (size_t)n);
-  g.kcnt = reinterpret_cast<int*>(k);
-  g.ksum = reinterpret_cast<long long*>(k + al16(4 * (size_t)(n + 1)));
-  g.kq_hi = g.ksum + (n + 1);
-  g.kq_lo = g.kq_hi + (n + 1);
-  g.rootc = reinterpret_cast<int*>(k + al16(4 * (size_t)(n + 1)) + 3 * al16(8 * (size_t)(n + 1)));
-  g.aeff = reinterpret_cast<float*>(g.ccnt);
-  g.E = reinterpret_cast<float*>(g.lsum);
-  g.cov = reinterpret_cast<unsigned char*>(g.l2);
+  group_scratch_carve(g, X, X + 4 * kClassWords * (size_t)n, n);
+  g.rootc = reinterpret_cast<int*>(X + 4 * (kClassWords * (size_t)n + kKeyWords * (size_t)(n + 1)));
   return g;
 }
 
 // Zero the sums of a separate-layout scratch (before the barrier that precedes
 // group_advantages<kPer, true>).
-__device__ __forceinline__ void group_scratch_zero(const GroupScratch& g, int n, int tid, int nt) {
-  for (int i = tid; i < n; i += nt) {
-    g.ccnt[i] = g.csum[i] = g.lsum[i] = 0;
-    g.l2[i] = 0;
-  }
-  for (int i = tid; i <= n; i += nt) {
-    g.kcnt[i] = 0;
-    g.ksum[i] = g.kq_hi[i] = g.kq_lo[i] = 0;
-  }
-  if (tid == 0) *g.rootc = 0;
+__device__ __forceinline__ void group_scratch_zero(unsigned char* X, int n, int tid, int nt) {
+  int* w = reinterpret_cast<int*>(X);
+  const int nw = kClassWords * n + kKeyWords * (n + 1) + 1;
+  for (int i = tid; i < nw; i += nt) w[i] = 0;
 }
 
-// Shared layout: the class, key and route arrays overlay one region (the
-// largest is the key sums, 28 B per key), for large groups; group_advantages
-// zeroes each in turn, at the cost of extra barriers.
+// Shared layout: the class, key and route arrays overlay one region (the largest
+// is the key sums), for large groups; group_advantages zeroes each in turn, at the
+// cost of extra barriers.
 __host__ __device__ constexpr size_t group_scratch_bytes(int n) {
-  return al16(28 * (size_t)(n + 1) + 32);
+  return al16(4 * kKeyWords * (size_t)(n + 1) + 32);
 }
 
 __device__ __forceinline__ GroupScratch group_scratch_shared(unsigned char* X, int n, int* rootc) {
   GroupScratch g;
-  g.ccnt = reinterpret_cast<int*>(X);
-  g.csum = g.ccnt + n;
-  g.lsum = g.csum + n;
-  g.l2 = reinterpret_cast<long long*>(X + al16(12 * (size_t)n));
-  g.kcnt = reinterpret_cast<int*>(X);
-  g.ksum = reinterpret_cast<long long*>(X + al16(4 * (size_t)(n + 1)));
-  g.kq_hi = g.ksum + (n + 1);
-  g.kq_lo = g.kq_hi + (n + 1);
-  g.aeff = reinterpret_cast<float*>(X);
-  g.E = g.aeff + n;
-  g.cov = reinterpret_cast<unsigned char*>(g.E + n);
+  group_scratch_carve(g, X, X, n);
   g.rootc = rootc;
   return g;
 }
@@ -165,8 +175,8 @@ __device__ __forceinline__ GroupScratch group_scratch_shared(unsigned char* X, i
 // that needs them (same operands, same operations, so the same value), which
 // saves a barrier per constant.  Sums go through integer atomics, so results do
 // not depend on the order in which threads add.
-template <int kPer, bool kZeroed, class Sync, class Eta, class Out>
-__device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const int* roll, const int* dep,
+template <int kPer, bool kZeroed, class IdxT, class Sync, class Eta, class Out>
+__device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const IdxT* roll, const IdxT* dep,
                                                  const int* rstart, const uint8_t* rew, const GroupScratch& sc,
                                                  const Params& p, int tid, int nt, Sync sync, Eta eta, Out out) {
   const float w = (float)p.w, eps = (float)p.eps;
@@ -174,7 +184,7 @@ __device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const 
   if (!kZeroed) {
     for (int i = tid; i < n; i += nt) {
       sc.ccnt[i] = sc.csum[i] = sc.lsum[i] = 0;
-      sc.l2[i] = 0;
+      sc.l2[2 * i] = sc.l2[2 * i + 1] = 0u;
     }
     if (tid == 0) *sc.rootc = 0;
     sync();
@@ -192,7 +202,7 @@ __device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const 
       atomicAdd(&sc.ccnt[lb[k]], 1);
       atomicAdd(&sc.csum[lb[k]], (int)rew[roll[i]]);
       atomicAdd(&sc.lsum[lb[k]], d);
-      atomicAdd(reinterpret_cast<unsigned long long*>(&sc.l2[lb[k]]), (unsigned long long)((long long)d * d));
+      red_chunks<2, 13>(&sc.l2[2 * lb[k]], (unsigned long long)d * d);  // d <= 4096: d^2 <= 2^24
     }
   }
   for (int r = tid; r < nr; r += nt) atomicAdd(sc.rootc, (int)rew[r]);
@@ -218,7 +228,7 @@ __device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const 
       // sum (l - mean)^2 = (Q sum l^2 - (sum l)^2) / Q with an exact integer numerator;
       // A_eff(v) = Sbar (mean l - l_v) / (sd + eps) = g (sum l - Q l_v)
       const long long ls = sc.lsum[L];
-      const float ss = (float)((long long)Q * sc.l2[L] - ls * ls) / (float)Q;
+      const float ss = (float)((long long)Q * (long long)sum_chunks<2, 13>(&sc.l2[2 * L]) - ls * ls) / (float)Q;
       const float sd = sqrtf(ss / (float)(Q - p.ddof));
       const float g = ((float)sc.csum[L] / (float)Q) / ((sd + eps) * (float)Q);
       route_end[k] = true;
@@ -238,10 +248,7 @@ __device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const 
   // ---- phase B: correctness groups, key = class of p(v), n = the prompt root
   if (!kZeroed) {
     sync();  // class sums no longer read
-    for (int i = tid; i <= n; i += nt) {
-      sc.kcnt[i] = 0;
-      sc.ksum[i] = sc.kq_hi[i] = sc.kq_lo[i] = 0;
-    }
+    for (int i = tid; i < (kKeyWords) * (n + 1); i += nt) reinterpret_cast<int*>(sc.kcnt)[i] = 0;
     sync();
   }
   long long rf[kPer];
@@ -252,7 +259,7 @@ __device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const 
       // |r| <= 1 and a group holds at most 4096 edges: a 2^50 fixed point cannot overflow
       rf[k] = __float2ll_rn(r[k] * 0x1p50f);
       atomicAdd(&sc.kcnt[key[k]], 1);
-      atomicAdd(reinterpret_cast<unsigned long long*>(&sc.ksum[key[k]]), (unsigned long long)rf[k]);
+      red_chunks<kSumWords, 18>(&sc.ksum[kSumWords * key[k]], (unsigned long long)(rf[k] + (1ll << 50)));
     }
   }
   sync();
@@ -261,9 +268,12 @@ __device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const 
   for (int k = 0; k < kPer; ++k) {
     dv[k] = 0.f;
     if (tid + k * nt < n) {
-      const long long mean = div_round(sc.ksum[key[k]], sc.kcnt[key[k]]);  // exact mean on the 2^-50 grid
+      const int cnt = sc.kcnt[key[k]];
+      // offsets removed in unsigned arithmetic (the biased sum can reach 2^63)
+      const long long tot = (long long)(sum_chunks<kSumWords, 18>(&sc.ksum[kSumWords * key[k]]) - ((unsigned long long)cnt << 50));
+      const long long mean = div_round(tot, cnt);  // exact mean on the 2^-50 grid
       dv[k] = (float)(rf[k] - mean) * 0x1p-50f;
-      fx_add32(&sc.kq_hi[key[k]], &sc.kq_lo[key[k]], dv[k] * dv[k]);
+      sq_add(&sc.kqh[kSqhWords * key[k]], &sc.kql[kSqlWords * key[k]], dv[k] * dv[k]);
     }
   }
   sync();
@@ -273,7 +283,9 @@ __device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const 
     acor[k] = 0.f;
     const int K = key[k], cnt = sc.kcnt[K];
     if (tid + k * nt < n && cnt >= 2) {  // groups of one edge get no advantage
-      const float ss = (float)sc.kq_hi[K] * 0x1p-36f + (float)sc.kq_lo[K] * 0x1p-76f;  // sum (r - mean)^2
+      const long long qh = (long long)sum_chunks<kSqhWords, 13>(&sc.kqh[kSqhWords * K]);
+      const long long ql = (long long)(sum_chunks<kSqlWords, 14>(&sc.kql[kSqlWords * K]) - ((unsigned long long)cnt << 39));
+      const float ss = (float)qh * 0x1p-36f + (float)ql * 0x1p-76f;  // sum (r - mean)^2
       acor[k] = dv[k] * (1.0f / (sqrtf(ss / (float)(cnt - p.ddof)) + eps));
     }
   }
@@ -289,14 +301,33 @@ __device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const 
     }
   }
   sync();
-  for (int rr = tid; rr < nr; rr += nt) {
-    float acc = 0.f;
-    unsigned char cov = 0;
-    for (int i = rstart[rr + 1] - 1; i >= rstart[rr]; --i) {
-      acc += sc.aeff[i];
-      cov |= sc.cov[i];
-      sc.E[i] = acc;
-      sc.cov[i] = cov;
+  // suffix sums along each rollout, one warp per rollout: 32 states at a time from the
+  // rollout's end, a shuffle scan within the warp plus the running total of later states
+  {
+    const int lane = tid & 31, nw = nt >> 5;
+    for (int rr = tid >> 5; rr < nr; rr += nw) {
+      const int lo = rstart[rr];
+      float carry = 0.f;
+      bool ccov = false;
+      for (int hi = rstart[rr + 1]; hi > lo; hi -= 32) {
+        const int i = hi - 1 - lane;  // lane 0 holds the last state of the chunk
+        const bool in = i >= lo;
+        float v = in ? sc.aeff[i] : 0.f;
+        const bool c = in && sc.cov[i] != 0;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+          const float y = __shfl_up_sync(0xffffffffu, v, off);
+          if (lane >= off) v += y;
+        }
+        const uint32_t cb = __ballot_sync(0xffffffffu, c);
+        const float tot = __shfl_sync(0xffffffffu, v, 31);
+        if (in) {
+          sc.E[i] = v + carry;
+          sc.cov[i] = (ccov || (cb & (0xFFFFFFFFu >> (31 - lane))) != 0) ? 1 : 0;
+        }
+        carry += tot;
+        ccov = ccov || cb != 0;
+      }
     }
   }
   sync();
