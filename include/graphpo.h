@@ -139,8 +139,29 @@ gpo_status gpo_workspace_size(const gpo_ctx* ctx, const gpo_batch* batch, size_t
 gpo_status gpo_compute(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* out,
                        void* workspace, size_t workspace_bytes, void* stream);
 
+/* The path for prompt groups [first_group, first_group + num_groups) only (the
+ * paper has no counterpart: it lets a caller overlap the upload of later
+ * groups' embeddings with the work on earlier ones).  `batch` and `out`
+ * describe the WHOLE batch, with the same layout, ownership and checks as for
+ * gpo_compute; only the listed groups' embedding rows must hold their values
+ * when the call runs on the GPU, and only their tokens and states are written
+ * (a group's tokens are all written by the call that covers the group).
+ * clear_status != 0 clears the workspace's status words first; calls for later
+ * ranges add to them, so that one gpo_sync_status after the last range reports
+ * the first error of any.  num_groups = 0 with clear_status = 1 only clears.
+ * Calls for disjoint ranges may run concurrently on different streams once the
+ * clearing call has completed; they share the workspace's status words only.
+ * A range other than the whole batch needs the group-resident path (bf16
+ * embeddings, max_states_per_group <= 384, no flags): otherwise
+ * GPO_ERR_UNSUPPORTED.  A range outside [0, num_groups] gives
+ * GPO_ERR_INVALID_ARG. */
+gpo_status gpo_compute_groups(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* out, int64_t first_group,
+                              int64_t num_groups, int clear_status, void* workspace, size_t workspace_bytes,
+                              void* stream);
+
 /* Waits for `stream` and returns the first error the kernels of the last
- * gpo_compute on this context reported (GPO_OK if none). */
+ * gpo_compute (or of the gpo_compute_groups calls since the last clearing one)
+ * on this context reported (GPO_OK if none). */
 gpo_status gpo_sync_status(gpo_ctx* ctx, void* stream);
 
 /* Static description of a status code. */

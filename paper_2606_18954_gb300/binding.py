@@ -55,7 +55,10 @@ class COutputs(ctypes.Structure):
 
 
 EXPORTS = ["gpo_create", "gpo_workspace_size", "gpo_compute", "gpo_sync_status", "gpo_status_string",
-           "gpo_last_error", "gpo_version", "gpo_destroy", "gpo_enable_timing", "gpo_stage_times", "gpo_compute_noalloc"]
+           "gpo_last_error", "gpo_version", "gpo_destroy", "gpo_enable_timing", "gpo_stage_times", "gpo_compute_noalloc",
+           "gpo_compute_groups"]
+
+FUSED_MAX_STATES = 384  # largest group the group-resident path (and gpo_compute_groups) serves
 
 _lib = None
 _lock = threading.Lock()
@@ -84,6 +87,10 @@ def load(build_if_missing: bool = False):
         L.gpo_compute.argtypes = [ctypes.c_void_p, ctypes.POINTER(CBatch), ctypes.POINTER(COutputs),
                                   ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]
         L.gpo_compute.restype = ctypes.c_int
+        L.gpo_compute_groups.argtypes = [ctypes.c_void_p, ctypes.POINTER(CBatch), ctypes.POINTER(COutputs),
+                                         ctypes.c_int64, ctypes.c_int64, ctypes.c_int, ctypes.c_void_p,
+                                         ctypes.c_size_t, ctypes.c_void_p]
+        L.gpo_compute_groups.restype = ctypes.c_int
         L.gpo_sync_status.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
         L.gpo_sync_status.restype = ctypes.c_int
         L.gpo_status_string.argtypes = [ctypes.c_int]
@@ -108,6 +115,11 @@ def load(build_if_missing: bool = False):
 
 def _ptr(t) -> Optional[int]:
     return None if t is None else t.data_ptr()
+
+
+def _c_outputs(out: dict) -> COutputs:
+    return COutputs(*[_ptr(out.get(k)) if out.get(k) is not None and out[k].numel() else None
+                      for k in ("adv", "adv_cor", "adv_eff", "eff_mask", "class_id", "node_score", "edge_adv")])
 
 
 @dataclasses.dataclass
@@ -254,11 +266,23 @@ class GraphPO:
         ws = self.workspace(batch) if workspace is None else workspace
         if stream is None:
             stream = torch.cuda.current_stream(batch.emb.device)
-        co = COutputs(*[_ptr(out.get(k)) if out.get(k) is not None and out[k].numel() else None
-                        for k in ("adv", "adv_cor", "adv_eff", "eff_mask", "class_id", "node_score", "edge_adv")])
+        co = _c_outputs(out)
         cb = batch.c_struct()
         code = self._lib.gpo_compute(self._h, ctypes.byref(cb), ctypes.byref(co), ws.data_ptr(), ws.numel(),
                                      ctypes.c_void_p(stream.cuda_stream))
+        if code != GPO_OK:
+            raise GraphPOError(code, self.last_error())
+
+    def compute_groups(self, batch: Batch, out: dict, first_group: int, num_groups: int, clear_status: bool,
+                       workspace, stream) -> None:
+        """gpo_compute_groups: the path for groups [first_group, first_group + num_groups) of the
+        whole `batch` into the whole `out` (see include/graphpo.h)."""
+        self._groups_raw(batch.c_struct(), _c_outputs(out), first_group, num_groups, clear_status, workspace, stream)
+
+    def _groups_raw(self, cb, co, first_group, num_groups, clear_status, workspace, stream) -> None:
+        code = self._lib.gpo_compute_groups(self._h, ctypes.byref(cb), ctypes.byref(co), int(first_group),
+                                            int(num_groups), int(bool(clear_status)), workspace.data_ptr(),
+                                            workspace.numel(), ctypes.c_void_p(stream.cuda_stream))
         if code != GPO_OK:
             raise GraphPOError(code, self.last_error())
 
@@ -291,14 +315,23 @@ class GraphPO:
         if code != GPO_OK:
             raise GraphPOError(code, self.last_error())
 
-    def compute_host(self, host_batch: Batch, out=None, stream=None) -> "torch.Tensor":
+    def compute_host(self, host_batch: Batch, out=None, stream=None, chunk_bytes=32 << 20) -> "torch.Tensor":
         """End-to-end call on HOST tensors (pinned for asynchronous copies): copies the
         inputs into device staging buffers (kept between calls of the same shape),
         runs the path and copies the per-token advantages back into `out` (a pinned
         float32 tensor of total_tokens elements, allocated if None).  Waits for the
-        result and raises on a device-side error."""
+        result and raises on a device-side error.
+
+        When the group-resident path serves the batch and its embeddings span at least
+        four chunks, the work is pipelined over chunks of groups (about `chunk_bytes` of
+        embeddings each; below four chunks the fixed cost of a pipeline stage outweighs
+        the overlap): chunk k's
+        embeddings are copied in on one stream while earlier chunks run (each on one
+        of a few compute streams, so that their kernels share the GPU) and the
+        advantages of finished chunks are copied back on a third stream."""
         import torch
         dev = torch.device("cuda", torch.cuda.current_device())
+        main = torch.cuda.current_stream(dev) if stream is None else stream
         names = ("group_rollout_off", "rollout_step_off", "step_len", "rollout_token_off", "emb", "reward",
                  "root_emb")
         host = [getattr(host_batch, n) for n in names]
@@ -308,15 +341,71 @@ class GraphPO:
             self._staged = staged
             self._stage_key = key
             self._stage_out = None
-        for h, d in zip(host, self._staged):
-            if h is not None:
-                d.copy_(h, non_blocking=True)
-        db = Batch(*self._staged[:6], host_batch.total_tokens, host_batch.max_states_per_group, self._staged[6])
-        if self._stage_out is None:
-            self._stage_out = self.alloc_outputs(db)
-        self.compute_into(db, self._stage_out, stream=stream)
         if out is None:
             out = torch.empty(host_batch.total_tokens, dtype=torch.float32, pin_memory=True)
-        out.copy_(self._stage_out["adv"], non_blocking=True)
-        self.check(stream)
+        emb_h = host_batch.emb
+        G = host_batch.num_groups
+        nchunk = min(G, max(1, emb_h.numel() * emb_h.element_size() // max(1, chunk_bytes)))
+        piped = (nchunk >= 4 and emb_h.dtype == torch.bfloat16 and self.params.flags == 0 and
+                 host_batch.max_states_per_group <= FUSED_MAX_STATES and emb_h.is_pinned())
+        with torch.cuda.stream(main):
+            for i, (h, d) in enumerate(zip(host, self._staged)):
+                if h is not None and (not piped or names[i] != "emb"):
+                    d.copy_(h, non_blocking=True)
+            db = Batch(*self._staged[:6], host_batch.total_tokens, host_batch.max_states_per_group,
+                       self._staged[6])
+            if self._stage_out is None:
+                self._stage_out = self.alloc_outputs(db)
+            res = self._stage_out["adv"]
+            if not piped:
+                self.compute_into(db, self._stage_out, stream=main)
+                out.copy_(res, non_blocking=True)
+                self.check(main)
+                return out
+            ws = self.workspace(db)
+            # chunks of groups with about equal numbers of states
+            so = host_batch.rollout_step_off
+            go = host_batch.group_rollout_off
+            to = host_batch.rollout_token_off
+            s_of_g = so[go.long()].tolist()
+            t_of_g = to[go.long()].tolist()
+            N = s_of_g[-1]
+            bounds, g = [0], 0
+            for k in range(1, nchunk):
+                target = N * k // nchunk
+                while g < G and s_of_g[g] < target:
+                    g += 1
+                if g > bounds[-1] and g < G:
+                    bounds.append(g)
+            bounds.append(G)
+            if getattr(self, "_pipe_streams", None) is None or self._pipe_streams[0].device != dev:
+                self._pipe_streams = [torch.cuda.Stream(dev) for _ in range(4)]  # in, out, 2 compute
+            s_in, s_out, comp = self._pipe_streams[0], self._pipe_streams[1], self._pipe_streams[2:]
+            cb, co = db.c_struct(), _c_outputs(self._stage_out)
+            self._groups_raw(cb, co, 0, 0, True, ws, main)  # clears the status words
+            ready = torch.cuda.Event()
+            ready.record(main)
+            s_in.wait_event(ready)
+            s_out.wait_event(ready)
+            for cs in comp:
+                cs.wait_event(ready)
+            emb_d = self._staged[4]
+            for k in range(len(bounds) - 1):
+                ga, gb = bounds[k], bounds[k + 1]
+                sa, sb = s_of_g[ga], s_of_g[gb]
+                with torch.cuda.stream(s_in):
+                    emb_d[sa:sb].copy_(emb_h[sa:sb], non_blocking=True)
+                    e_in = torch.cuda.Event()
+                    e_in.record(s_in)
+                cs = comp[k % len(comp)]
+                cs.wait_event(e_in)
+                self._groups_raw(cb, co, ga, gb - ga, False, ws, cs)
+                e_c = torch.cuda.Event()
+                e_c.record(cs)
+                s_out.wait_event(e_c)
+                ta, tb = t_of_g[ga], t_of_g[gb]
+                with torch.cuda.stream(s_out):
+                    out[ta:tb].copy_(res[ta:tb], non_blocking=True)
+            main.wait_stream(s_out)
+        self.check(main)
         return out

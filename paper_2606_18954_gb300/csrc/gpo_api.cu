@@ -254,8 +254,13 @@ gpo_status gpo_workspace_size(const gpo_ctx* ctx, const gpo_batch* batch, size_t
   return GPO_OK;
 }
 
-gpo_status gpo_compute(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* out, void* workspace,
-                       size_t workspace_bytes, void* stream) {
+}  // extern "C"
+
+namespace {
+
+// The path for groups [g0, g1) of the batch; clears the status words first if `clear`.
+gpo_status compute_impl(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* out, void* workspace,
+                        size_t workspace_bytes, int64_t g0, int64_t g1, bool clear, void* stream) {
   if (!ctx) return GPO_ERR_INVALID_ARG;
   ctx->msg[0] = 0;
   gpo_status s = check_batch(ctx, batch);
@@ -280,6 +285,8 @@ gpo_status gpo_compute(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* 
   sz.T = b.total_tokens;
   sz.stride = b.emb_row_stride;
   sz.maxn = b.max_states_per_group;
+  sz.g0 = (int)g0;
+  sz.g1 = (int)g1;
   Params pp;
   pp.kappa = p.kappa;
   pp.w = p.w;
@@ -324,9 +331,16 @@ gpo_status gpo_compute(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* 
   };
   cudaError_t e = cudaSuccess;
   if (ctx->timing) e = cudaEventRecord(ctx->ev[0], lc.stream);
-  if (e == cudaSuccess) e = cudaMemsetAsync(ws.status, 0, sizeof(uint32_t) * kStatusWords, lc.stream);
+  if (e == cudaSuccess && clear) e = cudaMemsetAsync(ws.status, 0, sizeof(uint32_t) * kStatusWords, lc.stream);
   const bool fused = use_tc && !(p.flags & GPO_FLAG_TILED) && sz.G > 0 && sz.maxn <= kFusedMaxStates;
-  if (fused) {
+  const bool whole = g0 == 0 && g1 == sz.G;
+  if (!whole && !fused && g1 > g0) {
+    return set_msg(ctx, "a group range needs the group-resident path (bf16, at most %d states per group, no flags)",
+                   kFusedMaxStates), GPO_ERR_UNSUPPORTED;
+  }
+  if (g1 <= g0) {
+    // nothing to compute (a call that only clears the status words)
+  } else if (fused) {
     if (e == cudaSuccess) e = stage("fused", launch_fused(lc, map, map32, b, *out, sz, ws, pp));
   } else {
   if (e == cudaSuccess) e = stage("prep", launch_prep(lc, b, sz, ws));
@@ -342,6 +356,28 @@ gpo_status gpo_compute(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* 
   ctx->last_status = ws.status;
   if (e != cudaSuccess) return set_msg(ctx, "launch failed: %s", cudaGetErrorString(e)), GPO_ERR_CUDA;
   return GPO_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+gpo_status gpo_compute(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* out, void* workspace,
+                       size_t workspace_bytes, void* stream) {
+  if (!ctx || !batch) return GPO_ERR_INVALID_ARG;
+  return compute_impl(ctx, batch, out, workspace, workspace_bytes, 0, batch->num_groups, true, stream);
+}
+
+gpo_status gpo_compute_groups(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* out, int64_t first_group,
+                              int64_t num_groups, int clear_status, void* workspace, size_t workspace_bytes,
+                              void* stream) {
+  if (!ctx || !batch) return GPO_ERR_INVALID_ARG;
+  if (first_group < 0 || num_groups < 0 || first_group > batch->num_groups ||
+      num_groups > batch->num_groups - first_group)
+    return set_msg(ctx, "group range [%lld, %lld) outside the batch's %lld groups", (long long)first_group,
+                   (long long)(first_group + num_groups), (long long)batch->num_groups), GPO_ERR_INVALID_ARG;
+  return compute_impl(ctx, batch, out, workspace, workspace_bytes, first_group, first_group + num_groups,
+                      clear_status != 0, stream);
 }
 
 gpo_status gpo_enable_timing(gpo_ctx* ctx, int enable) {

@@ -242,7 +242,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     int last_parity[kMaxSlots];
     for (int s = 0; s < kMaxSlots; ++s) last_parity[s] = -1;
     bool ok = true;
-    for (int g = blockIdx.x; g < sz.G && ok; g += gridDim.x) {
+    for (int g = sz.g0 + (int)blockIdx.x; g < sz.g1 && ok; g += gridDim.x) {
       int r0, nr, s0, n;
       if (!group_active(b, sz, g, r0, nr, s0, n)) continue;
       Plan pl;
@@ -281,7 +281,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t phase = 0;
     int u = 0;  // accumulator uses (passes) so far
     bool ok = true;
-    for (int g = blockIdx.x; g < sz.G && ok; g += gridDim.x) {
+    for (int g = sz.g0 + (int)blockIdx.x; g < sz.g1 && ok; g += gridDim.x) {
       int r0, nr, s0, n;
       if (!group_active(b, sz, g, r0, nr, s0, n)) continue;
       Plan pl;
@@ -328,7 +328,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int q = warp & 3;           // TMEM lane quarter of an epilogue warp
     const int wg = warp - 2;          // 0..13
     int u = 0;
-    for (int g = blockIdx.x; g < sz.G; g += gridDim.x) {
+    for (int g = sz.g0 + (int)blockIdx.x; g < sz.g1; g += gridDim.x) {
       int r0 = 0, nr = 0, s0 = 0, n = 0;
       const bool in_range = group_range(b, sz, g, r0, nr, s0, n);
       if (!(in_range && n > 0 && n <= kMaxN && n <= sz.maxn && nr > 0 && nr <= n)) {
@@ -487,7 +487,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tmem_wait_ld();
                 // bit j of `miss` = sign of acc_j / |z_j| - kappa |z_i| (one fma, exact product):
                 // set when the pair is below the threshold
-                uint32_t miss = 0u;
+                // (four partial masks keep the or-chains short)
+                uint32_t mp[4] = {0u, 0u, 0u, 0u};
                 const float4* rn4 = reinterpret_cast<const float4*>(gs->rn + cbase);
 #pragma unroll
                 for (int j4 = 0; j4 < 8; ++j4) {
@@ -496,10 +497,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                   for (int t = 0; t < 4; ++t) {
                     const int j = 4 * j4 + t;
-                    const uint32_t sgn = __float_as_uint(fmaf(__uint_as_float(r[j]), cc[t], -thr)) >> 31;
-                    miss |= sgn << j;
+                    mp[t] |= (__float_as_uint(fmaf(__uint_as_float(r[j]), cc[t], -thr)) >> 31) << j;
                   }
                 }
+                const uint32_t miss = (mp[0] | mp[1]) | (mp[2] | mp[3]);
                 uint32_t mk = vrow ? ~miss & bits_from(re - cbase) & ~bits_from(n - cbase) : 0u;
                 if (p.rule == GPO_MERGE_SAME_DEPTH && mk) {
                   uint32_t m2 = 0u;
@@ -673,8 +674,9 @@ cudaError_t setup_fused() {
 
 cudaError_t launch_fused(const LaunchCtx& lc, const CUtensorMap& map, const CUtensorMap& map32, const gpo_batch& b,
                          const gpo_outputs& o, const Sizes& sz, const Ws& ws, const Params& p) {
-  if (sz.G == 0) return cudaSuccess;
-  const int grid = sz.G < lc.num_sms ? sz.G : lc.num_sms;
+  const int ng = sz.g1 - sz.g0;
+  if (ng <= 0) return cudaSuccess;
+  const int grid = ng < lc.num_sms ? ng : lc.num_sms;
   fused_kernel<<<grid, kThreads, fused_smem(), lc.stream>>>(map, map32, b, o, sz, ws, p);
   return cudaGetLastError();
 }

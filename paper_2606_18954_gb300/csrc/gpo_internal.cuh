@@ -69,6 +69,8 @@ struct Sizes {
   int64_t T;
   int64_t stride;        // embedding row stride in elements
   int maxn;              // max states per group (host bound)
+  int g0, g1;            // groups processed by this call: [g0, g1) (the whole batch but for
+                         // gpo_compute_groups, which only the group-resident path serves)
 };
 
 struct Params {
