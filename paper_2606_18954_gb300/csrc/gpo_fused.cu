@@ -28,8 +28,11 @@ namespace gpo {
 
 namespace {
 
-constexpr int kMaxSlots = 8;                    // pipeline stages at most
-constexpr int kRingBytes = 160 * 1024;          // tile ring: slots of r32(max states) rows x 128 bytes
+constexpr int kMaxSlots = 8;                    // k-slices in flight at most (mbarrier pairs)
+constexpr int kRingBytes = 160 * 1024;          // tile ring
+constexpr int kPlaceBytes = kRingBytes - 96 * 128;  // slices lie below this: the MMA of a group's last
+                                                    // 128-row block reads its A operand up to 96 rows
+                                                    // past the slice (rows that feed unused lanes)
 constexpr int kThreads = 512;
 constexpr int kMaxN = kFusedMaxStates;          // 384
 constexpr int kBoxBytes = kTileM * 128;         // 128 rows x 128 bytes
@@ -53,6 +56,11 @@ struct Plan {
 };
 
 __device__ __forceinline__ int r16(int x) { return (x + 15) & ~15; }
+
+// Byte offset in the ring of the next k-slice of `bytes`: right after the previous
+// one, or back at 0 if it would reach past kPlaceBytes.  Producer and MMA warp
+// place the same sequence of slices with this rule.
+__device__ __forceinline__ int ring_place(int head, int bytes) { return head + bytes <= kPlaceBytes ? head : 0; }
 __device__ __forceinline__ int r32(int x) { return (x + 31) & ~31; }
 
 // Segments of the upper triangle: row block b against columns [128 b, n) in
@@ -199,13 +207,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint32_t* st = ws.status;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int KT = (sz.d + kTileK - 1) / kTileK;
-  // pipeline geometry of this launch: one slot holds a k-slice of r32(max states) rows.  The
-  // MMA of the last 128-row block reads its A operand up to the next multiple of 128 rows
-  // (rows past the group only feed accumulator lanes that are never read), so the ring
-  // keeps that much room behind the last slot.
-  const int maxr = min(max(sz.maxn, 1), kMaxN);
-  const int slot_bytes = r32(maxr) * 128;
-  const int nslots = min(kMaxSlots, (kRingBytes - (((maxr + kTileM - 1) & ~(kTileM - 1)) - r32(maxr)) * 128) / slot_bytes);
   const float kappa = (float)p.kappa;
 
   if (blockIdx.x == 0 && threadIdx.x == 0) {
@@ -237,10 +238,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     // ---------------------------------------------------------------- TMA producer (lane 0)
     if (lane == 0) {
-    int stage = 0;
-    uint32_t phase = 0;
-    int last_parity[kMaxSlots];
-    for (int s = 0; s < kMaxSlots; ++s) last_parity[s] = -1;
+    // A k-slice (64 embedding elements of the rows a pass reads) takes exactly its bytes
+    // of the ring; slice `seq` signals mbarrier pair seq % kMaxSlots.  The slices in flight
+    // form one run in ring order, from the oldest one's offset o to head (wrapping to 0 at
+    // most once), so a new slice at `off` is free to write when fewer than kMaxSlots are in
+    // flight and: the run does not wrap (o < head) and the slice follows head, or wraps to
+    // end by o; or the run wraps (o >= head) and the slice follows head and ends by o.
+    // Otherwise wait for the oldest slice's consumption and look again.
+    int head = 0;
+    uint32_t seq = 0, oldest = 0;  // slices issued; oldest slice not yet seen consumed
+    int f_off[kMaxSlots];
     bool ok = true;
     for (int g = sz.g0 + (int)blockIdx.x; g < sz.g1 && ok; g += gridDim.x) {
       int r0, nr, s0, n;
@@ -250,69 +257,81 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int rows = r32(n);  // rows [0, r32(n)) of the group; the MMAs read no further
       for (int pass = 0; pass < pl.npass && ok; ++pass) {
         const int row0 = pl.npass == 2 && pass == 0 ? kTileM : 0;  // pass 0 of two never reads block 0
-        for (int k = 0; k < KT; ++k) {
-          if (!mbar_wait(&ctl->empty[stage], phase ^ 1u, st, 20)) {
-            ok = false;
-            break;
+        const int bytes = (rows - row0) * 128;
+        for (int k = 0; k < KT && ok; ++k) {
+          const int off = ring_place(head, bytes);
+          while (oldest < seq) {
+            const int o = f_off[oldest % kMaxSlots];
+            const bool busy = seq - oldest >= (uint32_t)kMaxSlots ||
+                              (o < head ? (off != head && off + bytes > o) : (off != head || head + bytes > o));
+            if (!busy) break;
+            if (!mbar_wait(&ctl->empty[oldest % kMaxSlots], (oldest / kMaxSlots) & 1u, st, 20)) {
+              ok = false;
+              break;
+            }
+            ++oldest;
           }
-          unsigned char* t = tiles + stage * slot_bytes;
-          mbar_arrive_expect_tx(&ctl->full[stage], (uint32_t)((rows - row0) * 128));
-          last_parity[stage] = (int)phase;
+          if (!ok) break;
+          const int bi = (int)(seq % kMaxSlots);
+          unsigned char* t = tiles + off;
+          mbar_arrive_expect_tx(&ctl->full[bi], (uint32_t)bytes);
           for (int r = row0; r < rows;) {  // 128-row boxes, then 32-row boxes for the tail
             const bool big = rows - r >= kTileM;
-            tma_load_2d(t + r * 128, big ? &zmap : &zmap32, &ctl->full[stage], k * kTileK, s0 + r);
+            tma_load_2d(t + (r - row0) * 128, big ? &zmap : &zmap32, &ctl->full[bi], k * kTileK, s0 + r);
             r += big ? kTileM : kTailRows;
           }
-          if (++stage == nslots) {
-            stage = 0;
-            phase ^= 1u;
-          }
+          f_off[bi] = off;
+          head = off + bytes;
+          ++seq;
         }
       }
     }
-    for (int s = 0; s < kMaxSlots; ++s)
-      if (last_parity[s] >= 0) mbar_wait(&ctl->full[s], (uint32_t)last_parity[s], st, 21, 200000000ull, false);
+    for (uint32_t j = oldest; j < seq; ++j)  // copies still landing in shared memory
+      mbar_wait(&ctl->full[j % kMaxSlots], (j / kMaxSlots) & 1u, st, 21, 200000000ull, false);
     }
     __syncwarp();
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer (lane 0)
     if (lane == 0) {
-    int stage = 0;
-    uint32_t phase = 0;
-    int u = 0;  // accumulator uses (passes) so far
+    int head = 0;
+    uint32_t seq = 0;  // slices consumed (the producer's sequence)
+    int u = 0;         // accumulator uses (passes) so far
     bool ok = true;
     for (int g = sz.g0 + (int)blockIdx.x; g < sz.g1 && ok; g += gridDim.x) {
       int r0, nr, s0, n;
       if (!group_active(b, sz, g, r0, nr, s0, n)) continue;
       Plan pl;
       make_plan(n, pl);
+      const int rows = r32(n);
       for (int pass = 0; pass < pl.npass && ok; ++pass, ++u) {
+        const int row0 = pl.npass == 2 && pass == 0 ? kTileM : 0;
+        const int bytes = (rows - row0) * 128;
         if (!mbar_wait(&ctl->tempty, ((uint32_t)u & 1u) ^ 1u, st, 22)) {
           ok = false;
           break;
         }
         tc_fence_after();
         for (int k = 0; k < KT; ++k) {
-          if (!mbar_wait(&ctl->full[stage], phase, st, 23)) {
+          const int off = ring_place(head, bytes);
+          head = off + bytes;
+          const int bi = (int)(seq % kMaxSlots);
+          if (!mbar_wait(&ctl->full[bi], (seq / kMaxSlots) & 1u, st, 23)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t t = smem_u32(tiles + stage * slot_bytes);
+          const uint32_t t = smem_u32(tiles + off);
           for (int si = 0; si < pl.nseg[pass]; ++si) {
-            const Seg s = pl.seg[pass][si];
-            const uint64_t ad = smem_desc_k128(t + (uint32_t)(s.b * kBoxBytes));
-            const uint64_t bd = smem_desc_k128(t + (uint32_t)(s.c0 * 128));
-            const uint32_t idesc = idesc_bf16_f32(kTileM, r16(s.len));
+            const Seg sg = pl.seg[pass][si];
+            const uint64_t ad = smem_desc_k128(t + (uint32_t)((sg.b * kTileM - row0) * 128));
+            const uint64_t bd = smem_desc_k128(t + (uint32_t)((sg.c0 - row0) * 128));
+            const uint32_t idesc = idesc_bf16_f32(kTileM, r16(sg.len));
 #pragma unroll
             for (int kk = 0; kk < kTileK / 16; ++kk)
-              mma_bf16_ss(tmem + (uint32_t)s.tcol, ad + 2u * kk, bd + 2u * kk, idesc, (k | kk) != 0);
+              mma_bf16_ss(tmem + (uint32_t)sg.tcol, ad + 2u * kk, bd + 2u * kk, idesc, (k | kk) != 0);
           }
-          mma_commit(&ctl->empty[stage]);
-          if (++stage == nslots) {
-            stage = 0;
-            phase ^= 1u;
-          }
+          mma_commit(&ctl->empty[bi]);
+          ++seq;
         }
         if (ok) mma_commit(&ctl->tfull);
       }
