@@ -8,7 +8,9 @@ namespace gpo {
 
 namespace {
 
-constexpr int kPer = 4;  // states per thread (blockDim >= n / kPer)
+// States per thread: 2 for groups of up to 2048 states, 4 above (blockDim >= n / kPer, at
+// most 1024 threads).
+constexpr int kMaxRounds = 64;  // hook-and-shortcut rounds before falling back to root unions
 
 // Shared memory: labels, rollout/depth per state (16-bit: a group holds at most
 // 4096 states), rollout offsets, rewards, then the scratch of group_advantages.
@@ -17,6 +19,7 @@ __host__ __device__ inline size_t group_smem(int n) {
          al16((size_t)n) + group_scratch_bytes(n) + 64;
 }
 
+template <int kPer>
 __global__ void __launch_bounds__(1024) groups_kernel(gpo_batch b, gpo_outputs o, Sizes sz, Ws ws, Params p) {
   extern __shared__ __align__(16) unsigned char sm[];
   uint32_t* st = ws.status;
@@ -43,18 +46,61 @@ __global__ void __launch_bounds__(1024) groups_kernel(gpo_batch b, gpo_outputs o
   for (int r = tid; r < nr; r += nt) rew[r] = b.reward[gi.r0 + r];
   __syncthreads();
 
-  // equivalence classes from the items' spanning forests
+  // equivalence classes from the items' spanning forests, in the label forest lab
+  // (lab[x] <= x, within x's class): rounds of hooking over every listed pair (the larger of
+  // the two current labels is pointed at the smaller, an atomic min) and shortcutting
+  // (lab[x] = lab[lab[x]]) until no pair has unequal labels and every label is a root: then
+  // each class's label is its smallest member.  Lock-free root unions (correct from any such
+  // forest) finish the job if the rounds have not settled after kMaxRounds.
+  // Items are dealt to warps (one item per warp at a time, lanes over its edges); the items'
+  // edge counts are read once into shared memory (X, free until the group math).
   const int it0 = ws.group_items[g], it1 = ws.group_items[g + 1];
-  for (int it = it0; it < it1; ++it) {
-    const int ne = ws.edge_count[it];
-    const int2* E = ws.edges + (size_t)it * kEdgeCap;
-    for (int e = tid; e < ne; e += nt) {
-      const int2 uv = E[e];
-      const int u = uv.x - s0, v = uv.y - s0;
-      if ((unsigned)u < (unsigned)n && (unsigned)v < (unsigned)n) uf_union(lab, u, v);
-    }
-  }
+  const int nit = it1 - it0;
+  int* ecnt = reinterpret_cast<int*>(X);
+  const bool cached = (size_t)nit * sizeof(int) <= group_scratch_bytes(n);
+  if (cached)
+    for (int k = tid; k < nit; k += nt) ecnt[k] = min(ws.edge_count[it0 + k], kEdgeCap);
   __syncthreads();
+  const int lane = tid & 31, wid = tid >> 5, nwarp = nt >> 5;
+  bool settled = false;
+  for (int round = 0; round < kMaxRounds && !settled; ++round) {
+    int ch = 0;
+    for (int k = wid; k < nit; k += nwarp) {
+      const int ne = cached ? ecnt[k] : min(ws.edge_count[it0 + k], kEdgeCap);
+      const int2* E = ws.edges + (size_t)(it0 + k) * kEdgeCap;
+      for (int e = lane; e < ne; e += 32) {
+        const int2 uv = E[e];
+        const int u = uv.x - s0, v = uv.y - s0;
+        if ((unsigned)u < (unsigned)n && (unsigned)v < (unsigned)n) {
+          const int lu = lab[u], lv = lab[v];
+          if (lu != lv) {
+            atomicMin(&lab[max(lu, lv)], min(lu, lv));
+            ch = 1;
+          }
+        }
+      }
+    }
+    for (int x = tid; x < n; x += nt) {
+      const int l = lab[x], ll = lab[l];
+      if (ll != l) {
+        lab[x] = ll;
+        ch = 1;
+      }
+    }
+    settled = __syncthreads_or(ch) == 0;
+  }
+  if (!settled) {
+    for (int it = it0; it < it1; ++it) {
+      const int ne = ws.edge_count[it];
+      const int2* E = ws.edges + (size_t)it * kEdgeCap;
+      for (int e = tid; e < ne; e += nt) {
+        const int2 uv = E[e];
+        const int u = uv.x - s0, v = uv.y - s0;
+        if ((unsigned)u < (unsigned)n && (unsigned)v < (unsigned)n) uf_union(lab, u, v);
+      }
+    }
+    __syncthreads();
+  }
 
   // eta(p(v), v) from the fp32 row statistics; zero rows give 0
   auto eta = [&](int i) -> float {
@@ -87,18 +133,32 @@ __global__ void __launch_bounds__(1024) groups_kernel(gpo_batch b, gpo_outputs o
   group_advantages<kPer, false, int16_t>(n, nr, lab, roll, dep, rstart, rew, group_scratch_shared(X, n, &s_rootc), p,
                                          tid, nt, [] { __syncthreads(); }, eta, out);
 
-  // first token of every edge
-  for (int rr = tid; rr < nr; rr += nt) {
-    int64_t t = b.rollout_token_off[gi.r0 + rr];
-    for (int i = rstart[rr]; i < rstart[rr + 1]; ++i) {
-      ws.tok_start[s0 + i] = t;
-      t += b.step_len[s0 + i];
+  // first token of every edge: one warp per rollout, an exclusive scan of the step lengths
+  {
+    const int lane = tid & 31;
+    for (int rr = tid >> 5; rr < nr; rr += nt >> 5) {
+      int64_t t = b.rollout_token_off[gi.r0 + rr];
+      for (int i0 = rstart[rr]; i0 < rstart[rr + 1]; i0 += 32) {
+        const int i = i0 + lane;
+        const int64_t len = i < rstart[rr + 1] ? b.step_len[s0 + i] : 0;
+        int64_t incl = len;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int64_t y = __shfl_up_sync(0xffffffffu, incl, o);
+          if (lane >= o) incl += y;
+        }
+        if (i < rstart[rr + 1]) ws.tok_start[s0 + i] = t + incl - len;
+        t += __shfl_sync(0xffffffffu, incl, 31);
+      }
     }
   }
 }
 
+constexpr int kPerSmall = 2, kPerLarge = 4, kSmallMax = 2048;
+
 int groups_threads(int maxn) {
-  int t = (maxn + kPer - 1) / kPer;
+  const int per = maxn <= kSmallMax ? kPerSmall : kPerLarge;
+  int t = (maxn + per - 1) / per;
   t = (t + 31) & ~31;
   return t < 64 ? 64 : (t > 1024 ? 1024 : t);
 }
@@ -108,14 +168,20 @@ int groups_threads(int maxn) {
 size_t groups_smem_bytes(int maxn) { return group_smem(maxn < 1 ? 1 : maxn); }
 
 cudaError_t setup_groups() {
-  return cudaFuncSetAttribute(groups_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              (int)group_smem(GPO_MAX_GROUP_STATES));
+  const int bytes = (int)group_smem(GPO_MAX_GROUP_STATES);
+  cudaError_t e = cudaFuncSetAttribute(groups_kernel<kPerSmall>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(groups_kernel<kPerLarge>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  return e;
 }
 
 cudaError_t launch_groups(const LaunchCtx& lc, const gpo_batch& b, const gpo_outputs& o, const Sizes& sz,
                           const Ws& ws, const Params& p) {
   if (sz.G == 0) return cudaSuccess;
-  groups_kernel<<<sz.G, groups_threads(sz.maxn), groups_smem_bytes(sz.maxn), lc.stream>>>(b, o, sz, ws, p);
+  if (sz.maxn <= kSmallMax)
+    groups_kernel<kPerSmall><<<sz.G, groups_threads(sz.maxn), groups_smem_bytes(sz.maxn), lc.stream>>>(b, o, sz, ws, p);
+  else
+    groups_kernel<kPerLarge><<<sz.G, groups_threads(sz.maxn), groups_smem_bytes(sz.maxn), lc.stream>>>(b, o, sz, ws, p);
   return cudaGetLastError();
 }
 

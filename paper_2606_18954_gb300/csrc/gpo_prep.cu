@@ -65,22 +65,31 @@ __global__ void __launch_bounds__(kPlanThreads) prep_kernel(gpo_batch b, Sizes s
     }
     for (int r = a; r < c; ++r) ws.rollout_group[r] = g;
   }
-  for (int r = tid; r < sz.R; r += nth) {
+  // one warp per rollout: its lanes stride over the rollout's steps
+  const int lane = threadIdx.x & 31;
+  for (int r = tid >> 5; r < sz.R; r += nth >> 5) {
     const int s = so[r], e = so[r + 1];
     if (s < 0 || e <= s || e > sz.N) {  // every rollout has at least one step
-      report(st, GPO_ERR_SHAPE, 0, 4);
+      if (lane == 0) report(st, GPO_ERR_SHAPE, 0, 4);
       continue;
     }
-    if (b.reward[r] > 1) report(st, GPO_ERR_BAD_REWARD, 0, r);
+    if (lane == 0 && b.reward[r] > 1) report(st, GPO_ERR_BAD_REWARD, 0, r);
     int64_t sum = 0;
-    for (int v = s; v < e; ++v) {
+    bool bad = false;
+    for (int v = s + lane; v < e; v += 32) {
       const int L = b.step_len[v];
-      if (L < 1) report(st, GPO_ERR_SHAPE, 0, 5);
+      bad |= L < 1;
       sum += L;
       ws.state_meta[v] = make_int2(r, v - s + 1);
     }
-    const int64_t t0 = to[r], t1 = to[r + 1];
-    if (t0 < 0 || t1 > sz.T || t1 - t0 != sum) report(st, GPO_ERR_SHAPE, 0, 6);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    bad = __any_sync(0xffffffffu, bad);
+    if (lane == 0) {
+      if (bad) report(st, GPO_ERR_SHAPE, 0, 5);
+      const int64_t t0 = to[r], t1 = to[r + 1];
+      if (t0 < 0 || t1 > sz.T || t1 - t0 != sum) report(st, GPO_ERR_SHAPE, 0, 6);
+    }
   }
 
   // ---- last block: plan the work items
@@ -145,7 +154,7 @@ __global__ void __launch_bounds__(kPlanThreads) prep_kernel(gpo_batch b, Sizes s
 }
 
 cudaError_t launch_prep(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws) {
-  const int64_t work = (int64_t)sz.R + sz.G + 1;
+  const int64_t work = 32 * ((int64_t)sz.R + 1);  // a warp per rollout
   int blocks = (int)((work + kPlanThreads - 1) / kPlanThreads);
   blocks = blocks < 1 ? 1 : (blocks > 4 * lc.num_sms ? 4 * lc.num_sms : blocks);
   prep_kernel<<<blocks, kPlanThreads, 0, lc.stream>>>(b, sz, ws);
