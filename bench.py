@@ -135,15 +135,24 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows), "gpu_index": self.index}
 
 
-def traffic_for(kernel_file):
-    """DRAM bytes per launch from the committed ncu summary, if the kernel is unchanged since."""
+def kernel_source_sha256(kernel_file):
+    """Hash of a kernel's source file and the shared headers of the library."""
+    csrc = os.path.join(ROOT, "paper_2606_18954_gb300", "csrc")
+    h = hashlib.sha256()
+    for name in [kernel_file] + sorted(f for f in os.listdir(csrc) if f.endswith(".cuh")):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
+
+
+def traffic_for(kernel_file, workload):
+    """DRAM bytes per launch from the committed ncu summary of this kernel on this workload,
+    if the kernel's sources are unchanged since the capture."""
     try:
         with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
             t = json.load(f)
-        ent = t[kernel_file]
-        src = os.path.join(ROOT, "paper_2606_18954_gb300", "csrc", kernel_file)
-        h = hashlib.sha256(open(src, "rb").read()).hexdigest()
-        if h != ent["source_sha256"]:
+        ent = t[kernel_file][workload]
+        if kernel_source_sha256(kernel_file) != ent["source_sha256"]:
             return None, "kernel changed since the capture"
         return float(ent["bytes_per_launch"]), ent.get("note", "")
     except Exception:
@@ -337,7 +346,7 @@ def run_ours(args):
     else:
         roof = {"bound": "hbm", "achieved": sb / t_dom / 1e9, "peak": hbm, "unit": "GB/s"}
     roof["frac"] = roof["achieved"] / roof["peak"]
-    traffic, tnote = traffic_for(STAGE_SOURCE.get(dom, ""))
+    traffic, tnote = traffic_for(STAGE_SOURCE.get(dom, ""), args.config)
     roof.update(traffic=traffic, kernel=dom, peak_source=f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured"
                 else "fallback", traffic_note=tnote)
     path_t = max(alg["path_bytes"] / (hbm * 1e9), alg["flops"] / (tc * 1e12))
