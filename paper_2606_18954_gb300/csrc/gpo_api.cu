@@ -347,7 +347,7 @@ gpo_status compute_impl(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs*
   if (e == cudaSuccess && sz.N > 0) {
     e = stage("row_stats", launch_row_stats(lc, b, sz, ws));
     if (e == cudaSuccess)
-      e = stage("similarity", use_tc ? launch_sim_tc(lc, map, sz, ws, pp) : launch_sim_simt(lc, b, sz, ws, pp));
+      e = stage("similarity", use_tc ? launch_sim_tc(lc, map, b, sz, ws, pp) : launch_sim_simt(lc, b, sz, ws, pp));
     if (e == cudaSuccess) e = stage("groups", launch_groups(lc, b, *out, sz, ws, pp));
     if (e == cudaSuccess) e = stage("tokens", launch_tokens(lc, b, *out, sz, ws));
   }

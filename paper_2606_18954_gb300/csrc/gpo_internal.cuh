@@ -283,8 +283,8 @@ struct LaunchCtx {
 
 cudaError_t launch_prep(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws);
 cudaError_t launch_row_stats(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws);
-cudaError_t launch_sim_tc(const LaunchCtx& lc, const CUtensorMap& map, const Sizes& sz, const Ws& ws,
-                          const Params& p);
+cudaError_t launch_sim_tc(const LaunchCtx& lc, const CUtensorMap& map, const gpo_batch& b, const Sizes& sz,
+                          const Ws& ws, const Params& p);
 cudaError_t launch_sim_simt(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws,
                             const Params& p);
 cudaError_t launch_groups(const LaunchCtx& lc, const gpo_batch& b, const gpo_outputs& o, const Sizes& sz,

@@ -11,10 +11,14 @@
 //   warp 0 (one lane)  TMA producer: 128-row boxes of Z, 64 bf16 wide, 128B swizzle
 //   warp 1 (one lane)  MMA issuer: D[128 x N] += A[128 x 64] * B[N x 64]^T per k-step,
 //                      fp32 accumulators in TMEM, two buffers of 256 columns
-//   warps 4..7         epilogue: TMEM -> registers, cos = acc / (|z_i||z_j|),
-//                      pair mask + threshold, union into a shared-memory
-//                      union-find of the item's <=384 states, then the item's
-//                      spanning forest (<=383 edges) is written out.
+//   warps 4..15        epilogue, three warps per TMEM lane quarter splitting the
+//                      32-column chunks: pair test acc / |z_j| >= kappa |z_i| (one
+//                      fma per pair, comparable columns by one range mask per
+//                      chunk), linked pairs into per-warp edge lists, accumulator
+//                      released, then classes of the item's <= 384 states by
+//                      hook-and-shortcut rounds in shared memory, and the item's
+//                      spanning forest (<= 383 edges, state -> smallest state of
+//                      its class) written out.
 // The Gram block Z_g Z_g^T is never written to memory.
 #include "gpo_internal.cuh"
 
@@ -23,12 +27,15 @@ namespace gpo {
 namespace {
 
 constexpr int kStages = 4;
-constexpr int kThreads = 256;
+constexpr int kThreads = 512;
 constexpr int kBoxBytes = kTileM * 128;            // one 128-row x 128-byte box
 constexpr int kStageBytes = 3 * kBoxBytes;         // A box + two B boxes
 constexpr int kSlots = kTileM + kTileN;            // local union-find slots
 constexpr int kTmemCols = 512;                     // two accumulators of 256 columns
-constexpr int kEpiBarrier = 1;                     // named barrier of the 4 epilogue warps
+constexpr int kEpiBarrier = 1;                     // named barrier of the epilogue warps
+constexpr int kEpiThreads = 384;                   // warps 4..15
+constexpr int kEpiWarps = kEpiThreads / 32;
+constexpr int kWarpEdges = 256;                    // linked pairs listed per epilogue warp and item
 
 struct __align__(8) SmemCtl {
   uint64_t full[kStages];
@@ -38,13 +45,19 @@ struct __align__(8) SmemCtl {
   uint64_t drain;
   uint32_t tmem_base;
   int edge_n;
-  int lp[kSlots];
-  int cm_roll[kTileN];
+  int overflow;                    // some warp found more pairs than its list holds
+  int lp[kSlots];                  // label forest of the item's slots (rows, then columns)
   int cm_depth[kTileN];
-  float cm_rn[kTileN];
+  alignas(16) float cm_rn[kTileN];  // 1 / |z| of the item's columns
+  uint32_t elist[kEpiWarps][kWarpEdges];  // slot pairs (row slot | column slot << 16)
 };
 
-__device__ __forceinline__ void epi_sync() { asm volatile("bar.sync %0, 128;" ::"n"(kEpiBarrier) : "memory"); }
+__device__ __forceinline__ void epi_sync() {
+  asm volatile("bar.sync %0, %1;" ::"n"(kEpiBarrier), "n"(kEpiThreads) : "memory");
+}
+
+// Bits a..31 of a word (all for a <= 0, none for a >= 32).
+__device__ __forceinline__ uint32_t bits_from(int a) { return a <= 0 ? 0xFFFFFFFFu : (a >= 32 ? 0u : 0xFFFFFFFFu << a); }
 
 // Barrier of the 4 epilogue warps that also ORs a flag across them, so that
 // they all take the same early exit.
@@ -53,10 +66,10 @@ __device__ __forceinline__ bool epi_any(bool flag) {
   asm volatile(
       "{\n\t.reg .pred p, q;\n\t"
       "setp.ne.u32 p, %1, 0;\n\t"
-      "bar.red.or.pred q, %2, 128, p;\n\t"
+      "bar.red.or.pred q, %2, %3, p;\n\t"
       "selp.u32 %0, 1, 0, q;\n\t}"
       : "=r"(out)
-      : "r"((uint32_t)flag), "n"(kEpiBarrier)
+      : "r"((uint32_t)flag), "n"(kEpiBarrier), "n"(kEpiThreads)
       : "memory");
   return out != 0;
 }
@@ -86,7 +99,8 @@ __device__ __forceinline__ void lunion(int* p, int a, int b) {
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
-    sim_tc_kernel(const __grid_constant__ CUtensorMap zmap, Sizes sz, Ws ws, float kappa, int rule) {
+    sim_tc_kernel(const __grid_constant__ CUtensorMap zmap, const int32_t* __restrict__ rollout_step_off, Sizes sz,
+                  Ws ws, float kappa, int rule) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   // control block first, then the tiles on a 1024-byte boundary (128B swizzle); both are
   // smem_raw plus an offset, so the compiler keeps the shared address space
@@ -108,7 +122,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&ctl->tfull[b], 1);
-      mbar_init(&ctl->tempty[b], 4);
+      mbar_init(&ctl->tempty[b], kEpiWarps);
     }
     mbar_init(&ctl->drain, 1);
     fence_mbar_init();
@@ -207,87 +221,159 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else if (warp >= 4) {
     // ------------------------------------------------------------ epilogue
-    const int q = warp & 3;
-    const int t = q * 32 + lane;  // accumulator row = TMEM lane
+    const int q = warp & 3;            // TMEM lane quarter
+    const int rep = (warp - 4) >> 2;   // 0..2: which of the quarter's three warps
+    const int ew = warp - 4;           // epilogue warp 0..11
+    const int te = threadIdx.x - 128;  // 0..383
+    const int t = q * 32 + lane;       // accumulator row = TMEM lane
+    uint32_t* wlist = ctl->elist[ew];
     int m = 0;
     for (int it = blockIdx.x; it < nitems; it += gridDim.x, ++m) {
       const Item item = ws.items[it];
       const GroupInfo gi = ws.groups[item.group];
       const int send = gi.s0 + gi.n;
       const int buf = m & 1;
-      epi_sync();  // previous item finished with the column metadata
-      for (int c = t; c < item.ncols; c += 128) {
-        const int2 mt = ws.state_meta[item.col0 + c];
-        ctl->cm_roll[c] = mt.x;
-        ctl->cm_depth[c] = mt.y;
+      epi_sync();  // previous item finished with the metadata, lists and forest
+      for (int c = te; c < item.ncols; c += kEpiThreads) {
+        ctl->cm_depth[c] = ws.state_meta[item.col0 + c].y;
         ctl->cm_rn[c] = ws.rn[item.col0 + c];
       }
-      if (t == 0) ctl->edge_n = 0;
+      for (int c = item.ncols + te; c < kTileN; c += kEpiThreads) ctl->cm_rn[c] = 0.f;
+      if (te == 0) {
+        ctl->edge_n = 0;
+        ctl->overflow = 0;
+      }
+      // row constants: kappa |z_i| (+inf for a zero or absent row), end of the row's
+      // rollout (in the chain layout the comparable columns right of row i are exactly
+      // those at or after it), depth
       const int row = item.row0 + t;
-      const bool vrow = row < send;
-      int2 rmeta = make_int2(-1, -1);
-      float rn_i = 0.f;
-      if (vrow) {
-        rmeta = ws.state_meta[row];
-        rn_i = ws.rn[row];
+      float thr = __int_as_float(0x7f800000);
+      int re = send, di = -1;
+      if (row < send) {
+        const int2 mt = ws.state_meta[row];
+        const float rni = ws.rn[row];
+        if (rni > 0.f) thr = kappa / rni;
+        re = rollout_step_off[mt.x + 1];
+        di = mt.y;
       }
       epi_sync();
       const bool got = mbar_wait(&ctl->tfull[buf], (uint32_t)(m >> 1) & 1u, st, 15);
       if (epi_any(!got)) break;
       tc_fence_after();
-      // pass masks first (branch-free), unions afterwards over the few set bits
+      // linked pairs: chunks holding a column right of some row of the warp, dealt
+      // round-robin to the quarter's three warps; one pair per lane per step into the
+      // warp's list (slots by ballot), past its capacity straight into the forest
       const int nchunks = (item.ncols + 31) >> 5;
-      uint32_t masks[kTileN / 32];
-#pragma unroll
-      for (int ch = 0; ch < kTileN / 32; ++ch) masks[ch] = 0u;
-#pragma unroll
-      for (int ch = 0; ch < kTileN / 32; ++ch) {
-        if (ch >= nchunks) break;
-        // a chunk whose last column is at or above no row of this warp holds no pair col > row
-        if (item.col0 + ch * 32 + 31 <= item.row0 + q * 32) continue;
+      const int cend = item.col0 + item.ncols;
+      int wcount = 0, dealt = 0;
+      for (int ch = 0; ch < nchunks; ++ch) {
+        const int cb = item.col0 + ch * 32;
+        if (cb + 31 <= item.row0 + q * 32) continue;
+        if (dealt++ % 3 != rep) continue;
         uint32_t r[32];
         tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * kTileN + ch * 32), r);
         tmem_wait_ld();
-        uint32_t mk = 0u;
+        uint32_t mp[4] = {0u, 0u, 0u, 0u};
+        const float4* rn4 = reinterpret_cast<const float4*>(ctl->cm_rn + ch * 32);
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          const int c = ch * 32 + j;
-          const bool ok = (c < item.ncols) & (item.col0 + c > row) & (ctl->cm_roll[c] != rmeta.x) &
-                          ((rule != GPO_MERGE_SAME_DEPTH) | (ctl->cm_depth[c] == rmeta.y)) &
-                          (__uint_as_float(r[j]) * rn_i * ctl->cm_rn[c] >= kappa);
-          mk |= (uint32_t)ok << j;
+        for (int j4 = 0; j4 < 8; ++j4) {
+          const float4 c = rn4[j4];
+          const float cc[4] = {c.x, c.y, c.z, c.w};
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const int j = 4 * j4 + u;
+            mp[u] |= (__float_as_uint(fmaf(__uint_as_float(r[j]), cc[u], -thr)) >> 31) << j;
+          }
         }
-        masks[ch] = vrow ? mk : 0u;
+        const uint32_t miss = (mp[0] | mp[1]) | (mp[2] | mp[3]);
+        uint32_t mk = ~miss & bits_from(re - cb) & ~bits_from(cend - cb);
+        if (rule == GPO_MERGE_SAME_DEPTH && mk) {
+          uint32_t m2 = 0u;
+          for (uint32_t x = mk; x; x &= x - 1u) {
+            const int j = __ffs(x) - 1;
+            if (ctl->cm_depth[ch * 32 + j] == di) m2 |= 1u << j;
+          }
+          mk = m2;
+        }
+        for (uint32_t act = __ballot_sync(0xffffffffu, mk != 0); act; act = __ballot_sync(0xffffffffu, mk != 0)) {
+          const int slot = wcount + __popc(act & ((1u << lane) - 1u));
+          if (mk) {
+            const int col = cb + __ffs(mk) - 1;
+            mk &= mk - 1u;
+            const int sc = col < item.row0 + kTileM ? col - item.row0 : kTileM + (col - item.col0);
+            if (slot < kWarpEdges) wlist[slot] = (uint32_t)t | ((uint32_t)sc << 16);
+            else lunion(ctl->lp, t, sc);
+          }
+          wcount += __popc(act);
+        }
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&ctl->tempty[buf]);  // accumulator free for the next item
-#pragma unroll
-      for (int ch = 0; ch < kTileN / 32; ++ch) {
-        uint32_t mk = masks[ch];
-        while (mk) {
-          const int j = __ffs(mk) - 1;
-          mk &= mk - 1u;
-          const int col = item.col0 + ch * 32 + j;
-          const int slot_col = (col < item.row0 + kTileM) ? col - item.row0 : kTileM + (col - item.col0);
-          lunion(ctl->lp, t, slot_col);
-        }
+      if (lane == 0) {
+        mbar_arrive(&ctl->tempty[buf]);  // accumulator free for the next item
+        if (wcount > kWarpEdges) ctl->overflow = 1;
       }
       epi_sync();
-      // spanning forest of this item: one edge per non-root slot
+      // classes of the item's slots: hook-and-shortcut rounds over the listed pairs (the
+      // larger of two current labels is pointed at the smaller) until every pair has
+      // equal labels and every label is a root; lock-free root unions if a list overflowed
+      const int nw = min(wcount, kWarpEdges);
+      if (!ctl->overflow) {
+        bool conv = false;
+        for (int round = 0; round <= kSlots && !conv; ++round) {
+          bool chg = false;
+          for (int e = lane; e < nw; e += 32) {
+            const uint32_t ij = wlist[e];
+            const int lu = ctl->lp[ij & 0xFFFFu], lv = ctl->lp[ij >> 16];
+            if (lu != lv) {
+              atomicMin(&ctl->lp[max(lu, lv)], min(lu, lv));
+              chg = true;
+            }
+          }
+          for (int x = te; x < kSlots; x += kEpiThreads) {
+            const int l = ctl->lp[x], ll = ctl->lp[l];
+            if (ll != l) {
+              ctl->lp[x] = ll;
+              chg = true;
+            }
+          }
+          conv = !epi_any(chg);
+        }
+        if (!conv) {
+          for (int e0 = 0; e0 < nw; e0 += 32) {
+            if (e0 + lane < nw) lunion(ctl->lp, (int)(wlist[e0 + lane] & 0xFFFFu), (int)(wlist[e0 + lane] >> 16));
+            __syncwarp();
+          }
+          epi_sync();
+        }
+      } else {
+        for (int e0 = 0; e0 < nw; e0 += 32) {
+          if (e0 + lane < nw) lunion(ctl->lp, (int)(wlist[e0 + lane] & 0xFFFFu), (int)(wlist[e0 + lane] >> 16));
+          __syncwarp();
+        }
+        epi_sync();
+      }
+      // spanning forest of this item: one edge per non-root slot, to its class's root
       int2* out = ws.edges + (size_t)it * kEdgeCap;
-      for (int s = t; s < kSlots; s += 128) {
-        const int root = lfind(ctl->lp, s);
-        if (root != s) {
-          const int gs = s < kTileM ? item.row0 + s : item.col0 + (s - kTileM);
+      for (int s0 = 0; s0 < kSlots; s0 += kEpiThreads) {
+        const int sl = s0 + te;
+        int root = sl;
+        if (sl < kSlots) root = lfind(ctl->lp, sl);
+        const bool edge = sl < kSlots && root != sl;
+        const uint32_t act = __ballot_sync(0xffffffffu, edge);
+        int base = 0;
+        if (lane == 0 && act) base = atomicAdd(&ctl->edge_n, __popc(act));
+        base = __shfl_sync(0xffffffffu, base, 0);
+        if (edge) {
+          const int k = base + __popc(act & ((1u << lane) - 1u));
+          const int gs = sl < kTileM ? item.row0 + sl : item.col0 + (sl - kTileM);
           const int gr = root < kTileM ? item.row0 + root : item.col0 + (root - kTileM);
-          const int k = atomicAdd(&ctl->edge_n, 1);
           if (k < kEdgeCap) out[k] = make_int2(gr, gs);
         }
       }
       epi_sync();
-      for (int s = t; s < kSlots; s += 128) ctl->lp[s] = s;
-      if (t == 0) ws.edge_count[it] = min(ctl->edge_n, kEdgeCap);
+      for (int x = te; x < kSlots; x += kEpiThreads) ctl->lp[x] = x;
+      if (te == 0) ws.edge_count[it] = min(ctl->edge_n, kEdgeCap);
     }
   }
 
@@ -306,11 +392,12 @@ cudaError_t setup_sim_tc() {
                               (int)sim_tc_smem_bytes());
 }
 
-cudaError_t launch_sim_tc(const LaunchCtx& lc, const CUtensorMap& map, const Sizes& sz, const Ws& ws,
-                          const Params& p) {
+cudaError_t launch_sim_tc(const LaunchCtx& lc, const CUtensorMap& map, const gpo_batch& b, const Sizes& sz,
+                          const Ws& ws, const Params& p) {
   int grid = ws.max_items < lc.num_sms ? ws.max_items : lc.num_sms;
   if (grid < 1) return cudaSuccess;
-  sim_tc_kernel<<<grid, kThreads, sim_tc_smem_bytes(), lc.stream>>>(map, sz, ws, (float)p.kappa, p.rule);
+  sim_tc_kernel<<<grid, kThreads, sim_tc_smem_bytes(), lc.stream>>>(map, b.rollout_step_off, sz, ws, (float)p.kappa,
+                                                                      p.rule);
   return cudaGetLastError();
 }
 
