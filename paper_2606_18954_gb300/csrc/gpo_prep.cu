@@ -96,6 +96,7 @@ __global__ void __launch_bounds__(kPlanThreads) prep_kernel(gpo_batch b, Sizes s
   __shared__ int s_last;
   __shared__ int s_warp[32];
   __shared__ int s_carry;
+  __shared__ int s_incl[kPlanThreads], s_s0[kPlanThreads], s_n[kPlanThreads];
   __threadfence();
   __syncthreads();
   if (threadIdx.x == 0) s_last = atomicAdd(&st[kStTicket], 1u) == gridDim.x - 1;
@@ -124,22 +125,40 @@ __global__ void __launch_bounds__(kPlanThreads) prep_kernel(gpo_batch b, Sizes s
     }
     const int incl = block_incl_scan(cnt, s_warp);
     const int first = s_carry + incl - cnt;
-    if (ok && g < sz.G) {
-      ws.group_items[g] = first;
-      int k = first;
-      for (int rb = 0; rb * kTileM < n; ++rb)
-        for (int c0 = rb * kTileM; c0 < n; c0 += kTileN) {
-          if (k < ws.max_items) {
-            Item it;
-            it.row0 = s0 + rb * kTileM;
-            it.col0 = s0 + c0;
-            it.ncols = min(kTileN, n - c0);
-            it.group = g;
-            ws.items[k] = it;
-            ws.edge_count[k] = 0;
-          }
-          ++k;
-        }
+    if (ok && g < sz.G) ws.group_items[g] = first;
+    // the items of this batch of groups, written by the whole block: item j of the batch
+    // belongs to the group whose prefix range holds it (binary search in shared memory),
+    // then to the row block whose chunk range holds it
+    s_incl[threadIdx.x] = incl;
+    s_s0[threadIdx.x] = s0;
+    s_n[threadIdx.x] = n;
+    __syncthreads();
+    const int batch_items = s_incl[kPlanThreads - 1];
+    for (int j = threadIdx.x; j < batch_items && ok; j += kPlanThreads) {
+      int lo = 0, hi = kPlanThreads - 1;  // first t with s_incl[t] > j
+      while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (s_incl[mid] > j) hi = mid;
+        else lo = mid + 1;
+      }
+      const int gn = s_n[lo], gs0 = s_s0[lo];
+      int idx = j - (s_incl[lo] - items_for(gn));  // item index within the group
+      int rb = 0;
+      for (;; ++rb) {
+        const int c = (gn - rb * kTileM + kTileN - 1) / kTileN;
+        if (idx < c) break;
+        idx -= c;
+      }
+      const int k = s_carry + j;
+      if (k < ws.max_items) {
+        Item it;
+        it.row0 = gs0 + rb * kTileM;
+        it.col0 = gs0 + rb * kTileM + idx * kTileN;
+        it.ncols = min(kTileN, gn - rb * kTileM - idx * kTileN);
+        it.group = base + lo;
+        ws.items[k] = it;
+        ws.edge_count[k] = 0;
+      }
     }
     __syncthreads();
     if (threadIdx.x == kPlanThreads - 1) s_carry += incl;
@@ -256,13 +275,118 @@ __global__ void __launch_bounds__(256) row_stats_kernel(gpo_batch b, Sizes sz, W
   }
 }
 
+// bf16 rows of d = 8 * 32 * kNV elements at most: one warp walks a run of 32
+// consecutive rows (one coalesced metadata load for the run), holds a whole row in
+// registers (kNV 16-byte chunks per lane) and keeps it as the parent of the next
+// row, so every row is read once.  The prompt rows (|root|^2) and the dots of first
+// steps against them come from the generic kernel's formula with plain loads.
+template <int kNV>
+__global__ void __launch_bounds__(256) row_stats_run_kernel(gpo_batch b, Sizes sz, Ws ws) {
+  if (aborted(ws.status)) return;
+  const int lane = threadIdx.x & 31;
+  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  const int nvec = sz.d / 8;
+  const uint4* Z = reinterpret_cast<const uint4*>(b.emb);
+  const int64_t rs = sz.stride / 8;  // row stride in 16-byte chunks
+  auto load_row = [&](int64_t r, uint4 (&x)[kNV]) {
+#pragma unroll
+    for (int c = 0; c < kNV; ++c) {
+      const int k = lane + 32 * c;
+      x[c] = k < nvec ? Z[r * rs + k] : make_uint4(0u, 0u, 0u, 0u);
+    }
+  };
+  auto dot2 = [](uint32_t a, uint32_t b) {  // two bf16 pairs, fp32 products
+    return __uint_as_float(a << 16) * __uint_as_float(b << 16) +
+           __uint_as_float(a & 0xFFFF0000u) * __uint_as_float(b & 0xFFFF0000u);
+  };
+  for (int64_t base = warp * 32; base < sz.N; base += nwarps * 32) {
+    const int64_t nrun = min((int64_t)32, (int64_t)sz.N - base);
+    const int2 m = lane < nrun ? ws.state_meta[base + lane] : make_int2(0, 1);
+    uint4 prev[kNV], cur[kNV], nxt[kNV];
+    const int d0 = __shfl_sync(0xffffffffu, m.y, 0);
+    if (d0 > 1) load_row(base - 1, prev);
+    load_row(base, nxt);
+    for (int i = 0; i < nrun; ++i) {
+      const int dep = __shfl_sync(0xffffffffu, m.y, i);
+      const int rol = __shfl_sync(0xffffffffu, m.x, i);
+#pragma unroll
+      for (int c = 0; c < kNV; ++c) cur[c] = nxt[c];
+      if (i + 1 < nrun) load_row(base + i + 1, nxt);  // next row in flight during this one
+      float s2 = 0.f, sd = 0.f;
+#pragma unroll
+      for (int c = 0; c < kNV; ++c) {
+        const uint32_t w[4] = {cur[c].x, cur[c].y, cur[c].z, cur[c].w};
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+          const float lo = __uint_as_float(w[h] << 16), hi = __uint_as_float(w[h] & 0xFFFF0000u);
+          s2 = fmaf(lo, lo, s2);
+          s2 = fmaf(hi, hi, s2);
+        }
+      }
+      if (dep > 1) {
+#pragma unroll
+        for (int c = 0; c < kNV; ++c) {
+          sd += dot2(cur[c].x, prev[c].x) + dot2(cur[c].y, prev[c].y);
+          sd += dot2(cur[c].z, prev[c].z) + dot2(cur[c].w, prev[c].w);
+        }
+      } else if (b.root_emb) {
+        const uint16_t* R = reinterpret_cast<const uint16_t*>(b.root_emb) + (int64_t)ws.rollout_group[rol] * sz.stride;
+        const uint16_t* X = reinterpret_cast<const uint16_t*>(b.emb) + (base + i) * sz.stride;
+        for (int k = lane; k < sz.d; k += 32)
+          sd = fmaf(__uint_as_float((uint32_t)X[k] << 16), __uint_as_float((uint32_t)R[k] << 16), sd);
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        s2 += __shfl_xor_sync(0xffffffffu, s2, o);
+        sd += __shfl_xor_sync(0xffffffffu, sd, o);
+      }
+      if (lane == 0) {
+        const int64_t row = base + i;
+        if (!isfinite(s2) || !isfinite(sd)) report(ws.status, GPO_ERR_NONFINITE, 1, (int)row);
+        ws.nrm2[row] = s2;
+        ws.dotp[row] = sd;
+        ws.rn[row] = s2 > 0.f ? 1.0f / sqrtf(s2) : 0.f;
+      }
+#pragma unroll
+      for (int c = 0; c < kNV; ++c) prev[c] = cur[c];
+    }
+  }
+  // |root|^2 of every prompt embedding
+  if (b.root_emb) {
+    const uint16_t* R = reinterpret_cast<const uint16_t*>(b.root_emb);
+    for (int64_t g = warp; g < sz.G; g += nwarps) {
+      float s2 = 0.f;
+      for (int k = lane; k < sz.d; k += 32) {
+        const float x = __uint_as_float((uint32_t)R[g * sz.stride + k] << 16);
+        s2 = fmaf(x, x, s2);
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) s2 += __shfl_xor_sync(0xffffffffu, s2, o);
+      if (lane == 0) {
+        if (!isfinite(s2)) report(ws.status, GPO_ERR_NONFINITE, 1, (int)(sz.N + g));
+        ws.root_n2[g] = s2;
+      }
+    }
+  }
+}
+
 cudaError_t launch_row_stats(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws) {
   const int64_t jobs = (int64_t)sz.N + (b.root_emb ? sz.G : 0);
   if (jobs == 0) return cudaSuccess;
   int64_t blocks = (jobs * 32 + 255) / 256;
   const int64_t cap = (int64_t)lc.num_sms * 8;
   if (blocks > cap) blocks = cap;
-  if (b.emb_dtype == GPO_EMB_BF16)
+  const bool aligned16 = (reinterpret_cast<uintptr_t>(b.emb) & 15u) == 0 && sz.stride % 8 == 0 && sz.d % 8 == 0;
+  if (b.emb_dtype == GPO_EMB_BF16 && aligned16 && sz.d <= 8 * 32 * 8) {
+    int64_t rblocks = ((int64_t)sz.N + 255) / 256;  // a warp per 32 rows
+    if (rblocks < 1) rblocks = 1;
+    if (rblocks > (int64_t)lc.num_sms * 8) rblocks = (int64_t)lc.num_sms * 8;
+    if (sz.d <= 8 * 32 * 4)
+      row_stats_run_kernel<4><<<(int)rblocks, 256, 0, lc.stream>>>(b, sz, ws);
+    else
+      row_stats_run_kernel<8><<<(int)rblocks, 256, 0, lc.stream>>>(b, sz, ws);
+  } else if (b.emb_dtype == GPO_EMB_BF16)
     row_stats_kernel<true><<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
   else
     row_stats_kernel<false><<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
