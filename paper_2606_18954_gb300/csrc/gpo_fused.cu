@@ -249,6 +249,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t seq = 0, oldest = 0;  // slices issued; oldest slice not yet seen consumed
     int f_off[kMaxSlots];
     bool ok = true;
+    // L2 policy: pass 0 of a two-pass group keeps its rows (pass 1 reads them again),
+    // pass 1 drops them first (their last read)
+    const uint64_t keep = l2_policy_evict_last(), drop = l2_policy_evict_first();
     for (int g = sz.g0 + (int)blockIdx.x; g < sz.g1 && ok; g += gridDim.x) {
       int r0, nr, s0, n;
       if (!group_active(b, sz, g, r0, nr, s0, n)) continue;
@@ -258,6 +261,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int pass = 0; pass < pl.npass && ok; ++pass) {
         const int row0 = pl.npass == 2 && pass == 0 ? kTileM : 0;  // pass 0 of two never reads block 0
         const int bytes = (rows - row0) * 128;
+        const int hint = pl.npass == 1 ? 0 : (pass == 0 ? 1 : 2);
         for (int k = 0; k < KT && ok; ++k) {
           const int off = ring_place(head, bytes);
           while (oldest < seq) {
@@ -277,7 +281,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           mbar_arrive_expect_tx(&ctl->full[bi], (uint32_t)bytes);
           for (int r = row0; r < rows;) {  // 128-row boxes, then 32-row boxes for the tail
             const bool big = rows - r >= kTileM;
-            tma_load_2d(t + (r - row0) * 128, big ? &zmap : &zmap32, &ctl->full[bi], k * kTileK, s0 + r);
+            if (hint == 0)
+              tma_load_2d(t + (r - row0) * 128, big ? &zmap : &zmap32, &ctl->full[bi], k * kTileK, s0 + r);
+            else
+              tma_load_2d_hint(t + (r - row0) * 128, big ? &zmap : &zmap32, &ctl->full[bi], k * kTileK, s0 + r,
+                               hint == 1 ? keep : drop);
             r += big ? kTileM : kTailRows;
           }
           f_off[bi] = off;
