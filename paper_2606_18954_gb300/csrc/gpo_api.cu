@@ -56,13 +56,16 @@ void set_msg(gpo_ctx* c, const char* fmt, ...) {
 constexpr size_t kAlign = 256;
 inline size_t up(size_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
 
+int64_t max_blocks_for(int64_t N, int64_t G) { return N / 128 + G + 8; }  // sum of ceil(n/128)
+
 int64_t max_items_for(int64_t N, int64_t G, int64_t maxn) {
-  // sum over groups of items_for(n) <= sum n^2/32768 + 3n/256 + 1
-  return N * maxn / 32768 + (3 * N) / 256 + G + 8;
+  // per group: ceil(n/128) diagonal items plus the off-diagonal chunks of 256 columns,
+  // at most n^2/32768 + 3n/256 + 1
+  return N * maxn / 32768 + (3 * N) / 256 + G + max_blocks_for(N, G);
 }
 
 struct Layout {
-  size_t status, items, group_items, groups, state_meta, rollout_group, nrm2, dotp, rn, root_n2, edge_count,
+  size_t status, items, blk_ready, groups, state_meta, rollout_group, nrm2, dotp, rn, root_n2, edge_count,
       edges, e_adv, e_cor, e_eff, e_mask, tok_start, total;
   int max_items;
 };
@@ -80,7 +83,7 @@ bool layout(const gpo_batch& b, Layout& L) {
   };
   L.status = take(sizeof(uint32_t) * kStatusWords);
   L.items = take(sizeof(Item) * mi);
-  L.group_items = take(sizeof(int) * (G + 1));
+  L.blk_ready = take(sizeof(int) * mi);  // indexed by the diagonal items' positions
   L.groups = take(sizeof(GroupInfo) * G);
   L.state_meta = take(sizeof(int2) * N);
   L.rollout_group = take(sizeof(int) * R);
@@ -104,7 +107,7 @@ Ws workspace_views(void* base, const Layout& L) {
   Ws w;
   w.status = reinterpret_cast<uint32_t*>(p + L.status);
   w.items = reinterpret_cast<Item*>(p + L.items);
-  w.group_items = reinterpret_cast<int*>(p + L.group_items);
+  w.blk_ready = reinterpret_cast<int*>(p + L.blk_ready);
   w.groups = reinterpret_cast<GroupInfo*>(p + L.groups);
   w.state_meta = reinterpret_cast<int2*>(p + L.state_meta);
   w.rollout_group = reinterpret_cast<int*>(p + L.rollout_group);
@@ -345,7 +348,10 @@ gpo_status compute_impl(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs*
   } else {
   if (e == cudaSuccess) e = stage("prep", launch_prep(lc, b, sz, ws));
   if (e == cudaSuccess && sz.N > 0) {
-    e = stage("row_stats", launch_row_stats(lc, b, sz, ws));
+    // the tcgen05 similarity kernel takes the norms and parent dots from the Gram tiles
+    // themselves; only the prompt-embedding dots need a pass over the rows
+    if (!use_tc) e = stage("row_stats", launch_row_stats(lc, b, sz, ws));
+    else if (b.root_emb) e = stage("root_stats", launch_root_stats(lc, b, sz, ws));
     if (e == cudaSuccess)
       e = stage("similarity", use_tc ? launch_sim_tc(lc, map, b, sz, ws, pp) : launch_sim_simt(lc, b, sz, ws, pp));
     if (e == cudaSuccess) e = stage("groups", launch_groups(lc, b, *out, sz, ws, pp));

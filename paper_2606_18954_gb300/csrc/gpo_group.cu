@@ -54,20 +54,20 @@ __global__ void __launch_bounds__(1024) groups_kernel(gpo_batch b, gpo_outputs o
   // forest) finish the job if the rounds have not settled after kMaxRounds.
   // Items are dealt to warps (one item per warp at a time, lanes over its edges); the items'
   // edge counts are read once into shared memory (X, free until the group math).
-  const int it0 = ws.group_items[g], it1 = ws.group_items[g + 1];
-  const int nit = it1 - it0;
+  const int nit = gi.nblk + gi.noff;  // the group's diagonal items, then its off-diagonal ones
+  auto item_at = [&](int k) { return k < gi.nblk ? gi.blk0 + k : gi.off0 + (k - gi.nblk); };
   int* ecnt = reinterpret_cast<int*>(X);
   const bool cached = (size_t)nit * sizeof(int) <= group_scratch_bytes(n);
   if (cached)
-    for (int k = tid; k < nit; k += nt) ecnt[k] = min(ws.edge_count[it0 + k], kEdgeCap);
+    for (int k = tid; k < nit; k += nt) ecnt[k] = min(ws.edge_count[item_at(k)], kEdgeCap);
   __syncthreads();
   const int lane = tid & 31, wid = tid >> 5, nwarp = nt >> 5;
   bool settled = false;
   for (int round = 0; round < kMaxRounds && !settled; ++round) {
     int ch = 0;
     for (int k = wid; k < nit; k += nwarp) {
-      const int ne = cached ? ecnt[k] : min(ws.edge_count[it0 + k], kEdgeCap);
-      const int2* E = ws.edges + (size_t)(it0 + k) * kEdgeCap;
+      const int ne = cached ? ecnt[k] : min(ws.edge_count[item_at(k)], kEdgeCap);
+      const int2* E = ws.edges + (size_t)item_at(k) * kEdgeCap;
       for (int e = lane; e < ne; e += 32) {
         const int2 uv = E[e];
         const int u = uv.x - s0, v = uv.y - s0;
@@ -90,9 +90,9 @@ __global__ void __launch_bounds__(1024) groups_kernel(gpo_batch b, gpo_outputs o
     settled = __syncthreads_or(ch) == 0;
   }
   if (!settled) {
-    for (int it = it0; it < it1; ++it) {
-      const int ne = ws.edge_count[it];
-      const int2* E = ws.edges + (size_t)it * kEdgeCap;
+    for (int k = 0; k < nit; ++k) {
+      const int ne = min(ws.edge_count[item_at(k)], kEdgeCap);
+      const int2* E = ws.edges + (size_t)item_at(k) * kEdgeCap;
       for (int e = tid; e < ne; e += nt) {
         const int2 uv = E[e];
         const int u = uv.x - s0, v = uv.y - s0;

@@ -40,13 +40,15 @@ struct Item {
 struct GroupInfo {
   int s0, n;        // states [s0, s0+n)
   int r0, nr;       // rollouts [r0, r0+nr)
+  int blk0, nblk;   // its 128-row blocks: diagonal items [blk0, blk0+nblk)
+  int off0, noff;   // then its off-diagonal items [off0, off0+noff), off0 = blk0 + nblk
 };
 
 // Device pointers into the caller's workspace (computed on the host).
 struct Ws {
   uint32_t* status;      // [kStatusWords]
-  Item* items;           // [max_items]
-  int* group_items;      // [G+1]
+  Item* items;           // [max_items]: per group, its diagonal items, then its off-diagonal ones
+  int* blk_ready;        // [max_items]: at a diagonal item's position, set once it has written its norms
   GroupInfo* groups;     // [G]
   int2* state_meta;      // [N] {rollout, depth}
   int* rollout_group;    // [R]
@@ -147,6 +149,37 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32
     if (mbar_try_wait(bar, parity)) return true;
     if ((it & 255u) == 0u) {
       if (honor_abort && aborted(st)) return false;
+      if (globaltimer_ns() - t0 > limit_ns) {
+        report(st, GPO_ERR_TIMEOUT, where, 0);
+        return false;
+      }
+    }
+  }
+}
+
+// ------------------------------------------------------------------ flags between CTAs
+
+__device__ __forceinline__ int ld_acquire_gpu(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void st_release_gpu(int* p, int v) {
+  asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// Waits until *flag != 0 (acquire).  Gives up after `limit_ns` or when the abort flag
+// is raised, reporting GPO_ERR_TIMEOUT on a timeout; returns whether the flag was seen.
+__device__ __forceinline__ bool wait_flag(const int* flag, uint32_t* st, int where,
+                                          uint64_t limit_ns = 2000000000ull) {
+  if (ld_acquire_gpu(flag)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t it = 1;; ++it) {
+    __nanosleep(64);
+    if (ld_acquire_gpu(flag)) return true;
+    if ((it & 63u) == 0u) {
+      if (aborted(st)) return false;
       if (globaltimer_ns() - t0 > limit_ns) {
         report(st, GPO_ERR_TIMEOUT, where, 0);
         return false;
@@ -305,6 +338,7 @@ struct LaunchCtx {
 
 cudaError_t launch_prep(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws);
 cudaError_t launch_row_stats(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws);
+cudaError_t launch_root_stats(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws);
 cudaError_t launch_sim_tc(const LaunchCtx& lc, const CUtensorMap& map, const gpo_batch& b, const Sizes& sz,
                           const Ws& ws, const Params& p);
 cudaError_t launch_sim_simt(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws,

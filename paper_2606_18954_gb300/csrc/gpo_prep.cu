@@ -6,11 +6,20 @@ namespace gpo {
 
 constexpr int kPlanThreads = 1024;
 
-// Similarity work items of a group with n states: row blocks of 128 states,
-// each against the columns at or after its own first state, in chunks of 256.
-__host__ __device__ inline int items_for(int n) {
+// Similarity work items of a group with n states, in row blocks of 128 states: one
+// diagonal item per block (the block against itself; it also yields the block's
+// norms), and off-diagonal items (the block against the columns after it, in chunks
+// of 256).
+__host__ __device__ inline int blocks_for(int n) { return (n + kTileM - 1) / kTileM; }
+
+__host__ __device__ inline int offdiag_chunks(int n, int rb) {
+  const int rem = n - (rb + 1) * kTileM;
+  return rem > 0 ? (rem + kTileN - 1) / kTileN : 0;
+}
+
+__host__ __device__ inline int offdiag_for(int n) {
   int c = 0;
-  for (int rb = 0; rb * kTileM < n; ++rb) c += (n - rb * kTileM + kTileN - 1) / kTileN;
+  for (int rb = 0; rb * kTileM < n; ++rb) c += offdiag_chunks(n, rb);
   return c;
 }
 
@@ -106,67 +115,75 @@ __global__ void __launch_bounds__(kPlanThreads) prep_kernel(gpo_batch b, Sizes s
   if (threadIdx.x == 0) s_carry = 0;
   __syncthreads();
   const bool ok = !aborted(st);
+  // items group by group: a group's diagonal items (one per row block, block order), then
+  // its off-diagonal ones; every item an off-diagonal item waits for thus comes before it
   for (int base = 0; base < sz.G; base += kPlanThreads) {
     const int g = base + threadIdx.x;
-    int cnt = 0, s0 = 0, n = 0, r0 = 0;
+    int cnt = 0, nb = 0, s0 = 0, n = 0;
     if (ok && g < sz.G) {
-      r0 = go[g];
-      const int r1 = go[g + 1];
+      const int r0 = go[g], r1 = go[g + 1];
       s0 = so[r0];
       n = so[r1] - s0;
       if (n > sz.maxn || n > GPO_MAX_GROUP_STATES) report(st, GPO_ERR_UNSUPPORTED, 0, g);
+      nb = blocks_for(n);
+      cnt = nb + offdiag_for(n);
+    }
+    const int incl = block_incl_scan(cnt, s_warp);
+    if (ok && g < sz.G) {
       GroupInfo gi;
       gi.s0 = s0;
       gi.n = n;
-      gi.r0 = r0;
-      gi.nr = r1 - r0;
+      gi.r0 = go[g];
+      gi.nr = go[g + 1] - gi.r0;
+      gi.blk0 = s_carry + incl - cnt;
+      gi.nblk = nb;
+      gi.off0 = gi.blk0 + nb;
+      gi.noff = cnt - nb;
       ws.groups[g] = gi;
-      cnt = items_for(n);
     }
-    const int incl = block_incl_scan(cnt, s_warp);
-    const int first = s_carry + incl - cnt;
-    if (ok && g < sz.G) ws.group_items[g] = first;
-    // the items of this batch of groups, written by the whole block: item j of the batch
-    // belongs to the group whose prefix range holds it (binary search in shared memory),
-    // then to the row block whose chunk range holds it
     s_incl[threadIdx.x] = incl;
     s_s0[threadIdx.x] = s0;
     s_n[threadIdx.x] = n;
     __syncthreads();
-    const int batch_items = s_incl[kPlanThreads - 1];
-    for (int j = threadIdx.x; j < batch_items && ok; j += kPlanThreads) {
+    const int batch = s_incl[kPlanThreads - 1];
+    for (int j = threadIdx.x; j < batch && ok; j += kPlanThreads) {
       int lo = 0, hi = kPlanThreads - 1;  // first t with s_incl[t] > j
       while (lo < hi) {
         const int mid = (lo + hi) >> 1;
         if (s_incl[mid] > j) hi = mid;
         else lo = mid + 1;
       }
-      const int gn = s_n[lo], gs0 = s_s0[lo];
-      int idx = j - (s_incl[lo] - items_for(gn));  // item index within the group
-      int rb = 0;
-      for (;; ++rb) {
-        const int c = (gn - rb * kTileM + kTileN - 1) / kTileN;
-        if (idx < c) break;
-        idx -= c;
-      }
+      const int gn = s_n[lo], gs0 = s_s0[lo], gnb = blocks_for(gn);
+      int idx = j - (s_incl[lo] - gnb - offdiag_for(gn));  // item index within the group
       const int k = s_carry + j;
-      if (k < ws.max_items) {
-        Item it;
+      if (k >= ws.max_items) continue;
+      Item it;
+      it.group = base + lo;
+      if (idx < gnb) {  // diagonal item of row block idx
+        it.row0 = it.col0 = gs0 + idx * kTileM;
+        it.ncols = min(kTileM, gn - idx * kTileM);
+        ws.blk_ready[k] = 0;
+      } else {
+        idx -= gnb;
+        int rb = 0;
+        for (;; ++rb) {
+          const int c = offdiag_chunks(gn, rb);
+          if (idx < c) break;
+          idx -= c;
+        }
         it.row0 = gs0 + rb * kTileM;
-        it.col0 = gs0 + rb * kTileM + idx * kTileN;
-        it.ncols = min(kTileN, gn - rb * kTileM - idx * kTileN);
-        it.group = base + lo;
-        ws.items[k] = it;
-        ws.edge_count[k] = 0;
+        it.col0 = gs0 + (rb + 1) * kTileM + idx * kTileN;
+        it.ncols = min(kTileN, gn - (rb + 1) * kTileM - idx * kTileN);
       }
+      ws.items[k] = it;
+      ws.edge_count[k] = 0;
     }
     __syncthreads();
     if (threadIdx.x == kPlanThreads - 1) s_carry += incl;
     __syncthreads();
   }
   if (threadIdx.x == 0) {
-    int total = s_carry;
-    if (ok) ws.group_items[sz.G] = total;
+    const int total = s_carry;
     if (total > ws.max_items) report(st, GPO_ERR_WORKSPACE, 0, total);
     st[kStItems] = aborted(st) ? 0u : (uint32_t)total;
   }
@@ -210,7 +227,9 @@ __device__ __forceinline__ float load1(const void* base, int64_t elem) {
   return reinterpret_cast<const float*>(base)[elem];
 }
 
-template <bool kBf16>
+// kRootsOnly: only what the tcgen05 similarity kernel does not produce itself, i.e. the
+// dots of first steps with the prompt embeddings and |root|^2.
+template <bool kBf16, bool kRootsOnly>
 __global__ void __launch_bounds__(256) row_stats_kernel(gpo_batch b, Sizes sz, Ws ws) {
   if (aborted(ws.status)) return;
   const int lane = threadIdx.x & 31;
@@ -226,6 +245,7 @@ __global__ void __launch_bounds__(256) row_stats_kernel(gpo_batch b, Sizes sz, W
       row = job;
       rowp = b.emb;
       const int2 m = ws.state_meta[job];
+      if (kRootsOnly && m.y > 1) continue;
       if (m.y > 1) {
         parp = b.emb;
         prow = job - 1;
@@ -265,9 +285,11 @@ __global__ void __launch_bounds__(256) row_stats_kernel(gpo_batch b, Sizes sz, W
     if (lane == 0) {
       if (!isfinite(s2) || !isfinite(sd)) report(ws.status, GPO_ERR_NONFINITE, 1, (int)job);
       if (job < sz.N) {
-        ws.nrm2[row] = s2;
+        if (!kRootsOnly) {
+          ws.nrm2[row] = s2;
+          ws.rn[row] = s2 > 0.f ? 1.0f / sqrtf(s2) : 0.f;
+        }
         ws.dotp[row] = sd;
-        ws.rn[row] = s2 > 0.f ? 1.0f / sqrtf(s2) : 0.f;
       } else {
         ws.root_n2[row] = s2;
       }
@@ -371,6 +393,15 @@ __global__ void __launch_bounds__(256) row_stats_run_kernel(gpo_batch b, Sizes s
   }
 }
 
+cudaError_t launch_root_stats(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws) {
+  const int64_t jobs = (int64_t)sz.N + sz.G;
+  if (!b.root_emb || jobs == 0) return cudaSuccess;
+  int64_t blocks = (jobs * 32 + 255) / 256;
+  if (blocks > (int64_t)lc.num_sms * 8) blocks = (int64_t)lc.num_sms * 8;
+  row_stats_kernel<true, true><<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_row_stats(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws) {
   const int64_t jobs = (int64_t)sz.N + (b.root_emb ? sz.G : 0);
   if (jobs == 0) return cudaSuccess;
@@ -387,9 +418,9 @@ cudaError_t launch_row_stats(const LaunchCtx& lc, const gpo_batch& b, const Size
     else
       row_stats_run_kernel<8><<<(int)rblocks, 256, 0, lc.stream>>>(b, sz, ws);
   } else if (b.emb_dtype == GPO_EMB_BF16)
-    row_stats_kernel<true><<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
+    row_stats_kernel<true, false><<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
   else
-    row_stats_kernel<false><<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
+    row_stats_kernel<false, false><<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
   return cudaGetLastError();
 }
 

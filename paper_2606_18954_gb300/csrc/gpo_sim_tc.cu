@@ -5,9 +5,17 @@
 // rollouts; optionally also the same step depth) and whose cosine similarity
 // is >= kappa is linked; the equivalence classes are the connected components.
 //
-// Work item = 128 rows of one group x up to 256 columns of the same group
-// (col0 >= row0, so each unordered pair is visited once).  Persistent CTAs
-// (one per SM) walk the item list.  Warp roles:
+// Work items: per 128-row block of a group, a diagonal item (the block against
+// itself) and off-diagonal items (the block against up to 256 later columns), so
+// each unordered pair is visited once.  A group's diagonal items precede its
+// off-diagonal ones in the list.  A diagonal item takes the block's norms from the
+// diagonal of its Gram tile (|z_i|^2, and <z_i, z_{i+1}> from the super-diagonal),
+// writes them to the workspace and raises the block's ready flag; an off-diagonal
+// item waits (bounded) for the flags of its row and column blocks before its
+// epilogue reads them.  Every wait is on an item earlier in the list, diagonal items
+// never wait, and each CTA takes its items in list order, so every wait ends.
+// Persistent CTAs (one per SM) walk the item list.
+// Warp roles:
 //   warp 0 (one lane)  TMA producer: 128-row boxes of Z, 64 bf16 wide, 128B swizzle
 //   warp 1 (one lane)  MMA issuer: D[128 x N] += A[128 x 64] * B[N x 64]^T per k-step,
 //                      fp32 accumulators in TMEM, two buffers of 256 columns
@@ -232,34 +240,78 @@ __global__ void __launch_bounds__(kThreads, 1)
       const Item item = ws.items[it];
       const GroupInfo gi = ws.groups[item.group];
       const int send = gi.s0 + gi.n;
+      const bool diag = item.col0 == item.row0;
+      const int blk_row = gi.blk0 + (item.row0 - gi.s0) / kTileM;
       const int buf = m & 1;
       epi_sync();  // previous item finished with the metadata, lists and forest
-      for (int c = te; c < item.ncols; c += kEpiThreads) {
-        ctl->cm_depth[c] = ws.state_meta[item.col0 + c].y;
-        ctl->cm_rn[c] = ws.rn[item.col0 + c];
-      }
+      for (int c = te; c < item.ncols; c += kEpiThreads) ctl->cm_depth[c] = ws.state_meta[item.col0 + c].y;
       for (int c = item.ncols + te; c < kTileN; c += kEpiThreads) ctl->cm_rn[c] = 0.f;
       if (te == 0) {
         ctl->edge_n = 0;
         ctl->overflow = 0;
       }
-      // row constants: kappa |z_i| (+inf for a zero or absent row), end of the row's
-      // rollout (in the chain layout the comparable columns right of row i are exactly
-      // those at or after it), depth
+      // row constants: end of the row's rollout (in the chain layout the comparable columns
+      // right of row i are exactly those at or after it) and depth
       const int row = item.row0 + t;
-      float thr = __int_as_float(0x7f800000);
       int re = send, di = -1;
       if (row < send) {
         const int2 mt = ws.state_meta[row];
-        const float rni = ws.rn[row];
-        if (rni > 0.f) thr = kappa / rni;
         re = rollout_step_off[mt.x + 1];
         di = mt.y;
+      }
+      float thr = __int_as_float(0x7f800000);  // kappa |z_i|; +inf for a zero or absent row
+      if (!diag) {
+        // the norms of the row block and of the column blocks come from their diagonal items
+        bool ready = true;
+        if (te == 0) {
+          const int bc = gi.blk0 + (item.col0 - gi.s0) / kTileM;
+          ready = wait_flag(ws.blk_ready + blk_row, st, 16) && wait_flag(ws.blk_ready + bc, st, 16) &&
+                  (item.col0 + kTileM >= send || item.ncols <= kTileM || wait_flag(ws.blk_ready + bc + 1, st, 16));
+        }
+        if (epi_any(!ready)) break;
+        for (int c = te; c < item.ncols; c += kEpiThreads) ctl->cm_rn[c] = __ldcg(ws.rn + item.col0 + c);
+        if (row < send) {
+          const float rni = __ldcg(ws.rn + row);
+          if (rni > 0.f) thr = kappa / rni;
+        }
       }
       epi_sync();
       const bool got = mbar_wait(&ctl->tfull[buf], (uint32_t)(m >> 1) & 1u, st, 15);
       if (epi_any(!got)) break;
       tc_fence_after();
+      if (diag) {
+        // the block's norms: diagonal and super-diagonal of its Gram tile, read by one warp
+        // per lane quarter; published before the flag that releases the block
+        if (rep == 0 && q * 32 < item.ncols) {
+          const uint32_t base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * kTileN + q * 32);
+          uint32_t r[32];
+          tmem_ld_32x32b_x32(base, r);
+          tmem_wait_ld();
+          float dg = 0.f, up = 0.f;
+#pragma unroll
+          for (int k = 0; k < 32; ++k) {
+            if (k == lane) dg = __uint_as_float(r[k]);
+            if (k == lane + 1) up = __uint_as_float(r[k]);
+          }
+          if (q * 32 + 32 < item.ncols) {
+            tmem_ld_32x32b_x32(base + 32u, r);
+            tmem_wait_ld();
+            if (lane == 31) up = __uint_as_float(r[0]);
+          }
+          if (t < item.ncols) {
+            const float rni = dg > 0.f ? 1.0f / sqrtf(dg) : 0.f;
+            ws.nrm2[row] = dg;
+            ws.rn[row] = rni;
+            ctl->cm_rn[t] = rni;
+            if (!isfinite(dg)) report(st, GPO_ERR_NONFINITE, 1, row);
+            if (t + 1 < item.ncols && ctl->cm_depth[t + 1] > 1) ws.dotp[row + 1] = up;
+          }
+          __threadfence();
+        }
+        epi_sync();
+        if (te == 0) st_release_gpu(ws.blk_ready + blk_row, 1);
+        if (t < item.ncols && ctl->cm_rn[t] > 0.f) thr = kappa / ctl->cm_rn[t];
+      }
       // linked pairs: chunks holding a column right of some row of the warp, dealt
       // round-robin to the quarter's three warps; one pair per lane per step into the
       // warp's list (slots by ballot), past its capacity straight into the forest
@@ -273,6 +325,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint32_t r[32];
         tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * kTileN + ch * 32), r);
         tmem_wait_ld();
+        // <z of the block's last row, z of the next block's first row>: the parent dot of
+        // the next block's first state when it continues the same rollout
+        if (ch == 0 && q == 3 && lane == 31 && item.col0 == item.row0 + kTileM && ctl->cm_depth[0] > 1)
+          ws.dotp[item.col0] = __uint_as_float(r[0]);
         uint32_t mp[4] = {0u, 0u, 0u, 0u};
         const float4* rn4 = reinterpret_cast<const float4*>(ctl->cm_rn + ch * 32);
 #pragma unroll
