@@ -598,7 +598,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
             dot = gs->dn[i - 1];
           }
           const float n2v = gs->n2[i];
-          if (n1 > 0.f && n2v > 0.f) e = dot / sqrtf(n1 * n2v);
+          if (n1 > 0.f && n2v > 0.f) e = dot * rsqrtf(n1 * n2v);  // cos(p(v), v); a few ulp
           return e > 0.f ? e : 0.f;
         };
         auto out = [&](int i, int label, float S, float acor, float E, float dual, unsigned char mask) {

@@ -116,7 +116,7 @@ __global__ void __launch_bounds__(1024) groups_kernel(gpo_batch b, gpo_outputs o
       dot = ws.dotp[v];
     }
     const float n2 = ws.nrm2[v];
-    if (n1 > 0.f && n2 > 0.f) e = dot / sqrtf(n1 * n2);
+    if (n1 > 0.f && n2 > 0.f) e = dot * rsqrtf(n1 * n2);  // cos(p(v), v); a few ulp
     return e > 0.f ? e : 0.f;
   };
   auto out = [&](int i, int label, float S, float acor, float E, float dual, unsigned char mask) {

@@ -226,11 +226,14 @@ __device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const 
     if (Q >= 2) {
       // Sbar_Q = mean of S over Q = C_Q / |Q| (every member has t_own = 1);
       // sum (l - mean)^2 = (Q sum l^2 - (sum l)^2) / Q with an exact integer numerator;
-      // A_eff(v) = Sbar (mean l - l_v) / (sd + eps) = g (sum l - Q l_v)
+      // A_eff(v) = Sbar (mean l - l_v) / (sd + eps) = g (sum l - Q l_v),
+      // g = C_Q / (Q^2 (sd + eps)).  Fast reciprocal square root and division here (a few
+      // ulp; A_eff has no exact special value to keep).
       const long long ls = sc.lsum[L];
-      const float ss = (float)((long long)Q * (long long)sum_chunks<2, 13>(&sc.l2[2 * L]) - ls * ls) / (float)Q;
-      const float sd = sqrtf(ss / (float)(Q - p.ddof));
-      const float g = ((float)sc.csum[L] / (float)Q) / ((sd + eps) * (float)Q);
+      const float num = (float)((long long)Q * (long long)sum_chunks<2, 13>(&sc.l2[2 * L]) - ls * ls);
+      const float var = __fdividef(num, (float)Q * (float)(Q - p.ddof));
+      const float sd = var > 0.f ? var * rsqrtf(var) : 0.f;
+      const float g = __fdividef((float)sc.csum[L], (float)Q * (float)Q * (sd + eps));
       route_end[k] = true;
       aeff[k] = g * (float)(sc.lsum[L] - Q * d);
     }
@@ -275,6 +278,10 @@ __device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const 
       dv[k] = (float)(rf[k] - mean) * 0x1p-50f;
       sq_add(&sc.kqh[kSqhWords * key[k]], &sc.kql[kSqlWords * key[k]], dv[k] * dv[k]);
     }
+    if (kZeroed && tid + k * nt < n) {  // route arrays overlay the class sums, read last above
+      sc.aeff[tid + k * nt] = aeff[k];
+      sc.cov[tid + k * nt] = route_end[k] ? 1 : 0;
+    }
   }
   sync();
   float acor[kPer];
@@ -286,21 +293,25 @@ __device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const 
       const long long qh = (long long)sum_chunks<kSqhWords, 13>(&sc.kqh[kSqhWords * K]);
       const long long ql = (long long)(sum_chunks<kSqlWords, 14>(&sc.kql[kSqlWords * K]) - ((unsigned long long)cnt << 39));
       const float ss = (float)qh * 0x1p-36f + (float)ql * 0x1p-76f;  // sum (r - mean)^2
-      acor[k] = dv[k] * (1.0f / (sqrtf(ss / (float)(cnt - p.ddof)) + eps));
+      const float var = __fdividef(ss, (float)(cnt - p.ddof));
+      const float sd = var > 0.f ? var * rsqrtf(var) : 0.f;
+      acor[k] = dv[k] * __fdividef(1.0f, sd + eps);  // a zero deviation stays exactly 0
     }
   }
 
   // ---- phase C: every edge on root -> v receives A_eff(v) (suffix sums per rollout)
-  if (!kZeroed) sync();  // key sums no longer read (the route arrays overlay them)
+  if (!kZeroed) {  // the route arrays overlay the key sums, read last just above
+    sync();
 #pragma unroll
-  for (int k = 0; k < kPer; ++k) {
-    const int i = tid + k * nt;
-    if (i < n) {
-      sc.aeff[i] = aeff[k];
-      sc.cov[i] = route_end[k] ? 1 : 0;
+    for (int k = 0; k < kPer; ++k) {
+      const int i = tid + k * nt;
+      if (i < n) {
+        sc.aeff[i] = aeff[k];
+        sc.cov[i] = route_end[k] ? 1 : 0;
+      }
     }
+    sync();
   }
-  sync();
   // suffix sums along each rollout, one warp per rollout: 32 states at a time from the
   // rollout's end, a shuffle scan within the warp plus the running total of later states
   {
