@@ -89,21 +89,26 @@ __global__ void __launch_bounds__(kThreads) sim_simt_kernel(gpo_batch b, Sizes s
     for (int i = 0; i < 8; ++i)
 #pragma unroll
       for (int j = 0; j < 16; ++j) acc[i][j] = 0.f;
+    // only the tile's valid rows and columns are staged and multiplied (a thread's rows
+    // and columns past them accumulate stale values that the epilogue never reads)
+    const int nrows = min(kTileM, send - item.row0);
+    const bool busy = ty * 8 < nrows && tx * 16 < item.ncols;
 
     for (int k0 = 0; k0 < sz.d; k0 += kKc) {
       __syncthreads();
-      for (int e = threadIdx.x; e < kKc * kTileM; e += kThreads) {
+      for (int e = threadIdx.x; e < kKc * nrows; e += kThreads) {
         const int r = e / kKc, k = e % kKc;
         const int row = item.row0 + r;
         As[k][r] = (row < send && k0 + k < sz.d) ? ld_elem<kBf16>(b.emb, (int64_t)row * sz.stride + k0 + k) : 0.f;
       }
-      for (int e = threadIdx.x; e < kKc * kTileN; e += kThreads) {
+      for (int e = threadIdx.x; e < kKc * item.ncols; e += kThreads) {
         const int c = e / kKc, k = e % kKc;
         Bs[k][c] = (c < item.ncols && k0 + k < sz.d)
                        ? ld_elem<kBf16>(b.emb, (int64_t)(item.col0 + c) * sz.stride + k0 + k)
                        : 0.f;
       }
       __syncthreads();
+      if (busy) {
 #pragma unroll 4
       for (int k = 0; k < kKc; ++k) {
         float a[8], bv[16];
@@ -115,6 +120,7 @@ __global__ void __launch_bounds__(kThreads) sim_simt_kernel(gpo_batch b, Sizes s
         for (int i = 0; i < 8; ++i)
 #pragma unroll
           for (int j = 0; j < 16; ++j) acc[i][j] = fmaf(a[i], bv[j], acc[i][j]);
+      }
       }
     }
     __syncthreads();
