@@ -37,6 +37,8 @@ class _Batch(ctypes.Structure):
         ("group_rollout_off", ctypes.c_void_p), ("rollout_step_off", ctypes.c_void_p),
         ("step_len", ctypes.c_void_p), ("rollout_token_off", ctypes.c_void_p),
         ("emb", ctypes.c_void_p), ("reward", ctypes.c_void_p), ("root_emb", ctypes.c_void_p),
+        ("parent", ctypes.c_void_p), ("group_state_off", ctypes.c_void_p),
+        ("group_token_off", ctypes.c_void_p),
     ]
 
 
@@ -101,35 +103,56 @@ def _c(a, dtype):
     return np.ascontiguousarray(a, dtype=dtype)
 
 
+def _ptr(a):
+    return a.ctypes.data if a is not None and a.size else None
+
+
+def _make_batch(batch: dict, with_root: bool = True):
+    """The C batch for a dict batch (chain layout, or tree layout when it has
+    "parent"), plus the arrays it points into (kept alive by the caller)."""
+    go = _c(batch["group_rollout_off"], np.int32)
+    sl = _c(batch["step_len"], np.int32)
+    rw = _c(batch["reward"], np.uint8)
+    is_bf16 = batch["emb_dtype"] == "bf16"
+    emb = _c(batch["emb"], np.uint16 if is_bf16 else np.float32)
+    root = batch.get("root_emb") if with_root else None
+    if root is not None:
+        root = _c(root, np.uint16 if is_bf16 else np.float32)
+    G, R, N = len(go) - 1, len(rw), int(emb.shape[0])
+    if batch.get("parent") is not None:
+        par = _c(batch["parent"], np.int32)
+        gs = _c(batch["group_state_off"], np.int32)
+        gt = _c(batch["group_token_off"], np.int64)
+        so = to = None
+        T = int(batch.get("total_tokens", gt[-1] if len(gt) else 0))
+    else:
+        par = gs = gt = None
+        so = _c(batch["rollout_step_off"], np.int32)
+        to = _c(batch["rollout_token_off"], np.int64)
+        R = len(so) - 1
+        T = int(batch.get("total_tokens", to[-1] if len(to) else 0))
+    keep = [go, so, sl, to, rw, emb, root, par, gs, gt]
+
+    def off(a):  # offset arrays: never empty, passed whenever present
+        return a.ctypes.data if a is not None else None
+
+    b = _Batch(G, R, N, int(emb.shape[1]), int(is_bf16), int(emb.shape[1]), T,
+               off(go), off(so), _ptr(sl), off(to), _ptr(emb), _ptr(rw), _ptr(root),
+               _ptr(par), off(gs), off(gt))
+    return b, keep, dict(T=T, N=N, G=G)
+
+
 def run(batch: dict, params: dict | None = None, threads: int = 1, want=None) -> dict:
-    """Run the oracle on a batch (the dict layout of `workloads.make_batch`).
+    """Run the oracle on a batch (the dict layout of `workloads.make_batch`, or
+    the tree layout of `workloads.make_tree_batch`).
 
     Returns a dict of numpy arrays for every output in `want` (default: all).
     """
     lib = _load()
     p = default_params(batch) if params is None else dict(default_params(batch), **params)
-    keep = []
-    go = _c(batch["group_rollout_off"], np.int32)
-    so = _c(batch["rollout_step_off"], np.int32)
-    sl = _c(batch["step_len"], np.int32)
-    to = _c(batch["rollout_token_off"], np.int64)
-    rw = _c(batch["reward"], np.uint8)
-    emb = batch["emb"]
-    is_bf16 = batch["emb_dtype"] == "bf16"
-    emb = _c(emb, np.uint16 if is_bf16 else np.float32)
-    root = batch.get("root_emb")
-    if root is not None:
-        root = _c(root, np.uint16 if is_bf16 else np.float32)
-    keep += [go, so, sl, to, rw, emb, root]
-    G, R, N = len(go) - 1, len(so) - 1, int(emb.shape[0])
-    T = int(to[-1]) if len(to) else 0
-    b = _Batch(G, R, N, int(emb.shape[1]), int(is_bf16), int(emb.shape[1]), T,
-               go.ctypes.data, so.ctypes.data, sl.ctypes.data if N else None, to.ctypes.data,
-               emb.ctypes.data if N else None, rw.ctypes.data if R else None,
-               root.ctypes.data if root is not None else None)
+    b, keep, sizes = _make_batch(batch)
     pp = _Params(p["kappa"], p["w"], p["lambda_eff"], p["std_eps"], int(p["std_ddof"]),
                  int(p["merge_rule"]))
-    sizes = {"T": T, "N": N, "G": G}
     outs = {}
     o = _Outputs()
     for name, dt, per in _OUT_FIELDS:
@@ -138,6 +161,7 @@ def run(batch: dict, params: dict | None = None, threads: int = 1, want=None) ->
             outs[name] = arr
             setattr(o, name, arr.ctypes.data if sizes[per] else None)
     code = lib.oracle_run(ctypes.byref(b), ctypes.byref(pp), ctypes.byref(o), int(threads))
+    del keep
     if code != 0:
         raise OracleError(code)
     return outs
@@ -146,16 +170,7 @@ def run(batch: dict, params: dict | None = None, threads: int = 1, want=None) ->
 def validate(batch: dict) -> int:
     """Return the oracle's validation code (0 = ok) for a batch."""
     lib = _load()
-    go = _c(batch["group_rollout_off"], np.int32)
-    so = _c(batch["rollout_step_off"], np.int32)
-    sl = _c(batch["step_len"], np.int32)
-    to = _c(batch["rollout_token_off"], np.int64)
-    rw = _c(batch["reward"], np.uint8)
-    is_bf16 = batch["emb_dtype"] == "bf16"
-    emb = _c(batch["emb"], np.uint16 if is_bf16 else np.float32)
-    G, R, N = len(go) - 1, len(so) - 1, int(emb.shape[0])
-    T = int(batch.get("total_tokens", to[-1] if len(to) else 0))
-    b = _Batch(G, R, N, int(emb.shape[1]), int(is_bf16), int(emb.shape[1]), T,
-               go.ctypes.data, so.ctypes.data, sl.ctypes.data if N else None, to.ctypes.data,
-               emb.ctypes.data if N else None, rw.ctypes.data if R else None, None)
-    return lib.oracle_validate(ctypes.byref(b))
+    b, keep, _ = _make_batch(batch, with_root=False)
+    code = lib.oracle_validate(ctypes.byref(b))
+    del keep
+    return code

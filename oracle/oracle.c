@@ -19,6 +19,10 @@
  *   Sec. 4.5  A_dual(e) = A_cor(e) + lambda_eff * A_eff(e); every token of an
  *             edge carries the edge's advantage.
  *
+ * The same definitions serve both input layouts (oracle.h): in the chain layout
+ * every rollout is a path from the root, in the tree layout the provenance
+ * tree is given by parent pointers and its leaves are the terminal states.
+ *
  * Readings where the paper leaves a choice open (each is a parameter or a
  * stated constant): std = sqrt(sum (x-mean)^2 / (K - ddof)) and the
  * standardisation divides by (std + eps); correctness groups of one edge and
@@ -50,14 +54,71 @@ static double emb_value(const oracle_batch* b, const void* base, int64_t row, in
   return (double)((const float*)base)[row * b->emb_row_stride + k];
 }
 
+static int validate_embeddings(const oracle_batch* b) {
+  for (int64_t v = 0; v < b->num_states; ++v)
+    for (int k = 0; k < b->d; ++k)
+      if (!isfinite(emb_value(b, b->emb, v, k))) return ORACLE_ERR_NONFINITE;
+  if (b->root_emb)
+    for (int g = 0; g < b->num_groups; ++g)
+      for (int k = 0; k < b->d; ++k)
+        if (!isfinite(emb_value(b, b->root_emb, g, k))) return ORACLE_ERR_NONFINITE;
+  return ORACLE_OK;
+}
+
+/* Tree layout: offsets, parents that precede their children, depth-first
+ * pre-order (the strict descendants of u are exactly the states u+1 ..
+ * u + (number of descendants of u)), one rollout per leaf, token spans. */
+static int validate_tree(const oracle_batch* b) {
+  const int G = b->num_groups, R = b->num_rollouts, N = b->num_states;
+  const int32_t* go = b->group_rollout_off;
+  const int32_t* gs = b->group_state_off;
+  const int64_t* gt = b->group_token_off;
+  if (!go || !gs || !gt) return ORACLE_ERR_INVALID_ARG;
+  if (go[0] != 0 || go[G] != R || gs[0] != 0 || gs[G] != N || gt[0] != 0 || gt[G] != b->total_tokens)
+    return ORACLE_ERR_SHAPE;
+  for (int g = 0; g < G; ++g)
+    if (go[g + 1] < go[g] || gs[g + 1] < gs[g] || gt[g + 1] < gt[g]) return ORACLE_ERR_SHAPE;
+  for (int g = 0; g < G; ++g) {
+    const int s0 = gs[g], n = gs[g + 1] - gs[g];
+    for (int v = 0; v < n; ++v)
+      if (b->parent[s0 + v] < -1 || b->parent[s0 + v] >= v) return ORACLE_ERR_SHAPE;
+    int* desc = calloc(n > 0 ? n : 1, sizeof(int));
+    int* kids = calloc(n > 0 ? n : 1, sizeof(int));
+    if (!desc || !kids) return ORACLE_ERR_NOMEM;
+    for (int v = 0; v < n; ++v) {
+      if (b->parent[s0 + v] >= 0) kids[b->parent[s0 + v]]++;
+      for (int a = b->parent[s0 + v]; a >= 0; a = b->parent[s0 + a]) desc[a]++;
+    }
+    int bad = 0, leaves = 0;
+    for (int v = 0; v < n && !bad; ++v) {
+      leaves += kids[v] == 0;
+      for (int a = b->parent[s0 + v]; a >= 0; a = b->parent[s0 + a])
+        if (!(a < v && v <= a + desc[a])) bad = 1;
+    }
+    free(desc);
+    free(kids);
+    if (bad || leaves != go[g + 1] - go[g]) return ORACLE_ERR_SHAPE;
+    int64_t sum = 0;
+    for (int v = gs[g]; v < gs[g + 1]; ++v) {
+      if (b->step_len[v] < 1) return ORACLE_ERR_SHAPE;
+      sum += b->step_len[v];
+    }
+    if (gt[g + 1] - gt[g] != sum) return ORACLE_ERR_SHAPE;
+  }
+  for (int r = 0; r < R; ++r)
+    if (b->reward[r] > 1) return ORACLE_ERR_BAD_REWARD; /* R(z) in {0,1}, Sec. 4.3 */
+  return validate_embeddings(b);
+}
+
 int oracle_validate(const oracle_batch* b) {
   if (!b) return ORACLE_ERR_INVALID_ARG;
   const int G = b->num_groups, R = b->num_rollouts, N = b->num_states;
   if (G < 0 || R < 0 || N < 0 || b->d <= 0 || b->total_tokens < 0) return ORACLE_ERR_INVALID_ARG;
   if (b->emb_row_stride < b->d) return ORACLE_ERR_INVALID_ARG;
-  if (!b->group_rollout_off || !b->rollout_step_off || !b->rollout_token_off) return ORACLE_ERR_INVALID_ARG;
   if (N > 0 && (!b->step_len || !b->emb)) return ORACLE_ERR_INVALID_ARG;
   if (R > 0 && !b->reward) return ORACLE_ERR_INVALID_ARG;
+  if (b->parent) return validate_tree(b);
+  if (!b->group_rollout_off || !b->rollout_step_off || !b->rollout_token_off) return ORACLE_ERR_INVALID_ARG;
   const int32_t* go = b->group_rollout_off;
   const int32_t* so = b->rollout_step_off;
   const int64_t* to = b->rollout_token_off;
@@ -78,14 +139,7 @@ int oracle_validate(const oracle_batch* b) {
   }
   for (int r = 0; r < R; ++r)
     if (b->reward[r] > 1) return ORACLE_ERR_BAD_REWARD; /* R(z) in {0,1}, Sec. 4.3 */
-  for (int64_t v = 0; v < N; ++v)
-    for (int k = 0; k < b->d; ++k)
-      if (!isfinite(emb_value(b, b->emb, v, k))) return ORACLE_ERR_NONFINITE;
-  if (b->root_emb)
-    for (int g = 0; g < G; ++g)
-      for (int k = 0; k < b->d; ++k)
-        if (!isfinite(emb_value(b, b->root_emb, g, k))) return ORACLE_ERR_NONFINITE;
-  return ORACLE_OK;
+  return validate_embeddings(b);
 }
 
 /* ------------------------------------------------------------ one group -- */
@@ -138,8 +192,10 @@ static double std_of(const double* x, int n, double mean, int ddof) {
 static int run_group(const oracle_batch* b, const oracle_params* p, oracle_outputs* o, int g) {
   const int32_t* go = b->group_rollout_off;
   const int32_t* so = b->rollout_step_off;
+  const int tree = b->parent != NULL;
   const int r0 = go[g], r1 = go[g + 1];
-  const int32_t s0 = so[r0], s1 = so[r1];
+  const int32_t s0 = tree ? b->group_state_off[g] : so[r0];
+  const int32_t s1 = tree ? b->group_state_off[g + 1] : so[r1];
   const int Ng = s1 - s0, n = Ng + 1, d = b->d;
   if (r1 == r0) return ORACLE_OK; /* empty prompt group: nothing to label */
 
@@ -185,20 +241,36 @@ static int run_group(const oracle_batch* b, const oracle_params* p, oracle_outpu
   G.depth[0] = 0;
   G.rollout[0] = -1;
   G.terminal[0] = 0;
-  for (int rr = r0; rr < r1; ++rr) {
-    const int nr = so[rr + 1] - so[rr];
-    for (int h = 1; h <= nr; ++h) {
-      const int i = so[rr] + h - 1 - s0 + 1;
-      G.parent[i] = (h == 1) ? 0 : i - 1;
-      G.depth[i] = h;
-      G.rollout[i] = rr;
-      G.terminal[i] = (h == nr);
+  if (!tree) {
+    for (int rr = r0; rr < r1; ++rr) {
+      const int nr = so[rr + 1] - so[rr];
+      for (int h = 1; h <= nr; ++h) {
+        const int i = so[rr] + h - 1 - s0 + 1;
+        G.parent[i] = (h == 1) ? 0 : i - 1;
+        G.depth[i] = h;
+        G.rollout[i] = rr;
+        G.terminal[i] = (h == nr);
+      }
+    }
+  } else {
+    /* explicit provenance: parents precede their children, so depths follow in order */
+    for (int i = 1; i < n; ++i) {
+      G.parent[i] = b->parent[s0 + i - 1] + 1;
+      G.depth[i] = G.depth[G.parent[i]] + 1;
     }
   }
   for (int i = 1; i < n; ++i) G.child_off[G.parent[i] + 1]++;
   for (int i = 0; i < n; ++i) G.child_off[i + 1] += G.child_off[i];
   for (int i = 0; i < n; ++i) tmp[i] = G.child_off[i];
   for (int i = 1; i < n; ++i) G.child_list[tmp[G.parent[i]]++] = i;
+  if (tree) {
+    /* the terminal states are the leaves; leaf k (in state order) is rollout r0 + k */
+    int k = 0;
+    for (int i = 1; i < n; ++i) {
+      G.terminal[i] = G.child_off[i + 1] == G.child_off[i];
+      G.rollout[i] = G.terminal[i] ? r0 + k++ : -1;
+    }
+  }
 
   /* --- embeddings z_v (Sec. 4.2) --- */
   G.has_root_emb = b->root_emb != NULL;
@@ -349,9 +421,12 @@ static int run_group(const oracle_batch* b, const oracle_params* p, oracle_outpu
     if (o->edge_eff_mask) o->edge_eff_mask[v] = emask[i];
     if (o->cor_group_size) o->cor_group_size[v] = gsize[i];
   }
-  for (int rr = r0; rr < r1; ++rr) {
-    int64_t t = b->rollout_token_off[rr];
-    for (int v = so[rr]; v < so[rr + 1]; ++v) {
+  /* chain layout: each rollout's span holds its steps in order; tree layout: the
+     group's span holds every edge once, in state order */
+  for (int rr = tree ? 0 : r0; rr < (tree ? 1 : r1); ++rr) {
+    int64_t t = tree ? b->group_token_off[g] : b->rollout_token_off[rr];
+    const int v0 = tree ? s0 : so[rr], v1 = tree ? s1 : so[rr + 1];
+    for (int v = v0; v < v1; ++v) {
       const int i = v - s0 + 1;
       const double dual = a_cor[i] + p->lambda_eff * e_eff[i];
       for (int k = 0; k < b->step_len[v]; ++k, ++t) {

@@ -16,6 +16,19 @@
  *   emb [N x d] (bf16 bit patterns or float32, row stride emb_row_stride
  *   elements), root_emb [G x d] optional (NULL: eta on root edges is 0).
  *
+ * Tree layout (branching rollouts, GraphPO Sec. 4.2 layer-by-layer expansion
+ * with a branching schedule; selected by parent != NULL): group g owns states
+ * [group_state_off[g], group_state_off[g+1]) in depth-first pre-order (every
+ * subtree is a contiguous range starting at its top state); parent[v] is the
+ * group-local index of p(v), or -1 when p(v) is the prompt root.  The
+ * terminal states are the leaves; the group's rollouts [group_rollout_off[g],
+ * group_rollout_off[g+1]) are its leaves in state order and reward[r] is the
+ * verifier reward of leaf r.  Every direct edge's tokens appear once (the
+ * objective of Sec. 4.5 sums over direct edges): group g covers tokens
+ * [group_token_off[g], group_token_off[g+1]) and edge v's span follows those
+ * of the group's earlier states.  rollout_step_off and rollout_token_off are
+ * not read.
+ *
  * All outputs are optional (NULL = not wanted); per-token arrays are packed
  * like the input tokens, per-edge arrays are indexed by the state the edge
  * enters.
@@ -49,6 +62,9 @@ typedef struct {
   const void* emb;
   const uint8_t* reward;
   const void* root_emb;      /* optional, same dtype and stride as emb */
+  const int32_t* parent;          /* tree layout: [N] group-local p(v), -1 = root; NULL = chain */
+  const int32_t* group_state_off; /* tree layout: [G+1] */
+  const int64_t* group_token_off; /* tree layout: [G+1] */
 } oracle_batch;
 
 typedef struct {

@@ -16,6 +16,17 @@ itself is the direct edge entering it, GraphPO Sec. 4.2):
                                   or float32
   reward             uint8 [R]    verifier reward R(z) in {0, 1} of each rollout
 
+Tree layout (`make_tree_batch`: branching rollouts expanded layer by layer
+with a branching schedule b_1..b_H, GraphPO Sec. 4.2 and its branching-schedule
+study): each group's states are listed in depth-first pre-order and
+
+  group_rollout_off  int32 [G+1]  the group's leaves (terminal states) = its rollouts
+  group_state_off    int32 [G+1]  states of group g are [off[g], off[g+1])
+  parent             int32 [N]    group-local index of p(v); -1 for the prompt root
+  step_len           int32 [N]    tokens of the edge entering each state
+  group_token_off    int64 [G+1]  every edge's tokens once, in state order
+  reward             uint8 [R]    verifier reward of each leaf, leaves in state order
+
 Recipe per config (seed 20261202 + k, numpy default_rng, drawn group by group,
 rollout by rollout, step by step):
   * every prompt group owns K unit centroids (Gaussian, normalised);
@@ -28,6 +39,11 @@ rollout by rollout, step by step):
   * margin filter: any state with a cross-rollout cosine (computed in fp64 on the
     rounded values) within `margin` of kappa is redrawn until none is left, so
     that the threshold decision is unambiguous at any reasonable precision.
+Trees: the root expands b_1 children; a state at layer h < H ends its branch
+early with probability p_stop, else expands b_{h+1} children; states of layer H
+are terminal.  Structure first (pre-order), then step lengths, embeddings (the
+same centroid recipe with n_max = H), leaf rewards and the margin filter over
+the pairs not in an ancestor-descendant relation.
 """
 from __future__ import annotations
 
@@ -85,7 +101,41 @@ CONFIGS = {
 CONFIG_ORDER = ["tiny", "math", "agentic", "wide", "full"]
 
 
+@dataclasses.dataclass(frozen=True)
+class TreeSpec:
+    name: str
+    groups: int
+    schedule: tuple               # b_1..b_H: children of every expanded state of layer h-1
+    d: int
+    dtype: str                    # "bf16" | "f32"
+    centroids: int
+    sigma: float
+    kappa: float
+    lengths: tuple                # ("per_step", lo, hi): each edge U[lo, hi] tokens
+    rewards: tuple                # as Spec.rewards
+    p_stop: float = 0.1           # a state above the last layer ends its branch early
+    p_share: float = 0.48
+    margin: float = 1e-3
+    w: float = 0.7
+    lambda_eff: float = 1.0
+
+    def scaled(self, groups: Optional[int] = None, **kw) -> "TreeSpec":
+        if groups is not None:
+            kw["groups"] = groups
+        return dataclasses.replace(self, **kw)
+
+
+# Branching rollouts with the schedule {2,5,4,2,2} (the best of the paper's branching
+# study): at most 2 + 10 + 40 + 80 + 160 = 292 states and 160 leaves per prompt.
+TREE_CONFIGS = {
+    "tree": TreeSpec("tree", 128, (2, 5, 4, 2, 2), 1024, "bf16", 32, 0.08, 0.92,
+                     ("per_step", 64, 512), ("beta", 2.0, 2.0)),
+}
+
+
 def config_seed(name: str) -> int:
+    if name in TREE_CONFIGS:
+        return BASE_SEED + len(CONFIG_ORDER) + list(TREE_CONFIGS).index(name)
     return BASE_SEED + CONFIG_ORDER.index(name)
 
 
@@ -209,8 +259,10 @@ def make_batch(spec: Spec, seed: Optional[int] = None, margin_check: bool = True
     )
 
 
-def _margin_filter(rng, spec, cents, n_max, store, exact, cid, roll, depth) -> int:
-    """Redraw states whose cross-rollout cosine lies within `margin` of kappa (in place)."""
+def _margin_filter(rng, spec, cents, n_max, store, exact, cid, roll, depth, comparable=None) -> int:
+    """Redraw states whose cosine with a comparable state lies within `margin` of kappa
+    (in place).  Comparable: another rollout (chain layout), or `comparable(rows)`, a
+    [len(rows), n] boolean matrix."""
     redraws = 0
     rows = np.arange(len(exact))
     for _ in range(1000):
@@ -219,7 +271,10 @@ def _margin_filter(rng, spec, cents, n_max, store, exact, cid, roll, depth) -> i
         Zn = exact / nrm[:, None]
         C = Zn[rows] @ Zn.T
         bad = np.abs(C - spec.kappa) < spec.margin
-        bad &= roll[rows][:, None] != roll[None, :]
+        if comparable is None:
+            bad &= roll[rows][:, None] != roll[None, :]
+        else:
+            bad &= comparable(rows)
         ii, jj = np.nonzero(bad)
         if len(ii) == 0:
             return redraws
@@ -234,7 +289,142 @@ def _margin_filter(rng, spec, cents, n_max, store, exact, cid, roll, depth) -> i
     raise RuntimeError("margin filter did not converge")
 
 
+def _tree_shape(rng, spec: TreeSpec):
+    """Parents (group-local, -1 = root) and depths of one group, in pre-order."""
+    H = len(spec.schedule)
+    par, dep = [], []
+
+    def expand(p, h):  # children of node p (-1 = root) at depth h
+        for _ in range(spec.schedule[h]):
+            v = len(par)
+            par.append(p)
+            dep.append(h + 1)
+            if h + 1 < H and not (rng.random() < spec.p_stop):
+                expand(v, h + 1)
+
+    expand(-1, 0)
+    return np.asarray(par, dtype=np.int32), np.asarray(dep, dtype=np.int64)
+
+
+def subtree_end(parent: np.ndarray) -> np.ndarray:
+    """End (exclusive, group-local) of each state's subtree for a pre-order group."""
+    n = len(parent)
+    end = np.arange(1, n + 1, dtype=np.int64)
+    for v in range(n - 1, -1, -1):
+        if parent[v] >= 0:
+            end[parent[v]] = max(end[parent[v]], end[v])
+    return end
+
+
+def make_tree_batch(spec: TreeSpec, seed: Optional[int] = None, margin_check: bool = True) -> dict:
+    """Draw one tree-layout batch for `spec`.  Deterministic in (spec, seed)."""
+    if seed is None:
+        seed = config_seed(spec.name)
+    rng = np.random.default_rng(seed)
+    H, G, d = len(spec.schedule), spec.groups, spec.d
+    pars, lens, store, planted, rewards, nleaf, nstate = [], [], [], [], [], [], []
+    resampled = 0
+    for g in range(G):
+        cents = _unit(rng, spec.centroids, d)
+        if spec.rewards[0] == "bernoulli":
+            p = spec.rewards[1]
+        else:
+            p = rng.beta(spec.rewards[1], spec.rewards[2])
+        par, dep = _tree_shape(rng, spec)
+        n = len(par)
+        end = subtree_end(par)
+        leaves = int(np.sum(end == np.arange(1, n + 1)))
+        lens.append(rng.integers(spec.lengths[1], spec.lengths[2] + 1, size=n).astype(np.int32))
+        z, cid = _draw_states(rng, spec, cents, dep, H)
+        s, e = _round(spec, z)
+        rewards.extend((rng.random(leaves) < p).astype(np.uint8).tolist())
+        if margin_check:
+            idx = np.arange(n)
+
+            def comparable(rows, end=end, idx=idx):
+                r = rows[:, None]
+                return ((idx[None, :] >= end[r]) | (r >= end[idx][None, :])) & (r != idx[None, :])
+
+            resampled += _margin_filter(rng, spec, cents, H, s, e, cid, None, dep, comparable)
+        pars.append(par)
+        store.append(s)
+        planted.append(cid)
+        nleaf.append(leaves)
+        nstate.append(n)
+    step_len = np.concatenate(lens).astype(np.int32) if lens else np.zeros(0, np.int32)
+    gso = np.zeros(G + 1, dtype=np.int32)
+    gso[1:] = np.cumsum(nstate)
+    gro = np.zeros(G + 1, dtype=np.int32)
+    gro[1:] = np.cumsum(nleaf)
+    gto = np.zeros(G + 1, dtype=np.int64)
+    if len(step_len):
+        gto[1:] = np.cumsum([int(l.astype(np.int64).sum()) for l in lens])
+    emb = np.concatenate(store) if store else np.zeros((0, d))
+    emb = emb.astype(np.uint16 if spec.dtype == "bf16" else np.float32)
+    return dict(
+        spec=spec, seed=seed, layout="tree",
+        group_rollout_off=gro, group_state_off=gso,
+        parent=np.concatenate(pars).astype(np.int32) if pars else np.zeros(0, np.int32),
+        step_len=step_len, group_token_off=gto, total_tokens=int(gto[-1]),
+        emb=np.ascontiguousarray(emb), emb_dtype=spec.dtype,
+        reward=np.asarray(rewards, dtype=np.uint8),
+        planted_centroid=np.concatenate(planted).astype(np.int32) if planted else np.zeros(0, np.int32),
+        kappa=spec.kappa, w=spec.w, lambda_eff=spec.lambda_eff, margin_resampled=resampled,
+    )
+
+
+def is_tree(batch: dict) -> bool:
+    return batch.get("parent") is not None
+
+
+def as_tree(batch: dict) -> dict:
+    """The same chain-layout batch written in the tree layout: each rollout is a path
+    from the root, its last state its leaf; tokens stay where they are."""
+    go, so, to = batch["group_rollout_off"], batch["rollout_step_off"], batch["rollout_token_off"]
+    N = int(so[-1])
+    gso = so[go].astype(np.int32)
+    parent = np.arange(N, dtype=np.int64) - np.repeat(gso[:-1], np.diff(gso)) - 1
+    first = so[:-1]
+    parent[first] = -1
+    out = {k: v for k, v in batch.items() if k not in ("rollout_step_off", "rollout_token_off")}
+    out.update(layout="tree", group_state_off=gso, parent=parent.astype(np.int32),
+               group_token_off=to[go].astype(np.int64), total_tokens=int(to[-1]))
+    return out
+
+
 def sub_batch(batch: dict, groups) -> dict:
+    if is_tree(batch):
+        return _sub_batch_tree(batch, groups)
+    return _sub_batch_chain(batch, groups)
+
+
+def _sub_batch_tree(batch: dict, groups) -> dict:
+    groups = list(groups)
+    go, gs, gt = batch["group_rollout_off"], batch["group_state_off"], batch["group_token_off"]
+    rolls, states, toks = [], [], []
+    ro, so, to = [0], [0], [0]
+    for g in groups:
+        rolls.append(np.arange(go[g], go[g + 1]))
+        states.append(np.arange(gs[g], gs[g + 1]))
+        toks.append((int(gt[g]), int(gt[g + 1])))
+        ro.append(ro[-1] + int(go[g + 1] - go[g]))
+        so.append(so[-1] + int(gs[g + 1] - gs[g]))
+        to.append(to[-1] + int(gt[g + 1] - gt[g]))
+    rolls = np.concatenate(rolls) if rolls else np.zeros(0, dtype=np.int64)
+    states = np.concatenate(states) if states else np.zeros(0, dtype=np.int64)
+    out = dict(batch)
+    out.update(
+        group_rollout_off=np.asarray(ro, dtype=np.int32), group_state_off=np.asarray(so, dtype=np.int32),
+        group_token_off=np.asarray(to, dtype=np.int64), total_tokens=int(to[-1]),
+        parent=batch["parent"][states].astype(np.int32), step_len=batch["step_len"][states].astype(np.int32),
+        emb=np.ascontiguousarray(batch["emb"][states]), reward=batch["reward"][rolls].astype(np.uint8),
+        planted_centroid=batch["planted_centroid"][states], source_groups=groups,
+        source_rollouts=rolls, source_states=states, source_token_spans=toks,
+    )
+    return out
+
+
+def _sub_batch_chain(batch: dict, groups) -> dict:
     """The batch restricted to the listed prompt groups (in the given order).
 
     Groups are independent in the method, so a sub-batch's outputs equal the
@@ -276,12 +466,23 @@ def sub_batch(batch: dict, groups) -> dict:
 
 def token_index(batch: dict, sub: dict) -> np.ndarray:
     """For a sub-batch, the packed token positions of its tokens in the full batch."""
+    if is_tree(sub):
+        parts = [np.arange(a, b) for a, b in sub["source_token_spans"]]
+        return np.concatenate(parts) if parts else np.zeros(0, dtype=np.int64)
     to = batch["rollout_token_off"]
     parts = [np.arange(to[r], to[r + 1]) for r in sub["source_rollouts"]]
     return np.concatenate(parts) if parts else np.zeros(0, dtype=np.int64)
 
 
 def summary(batch: dict) -> dict:
+    if is_tree(batch):
+        go, gs = batch["group_rollout_off"], batch["group_state_off"]
+        G = len(gs) - 1
+        ng = np.diff(gs).astype(int).tolist()
+        return dict(groups=G, rollouts=int(go[-1]), states=int(gs[-1]), tokens=int(batch["group_token_off"][-1]),
+                    d=int(batch["emb"].shape[1]), dtype=batch["emb_dtype"], layout="tree",
+                    max_states_per_group=max(ng) if ng else 0,
+                    mean_states_per_group=(sum(ng) / G) if G else 0.0)
     go, so = batch["group_rollout_off"], batch["rollout_step_off"]
     G = len(go) - 1
     R = len(so) - 1
