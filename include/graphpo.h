@@ -24,6 +24,23 @@
  * order, so rollout_token_off[r+1] - rollout_token_off[r] = sum of its
  * step_len.  rollout_step_off[0] = rollout_token_off[0] = 0.
  *
+ * Tree layout (branching rollouts, selected by parent != NULL; GraphPO Sec. 4.2
+ * expands every active state of layer h-1 into b_h continuations, Algorithm S.1,
+ * and its branching-schedule study): group g owns states [group_state_off[g],
+ * group_state_off[g+1]) listed in depth-first pre-order, so that the subtree of a
+ * state is the contiguous range that starts at it; parent[v] is the group-local
+ * index of the generation predecessor p(v) (always < the state's own local index)
+ * or -1 when p(v) is the prompt root.  The terminal states are the leaves of that
+ * tree; the group's rollouts [group_rollout_off[g], group_rollout_off[g+1]) are
+ * its leaves in state order and reward[r] is the verifier reward of leaf r (so
+ * num_rollouts = number of leaves).  The tokens of every direct edge appear once:
+ * group g covers tokens [group_token_off[g], group_token_off[g+1]) and the span of
+ * the edge entering state v follows those of the group's earlier states, so
+ * group_token_off[g+1] - group_token_off[g] = the group's sum of step_len.
+ * rollout_step_off and rollout_token_off are not read (they may be NULL).  A
+ * chain-layout batch written this way (every rollout a path from the root) gives
+ * the same results.
+ *
  * Memory: every array pointer in gpo_batch and gpo_outputs is DEVICE memory of
  * the current CUDA device, owned by the caller; the library never allocates
  * on the compute path.  The caller also provides the workspace
@@ -35,9 +52,12 @@
  * GPO_MAX_GROUP_STATES) make gpo_compute return an error before anything is
  * enqueued.  Problems that need the device arrays (non-monotone offsets, step
  * lengths that do not tile a rollout's tokens, rewards outside {0,1},
- * non-finite embeddings) are found by the kernels, which then skip the rest
- * of the work; gpo_sync_status returns them.  Outputs are undefined after any
- * error.  No C++ exception, abort or device trap crosses this interface.
+ * non-finite embeddings; in the tree layout also parents that are not earlier
+ * states, an order that is not a depth-first pre-order, or a leaf count that
+ * differs from the group's rollout count) are found by the kernels, which then
+ * skip the rest of the work; gpo_sync_status returns them.  Outputs are
+ * undefined after any error.  No C++ exception, abort or device trap crosses
+ * this interface.
  *
  * Threading: a context may be used by one host thread at a time; calls on
  * one context and one stream are ordered by the stream.  Calls that share a
@@ -102,7 +122,7 @@ typedef struct {
   int32_t emb_dtype;      /* gpo_emb_dtype */
   int32_t max_states_per_group; /* upper bound on any group's state count (sizes the workspace) */
   int64_t emb_row_stride; /* elements between rows; row bytes must be a multiple of 16 */
-  int64_t total_tokens;   /* T = rollout_token_off[R] */
+  int64_t total_tokens;   /* T = rollout_token_off[R] (tree layout: group_token_off[G]) */
   const int32_t* group_rollout_off; /* [G+1] */
   const int32_t* rollout_step_off;  /* [R+1] */
   const int32_t* step_len;          /* [N] */
@@ -111,6 +131,10 @@ typedef struct {
   const uint8_t* reward;            /* [R] verifier rewards in {0,1} */
   const void* root_emb;             /* optional [G x emb_row_stride] prompt embeddings; NULL:
                                        eta on the first step of every rollout is 0 */
+  /* Tree layout only (all three NULL for the chain layout): */
+  const int32_t* parent;            /* [N] group-local index of p(v), -1 = the prompt root */
+  const int32_t* group_state_off;   /* [G+1] states of each group, pre-order */
+  const int64_t* group_token_off;   /* [G+1] packed token span of each group */
 } gpo_batch;
 
 typedef struct {

@@ -45,7 +45,9 @@ class CBatch(ctypes.Structure):
                 ("total_tokens", ctypes.c_int64),
                 ("group_rollout_off", ctypes.c_void_p), ("rollout_step_off", ctypes.c_void_p),
                 ("step_len", ctypes.c_void_p), ("rollout_token_off", ctypes.c_void_p),
-                ("emb", ctypes.c_void_p), ("reward", ctypes.c_void_p), ("root_emb", ctypes.c_void_p)]
+                ("emb", ctypes.c_void_p), ("reward", ctypes.c_void_p), ("root_emb", ctypes.c_void_p),
+                ("parent", ctypes.c_void_p), ("group_state_off", ctypes.c_void_p),
+                ("group_token_off", ctypes.c_void_p)]
 
 
 class COutputs(ctypes.Structure):
@@ -124,16 +126,27 @@ def _c_outputs(out: dict) -> COutputs:
 
 @dataclasses.dataclass
 class Batch:
-    """Device tensors of one batch in chain layout (see include/graphpo.h)."""
+    """Device tensors of one batch (see include/graphpo.h).  Chain layout: every rollout a
+    path from the prompt root (rollout_step_off, rollout_token_off).  Tree layout
+    (`parent` given): states in depth-first pre-order per group, parent = group-local
+    index of p(v) or -1, leaves = rollouts (group_state_off, group_token_off); the
+    chain-only offsets are then None."""
     group_rollout_off: "torch.Tensor"   # int32 [G+1]
-    rollout_step_off: "torch.Tensor"    # int32 [R+1]
+    rollout_step_off: "Optional[torch.Tensor]"   # int32 [R+1] (chain layout)
     step_len: "torch.Tensor"            # int32 [N]
-    rollout_token_off: "torch.Tensor"   # int64 [R+1]
+    rollout_token_off: "Optional[torch.Tensor]"  # int64 [R+1] (chain layout)
     emb: "torch.Tensor"                 # bf16 or fp32 [N, d], unit stride in d
     reward: "torch.Tensor"              # uint8 [R]
     total_tokens: int
     max_states_per_group: int
     root_emb: "Optional[torch.Tensor]" = None
+    parent: "Optional[torch.Tensor]" = None           # int32 [N] (tree layout)
+    group_state_off: "Optional[torch.Tensor]" = None  # int32 [G+1] (tree layout)
+    group_token_off: "Optional[torch.Tensor]" = None  # int64 [G+1] (tree layout)
+
+    @property
+    def is_tree(self):
+        return self.parent is not None
 
     @property
     def num_groups(self):
@@ -141,7 +154,7 @@ class Batch:
 
     @property
     def num_rollouts(self):
-        return self.rollout_step_off.numel() - 1
+        return self.reward.numel() if self.is_tree else self.rollout_step_off.numel() - 1
 
     @property
     def num_states(self):
@@ -160,11 +173,14 @@ class Batch:
                       _ptr(self.group_rollout_off), _ptr(self.rollout_step_off),
                       _ptr(self.step_len) if self.step_len.numel() else None, _ptr(self.rollout_token_off),
                       _ptr(e) if e.numel() else None, _ptr(self.reward) if self.reward.numel() else None,
-                      _ptr(self.root_emb))
+                      _ptr(self.root_emb),
+                      _ptr(self.parent) if self.parent is not None and self.parent.numel() else None,
+                      _ptr(self.group_state_off), _ptr(self.group_token_off))
 
     @staticmethod
     def from_arrays(arrs: dict, device="cuda", pin: bool = False) -> "Batch":
-        """From the numpy dict layout of `workloads.make_batch` (copied to `device`)."""
+        """From the numpy dict layout of `workloads.make_batch` or `workloads.make_tree_batch`
+        (copied to `device`)."""
         import torch
 
         def t(a, dt):
@@ -182,6 +198,14 @@ class Batch:
             root = arrs.get("root_emb")
             root = t(root, np.float32) if root is not None else None
         go = np.asarray(arrs["group_rollout_off"])
+        if arrs.get("parent") is not None:
+            gso = np.asarray(arrs["group_state_off"])
+            gto = np.asarray(arrs["group_token_off"])
+            ng = np.diff(gso)
+            return Batch(t(go, np.int32), None, t(arrs["step_len"], np.int32), None, emb,
+                         t(arrs["reward"], np.uint8), int(gto[-1]) if len(gto) else 0,
+                         int(ng.max()) if len(ng) else 0, root, parent=t(arrs["parent"], np.int32),
+                         group_state_off=t(gso, np.int32), group_token_off=t(gto, np.int64))
         so = np.asarray(arrs["rollout_step_off"])
         ng = so[go[1:]] - so[go[:-1]] if len(go) > 1 else np.zeros(0)
         return Batch(t(go, np.int32), t(so, np.int32), t(arrs["step_len"], np.int32),
@@ -193,7 +217,8 @@ class Batch:
         f = lambda x: None if x is None else x.to(device, non_blocking=non_blocking)
         return Batch(f(self.group_rollout_off), f(self.rollout_step_off), f(self.step_len),
                      f(self.rollout_token_off), f(self.emb), f(self.reward), self.total_tokens,
-                     self.max_states_per_group, f(self.root_emb))
+                     self.max_states_per_group, f(self.root_emb), f(self.parent), f(self.group_state_off),
+                     f(self.group_token_off))
 
 
 class GraphPO:
@@ -333,7 +358,7 @@ class GraphPO:
         dev = torch.device("cuda", torch.cuda.current_device())
         main = torch.cuda.current_stream(dev) if stream is None else stream
         names = ("group_rollout_off", "rollout_step_off", "step_len", "rollout_token_off", "emb", "reward",
-                 "root_emb")
+                 "root_emb", "parent", "group_state_off", "group_token_off")
         host = [getattr(host_batch, n) for n in names]
         key = (dev, tuple(None if t is None else (tuple(t.shape), t.dtype) for t in host))
         if getattr(self, "_stage_key", None) != key:
@@ -353,7 +378,7 @@ class GraphPO:
                 if h is not None and (not piped or names[i] != "emb"):
                     d.copy_(h, non_blocking=True)
             db = Batch(*self._staged[:6], host_batch.total_tokens, host_batch.max_states_per_group,
-                       self._staged[6])
+                       *self._staged[6:])
             if self._stage_out is None:
                 self._stage_out = self.alloc_outputs(db)
             res = self._stage_out["adv"]
@@ -364,11 +389,15 @@ class GraphPO:
                 return out
             ws = self.workspace(db)
             # chunks of groups with about equal numbers of states
-            so = host_batch.rollout_step_off
-            go = host_batch.group_rollout_off
-            to = host_batch.rollout_token_off
-            s_of_g = so[go.long()].tolist()
-            t_of_g = to[go.long()].tolist()
+            if host_batch.is_tree:
+                s_of_g = host_batch.group_state_off.tolist()
+                t_of_g = host_batch.group_token_off.tolist()
+            else:
+                so = host_batch.rollout_step_off
+                go = host_batch.group_rollout_off
+                to = host_batch.rollout_token_off
+                s_of_g = so[go.long()].tolist()
+                t_of_g = to[go.long()].tolist()
             N = s_of_g[-1]
             bounds, g = [0], 0
             for k in range(1, nchunk):

@@ -66,9 +66,14 @@ int64_t max_items_for(int64_t N, int64_t G, int64_t maxn) {
 
 struct Layout {
   size_t status, items, blk_ready, groups, state_meta, rollout_group, nrm2, dotp, rn, root_n2, edge_count,
-      edges, e_adv, e_cor, e_eff, e_mask, tok_start, total;
+      edges, e_adv, e_cor, e_eff, e_mask, tok_start, tree_par, tree_end, tree_own, tree_x, x_n2, x_dot, x_root_n2,
+      total;
   int max_items;
+  bool tree;
 };
+
+// 4-byte words of the tree layout's group-math sums: tree_scratch_words(n) = 23 n + 11 per group
+constexpr int64_t kTreeWordsPerState = 23, kTreeWordsPerGroup = 11;
 
 bool layout(const gpo_batch& b, Layout& L) {
   const int64_t G = b.num_groups, R = b.num_rollouts, N = b.num_states;
@@ -98,6 +103,16 @@ bool layout(const gpo_batch& b, Layout& L) {
   L.e_eff = take(sizeof(float) * N);
   L.e_mask = take(N);
   L.tok_start = take(sizeof(int64_t) * N);
+  L.x_n2 = take(sizeof(float2) * N);
+  L.x_dot = take(sizeof(float2) * N);
+  L.x_root_n2 = take(sizeof(float2) * G);
+  L.tree = b.parent != nullptr;
+  if (L.tree) {
+    L.tree_par = take(sizeof(int) * N);
+    L.tree_end = take(sizeof(int) * N);
+    L.tree_own = take(sizeof(int2) * N);
+    L.tree_x = take(4 * (size_t)(kTreeWordsPerState * N + kTreeWordsPerGroup * G));
+  }
   L.total = o;
   return true;
 }
@@ -122,6 +137,13 @@ Ws workspace_views(void* base, const Layout& L) {
   w.e_eff = reinterpret_cast<float*>(p + L.e_eff);
   w.e_mask = p + L.e_mask;
   w.tok_start = reinterpret_cast<int64_t*>(p + L.tok_start);
+  w.tree_par = L.tree ? reinterpret_cast<int*>(p + L.tree_par) : nullptr;
+  w.tree_end = L.tree ? reinterpret_cast<int*>(p + L.tree_end) : nullptr;
+  w.tree_own = L.tree ? reinterpret_cast<int2*>(p + L.tree_own) : nullptr;
+  w.tree_x = L.tree ? reinterpret_cast<int*>(p + L.tree_x) : nullptr;
+  w.x_n2 = reinterpret_cast<float2*>(p + L.x_n2);
+  w.x_dot = reinterpret_cast<float2*>(p + L.x_dot);
+  w.x_root_n2 = reinterpret_cast<float2*>(p + L.x_root_n2);
   w.max_items = L.max_items;
   return w;
 }
@@ -153,8 +175,14 @@ gpo_status check_batch(gpo_ctx* c, const gpo_batch* b) {
   const int64_t esz = b->emb_dtype == GPO_EMB_BF16 ? 2 : 4;
   if ((b->emb_row_stride * esz) % 16 != 0)
     return set_msg(c, "embedding row bytes must be a multiple of 16"), GPO_ERR_UNSUPPORTED;
-  if (!b->group_rollout_off || !b->rollout_step_off || !b->rollout_token_off)
+  if (b->parent) {
+    if (!b->group_rollout_off || !b->group_state_off || !b->group_token_off)
+      return set_msg(c, "tree layout: an offset array is NULL"), GPO_ERR_INVALID_ARG;
+  } else if (b->group_state_off || b->group_token_off) {
+    return set_msg(c, "group_state_off / group_token_off given without parent"), GPO_ERR_INVALID_ARG;
+  } else if (!b->group_rollout_off || !b->rollout_step_off || !b->rollout_token_off) {
     return set_msg(c, "offset array is NULL"), GPO_ERR_INVALID_ARG;
+  }
   if (b->num_states > 0 && (!b->step_len || !b->emb)) return set_msg(c, "step_len/emb NULL"), GPO_ERR_INVALID_ARG;
   if (b->num_rollouts > 0 && !b->reward) return set_msg(c, "reward NULL"), GPO_ERR_INVALID_ARG;
   if ((b->emb && !aligned(b->emb, 16)) || (b->root_emb && !aligned(b->root_emb, 16)))
@@ -230,6 +258,7 @@ gpo_status gpo_create(gpo_ctx** out, const gpo_params* params) {
     }
   }
   if (setup_sim_tc() != cudaSuccess || setup_groups() != cudaSuccess || setup_fused() != cudaSuccess ||
+      setup_tree_prep() != cudaSuccess ||
       cudaMallocHost(&c->host_status, sizeof(uint32_t) * kStatusWords) != cudaSuccess) {
     cudaGetLastError();
     delete c;
@@ -344,14 +373,16 @@ gpo_status compute_impl(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs*
   if (g1 <= g0) {
     // nothing to compute (a call that only clears the status words)
   } else if (fused) {
+    if (e == cudaSuccess) e = stage("exact_stats", launch_exact_stats(lc, b, sz, ws));
     if (e == cudaSuccess) e = stage("fused", launch_fused(lc, map, map32, b, *out, sz, ws, pp));
   } else {
+  if (e == cudaSuccess && b.parent) e = stage("tree_prep", launch_tree_prep(lc, b, sz, ws));
   if (e == cudaSuccess) e = stage("prep", launch_prep(lc, b, sz, ws));
   if (e == cudaSuccess && sz.N > 0) {
-    // the tcgen05 similarity kernel takes the norms and parent dots from the Gram tiles
-    // themselves; only the prompt-embedding dots need a pass over the rows
-    if (!use_tc) e = stage("row_stats", launch_row_stats(lc, b, sz, ws));
-    else if (b.root_emb) e = stage("root_stats", launch_root_stats(lc, b, sz, ws));
+    // eta takes compensated norms and parent dots (exact_stats); the fp32 norms of the
+    // threshold test come from the Gram tiles (tcgen05) or from row_stats (CUDA cores)
+    e = stage("exact_stats", launch_exact_stats(lc, b, sz, ws));
+    if (e == cudaSuccess && !use_tc) e = stage("row_stats", launch_row_stats(lc, b, sz, ws));
     if (e == cudaSuccess)
       e = stage("similarity", use_tc ? launch_sim_tc(lc, map, b, sz, ws, pp) : launch_sim_simt(lc, b, sz, ws, pp));
     if (e == cudaSuccess) e = stage("groups", launch_groups(lc, b, *out, sz, ws, pp));

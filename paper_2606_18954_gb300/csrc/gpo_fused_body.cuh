@@ -82,12 +82,14 @@ __device__ __forceinline__ void make_plan(int n, Plan& pl) {
   }
 }
 
-// The group's rollout and state ranges; false if they are out of range.
+// The group's rollout and state ranges; false if they are out of range.  Tree layout:
+// the rollouts are the group's leaves and the states come from group_state_off.
 __device__ __forceinline__ bool group_range(const gpo_batch& b, const Sizes& sz, int g, int& r0, int& nr, int& s0,
                                             int& n) {
   const int a = b.group_rollout_off[g], c = b.group_rollout_off[g + 1];
   if (a < 0 || c < a || c > sz.R) return false;
-  const int x = b.rollout_step_off[a], y = b.rollout_step_off[c];
+  const int x = b.parent ? b.group_state_off[g] : b.rollout_step_off[a];
+  const int y = b.parent ? b.group_state_off[g + 1] : b.rollout_step_off[c];
   if (x < 0 || y < x || y > sz.N) return false;
   r0 = a;
   nr = c - a;
@@ -104,28 +106,40 @@ __device__ __forceinline__ bool group_active(const gpo_batch& b, const Sizes& sz
 
 struct __align__(16) GroupSmem {
   int lab[kMaxN];
-  int roll[kMaxN];
+  union {
+    int roll[kMaxN];     // chain layout: rollout of each state (local)
+    int par[kMaxN];      // tree layout: parent of each state (local, -1 = the prompt root)
+  };
   int dep[kMaxN];
   int slen[kMaxN];
-  int rstart[kMaxN + 1];
+  union {
+    int rstart[kMaxN + 1];  // chain layout: local state offsets of the rollouts
+    int cown[kMaxN + 1];    // tree layout: c_own, rewards of the subtree's leaves
+  };
   float n2[kMaxN];
-  float dn[kMaxN];       // <z_i, z_{i+1}>
   alignas(16) float rn[kMaxN];  // 1 / |z_i| (0 for a zero row), read four at a time
   float thr[kMaxN];      // kappa |z_i| (+inf for a zero row or a row that is not tested)
-  int rend[kMaxN];       // end (local, exclusive) of the rollout of state i
-  float root_dot[kMaxN]; // <root, z of the first state of rollout r>
+  int rend[kMaxN];       // end (local, exclusive) of the rollout (tree: of the subtree) of state i;
+                         // the columns right of i that are not its descendants are [rend, n)
   float eadv[kMaxN], ecor[kMaxN], eeff[kMaxN];
-  int64_t tok0[kMaxN + 1];
+  union {
+    int64_t tok0[kMaxN + 1];   // chain layout: token offsets of the rollouts
+    int town[2 * kMaxN + 2];   // tree layout: t_own, leaves of the subtree
+  };
   int64_t tstart[kMaxN];
   uint8_t rew[kMaxN];
   uint8_t emask[kMaxN];
   int flags;             // bit 0: group invalid
   int overflow;          // some warp found more pairs than its part of elist holds
-  float root_n2;
   Plan plan;
   uint32_t elist[kEdgeList];  // linked pairs of the group, kWarpEdges per epilogue warp: i | j << 16
   alignas(16) unsigned char X[group_scratch_sep_bytes(kMaxN)];  // group-math sums (separate layout)
 };
+// Tree layout: the group math's sums (tree_scratch) take elist and X, free once the drain
+// has built the classes; during the set-up elist holds the scan's warp totals.
+constexpr size_t kTreeXOff = offsetof(GroupSmem, elist);
+static_assert(offsetof(GroupSmem, X) + sizeof(GroupSmem::X) - kTreeXOff >= tree_scratch_bytes(kMaxN),
+              "tree scratch does not fit");
 
 struct __align__(8) Ctl {
   uint64_t full[kMaxSlots];
@@ -167,6 +181,106 @@ __device__ __forceinline__ float pick(const uint32_t (&r)[32], int j) {
   return v;
 }
 
+// Tree-layout set-up of group g (Sec. 4.2 branching rollouts: parents precede their
+// children, depth-first pre-order): checks, depth, subtree end, own terminal statistics
+// (Sec. 4.3: c_own / t_own of a state = the rewards / the number of the leaves of its
+// subtree, the leaves in state order being the group's rollouts) and the first token of
+// every edge.  One state per group thread (kGThreads >= kMaxN); every group thread calls
+// it.  An invalid group gets bit 0 of gs->flags (visible to all on return).
+__device__ __forceinline__ void tree_setup(const gpo_batch& b, const Sizes& sz, GroupSmem* gs, int g, int r0, int nr,
+                                           int s0, int n, int gt, int wg, int lane, uint32_t* st) {
+  const int64_t t0 = b.group_token_off[g], t1 = b.group_token_off[g + 1];
+  const int i = gt;
+  int pp = -1;
+  bool bad = gt == 0 && (t0 < 0 || t1 < t0 || t1 > sz.T);
+  if (i < n) {
+    pp = b.parent[s0 + i];
+    const int L = b.step_len[s0 + i];
+    gs->lab[i] = i;
+    gs->slen[i] = L;
+    gs->par[i] = pp;
+    gs->rend[i] = i + 1;
+    gs->cown[i] = 0;
+    gs->town[i] = 0;
+    bad = bad || pp < -1 || pp >= i || L < 1;
+  }
+  bad = bar_any<kBarGroup, kGThreads>(bad);
+  bool bad2 = false;
+  if (!bad && i < n) {
+    if (pp >= 0) {  // pre-order: p(v) lies on the path from the root to the state before v
+      int x = i - 1;
+      while (x > pp) x = gs->par[x];
+      bad2 = x != pp;
+    }
+    int d = 1;
+    for (int x = pp; x >= 0; x = gs->par[x]) {  // par[x] < x: at most i steps
+      ++d;
+      atomicMax(&gs->rend[x], i + 1);
+    }
+    gs->dep[i] = d;
+  }
+  bad = bar_any<kBarGroup, kGThreads>(bad2) || bad;
+  if (bad) {
+    if (gt == 0) {
+      report(st, GPO_ERR_SHAPE, 2, g);
+      atomicOr(&gs->flags, 1);
+    }
+    bar_group();
+    return;
+  }
+  // leaf index and first token: block-wide scans of (is leaf, step length) in state order
+  const bool leaf = i < n && gs->rend[i] == i + 1;
+  int lc = leaf ? 1 : 0;
+  long long tc = i < n ? gs->slen[i] : 0;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, lc, o);
+    const long long z = __shfl_up_sync(0xffffffffu, tc, o);
+    if (lane >= o) {
+      lc += y;
+      tc += z;
+    }
+  }
+  int* wl = reinterpret_cast<int*>(gs->X);             // warp totals (X is free until the group math)
+  long long* wt = reinterpret_cast<long long*>(gs->X + 64);
+  if (lane == 31) {
+    wl[wg] = lc;
+    wt[wg] = tc;
+  }
+  bar_group();
+  int lbase = 0, ltot = 0;
+  long long tbase = 0, ttot = 0;
+  for (int w = 0; w < kGThreads / 32; ++w) {
+    if (w < wg) {
+      lbase += wl[w];
+      tbase += wt[w];
+    }
+    ltot += wl[w];
+    ttot += wt[w];
+  }
+  if (gt == 0 && (ltot != nr || ttot != t1 - t0)) {
+    report(st, GPO_ERR_SHAPE, 2, g);
+    atomicOr(&gs->flags, 1);
+  }
+  if (i < n) gs->tstart[i] = t0 + tbase + tc - gs->slen[i];
+  if (leaf) {
+    const int li = lbase + lc - 1;  // < ltot
+    if (li < nr) {
+      const int rw = b.reward[r0 + li];
+      if (rw > 1) {
+        report(st, GPO_ERR_BAD_REWARD, 2, r0 + li);
+        atomicOr(&gs->flags, 1);
+      } else {
+        for (int x = i; x >= 0; x = gs->par[x]) {
+          atomicAdd(&gs->cown[x], rw);
+          atomicAdd(&gs->town[x], 1);
+        }
+      }
+    }
+  }
+  bar_group();
+}
+
 __global__ void __launch_bounds__(kThreads, kMinBlocks)
     fused_kernel(const __grid_constant__ CUtensorMap zmap, const __grid_constant__ CUtensorMap zmap32, gpo_batch b,
                  gpo_outputs o, Sizes sz, Ws ws, Params p) {
@@ -183,10 +297,16 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
   const int KT = (sz.d + kTileK - 1) / kTileK;
   const float kappa = (float)p.kappa;
 
+  const bool tree = b.parent != nullptr;
   if (blockIdx.x == 0 && threadIdx.x == 0) {
     if (b.group_rollout_off[0] != 0 || b.group_rollout_off[sz.G] != sz.R) report(st, GPO_ERR_SHAPE, 2, 0);
-    if (b.rollout_step_off[0] != 0 || b.rollout_step_off[sz.R] != sz.N) report(st, GPO_ERR_SHAPE, 2, 1);
-    if (b.rollout_token_off[0] != 0 || b.rollout_token_off[sz.R] != sz.T) report(st, GPO_ERR_SHAPE, 2, 2);
+    if (tree) {
+      if (b.group_state_off[0] != 0 || b.group_state_off[sz.G] != sz.N) report(st, GPO_ERR_SHAPE, 2, 1);
+      if (b.group_token_off[0] != 0 || b.group_token_off[sz.G] != sz.T) report(st, GPO_ERR_SHAPE, 2, 2);
+    } else {
+      if (b.rollout_step_off[0] != 0 || b.rollout_step_off[sz.R] != sz.N) report(st, GPO_ERR_SHAPE, 2, 1);
+      if (b.rollout_token_off[0] != 0 || b.rollout_token_off[sz.R] != sz.T) report(st, GPO_ERR_SHAPE, 2, 2);
+    }
   }
   if (threadIdx.x == 0) {
     for (int s = 0; s < kMaxSlots; ++s) {
@@ -334,7 +454,10 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
       const bool in_range = group_range(b, sz, g, r0, nr, s0, n);
       if (!(in_range && n > 0 && n <= kMaxN && n <= sz.maxn && nr > 0 && nr <= n)) {
         if (gt == 0) {
-          if (!in_range || nr > n || (nr > 0 && n == 0)) report(st, GPO_ERR_SHAPE, 2, g);
+          // tree layout: states need leaves, and an empty group has no tokens
+          const bool tree_bad = tree && in_range &&
+                                ((nr == 0 && n > 0) || (n == 0 && b.group_token_off[g + 1] != b.group_token_off[g]));
+          if (!in_range || nr > n || (nr > 0 && n == 0) || tree_bad) report(st, GPO_ERR_SHAPE, 2, g);
           else if (n > kMaxN || n > sz.maxn) report(st, GPO_ERR_UNSUPPORTED, 2, g);
         }
         continue;
@@ -345,6 +468,9 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
         gs->overflow = 0;
       }
 
+      if (tree) {
+        tree_setup(b, sz, gs, g, r0, nr, s0, n, gt, wg, lane, st);
+      } else {
       // ---- validate the group and lay out its states (Sec. 4.2 chain layout)
       for (int r = gt; r <= nr; r += kGThreads) {
         gs->rstart[r] = b.rollout_step_off[r0 + r] - s0;
@@ -381,33 +507,13 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
         }
       }
       bar_group();
+      }
       const bool valid = (gs->flags & 1) == 0;
 
       // ---- drain the accumulator pass by pass (warps 4..15); warps 2..3 fetch
       //      the prompt-embedding dots when a root embedding is given
       bool fail = false;
-      if (!epi) {
-        if (b.root_emb && valid) {
-          const int64_t rb = (int64_t)g * sz.stride;
-          const uint16_t* Rz = reinterpret_cast<const uint16_t*>(b.root_emb);
-          const uint16_t* Z = reinterpret_cast<const uint16_t*>(b.emb);
-          for (int r = wg; r < nr + 1; r += 2) {  // r == nr: |root|^2
-            const int64_t zb = (int64_t)(s0 + gs->rstart[r < nr ? r : 0]) * sz.stride;
-            float acc = 0.f;
-            for (int k = lane; k < sz.d; k += 32) {
-              const float x = __uint_as_float((uint32_t)Rz[rb + k] << 16);
-              const float y = r < nr ? __uint_as_float((uint32_t)Z[zb + k] << 16) : x;
-              acc = fmaf(x, y, acc);
-            }
-#pragma unroll
-            for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
-            if (lane == 0) {
-              if (r < nr) gs->root_dot[r] = acc;
-              else gs->root_n2 = acc;
-            }
-          }
-        }
-      } else {
+      if (epi) {
         const Plan& pl = gs->plan;
         const int te = threadIdx.x - 128;     // 0..383
         const int t128 = q * 32 + lane;       // accumulator lane = row within a 128-row block
@@ -423,8 +529,8 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
           }
           tc_fence_after();
           const int nseg = pl.nseg[pass];
-          // norms and super-diagonal dots from the diagonal segments of this pass (row
-          // block b is read by the quarter's warp b % 3)
+          // squared norms (for the threshold test) from the diagonal of the diagonal segments
+          // of this pass (row block b is read by the quarter's warp b % 3)
 #pragma unroll 1
           for (int si = 0; si < nseg; ++si) {
             const Seg sg = pl.seg[pass][si];
@@ -435,15 +541,8 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
             tmem_ld_32x32b_x32(base + (uint32_t)(q * 32), r);
             tmem_wait_ld();
             const float dg = pick(r, lane);
-            float up = pick(r, lane + 1);
-            if (q * 32 + 32 < sg.len) {
-              tmem_ld_32x32b_x32(base + (uint32_t)(q * 32 + 32), r);
-              tmem_wait_ld();
-              if (lane == 31) up = __uint_as_float(r[0]);
-            }
             if (i < n) {
               gs->n2[i] = dg;
-              if (i + 1 < n) gs->dn[i] = up;
               if (!isfinite(dg)) report(st, GPO_ERR_NONFINITE, 2, s0 + i);
             }
           }
@@ -586,20 +685,11 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
 
       // ---- graph reward and dual-group advantage of every edge
       if (valid) {
-        auto eta = [&](int i) -> float {
-          float e = 0.f, n1 = 0.f, dot = 0.f;
-          if (gs->dep[i] == 1) {
-            if (b.root_emb) {
-              n1 = gs->root_n2;
-              dot = gs->root_dot[gs->roll[i]];
-            }
-          } else {
-            n1 = gs->n2[i - 1];
-            dot = gs->dn[i - 1];
-          }
-          const float n2v = gs->n2[i];
-          if (n1 > 0.f && n2v > 0.f) e = dot * rsqrtf(n1 * n2v);  // cos(p(v), v); a few ulp
-          return e > 0.f ? e : 0.f;
+        // eta(p(v), v) from the compensated row statistics (pairs; see exact_stats_kernel)
+        auto eta = [&](int i) -> float2 {
+          const float2 z = make_float2(0.f, 0.f);
+          const float2 n1 = gs->dep[i] == 1 ? (b.root_emb ? ws.x_root_n2[g] : z) : ws.x_n2[s0 + i - 1];
+          return ff_eta(ws.x_dot[s0 + i], n1, ws.x_n2[s0 + i]);
         };
         auto out = [&](int i, int label, float S, float acor, float E, float dual, unsigned char mask) {
           gs->eadv[i] = dual;
@@ -611,8 +701,20 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
           if (o.class_id) o.class_id[v] = s0 + label;
           if (o.node_score) o.node_score[v] = S;
         };
-        group_advantages<1, true>(n, nr, gs->lab, gs->roll, gs->dep, gs->rstart, gs->rew, group_scratch_sep(gs->X, n),
-                                  p, gt, kGThreads, [] { bar_group(); }, eta, out);
+        if (tree) {
+          auto eta_t = [&](int i) -> float2 {
+            const float2 z = make_float2(0.f, 0.f);
+            const int pp = gs->par[i];
+            const float2 n1 = pp < 0 ? (b.root_emb ? ws.x_root_n2[g] : z) : ws.x_n2[s0 + pp];
+            return ff_eta(ws.x_dot[s0 + i], n1, ws.x_n2[s0 + i]);
+          };
+          group_advantages_tree<1>(n, nr, gs->lab, gs->par, gs->dep, gs->rend, gs->cown, gs->town,
+                                   tree_scratch(smem_raw + kTreeXOff, n), p, gt, kGThreads, [] { bar_group(); },
+                                   eta_t, out);
+        } else {
+          group_advantages<1, true>(n, nr, gs->lab, gs->roll, gs->dep, gs->rstart, gs->rew,
+                                    group_scratch_sep(gs->X, n), p, gt, kGThreads, [] { bar_group(); }, eta, out);
+        }
         // ---- every token of an edge carries the edge's advantage (Sec. 4.5).  State-major:
         //      each half-warp takes a state, its 16 lanes write the whole 16-byte chunks of the
         //      state's token span, then the at most 3 + 3 tokens of its partial first and last

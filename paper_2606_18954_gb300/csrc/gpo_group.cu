@@ -29,21 +29,39 @@ __global__ void __launch_bounds__(1024) groups_kernel(gpo_batch b, gpo_outputs o
   const int n = gi.n, s0 = gi.s0, nr = gi.nr, nt = blockDim.x, tid = threadIdx.x;
   if (nr == 0 || n == 0 || n > sz.maxn) return;
 
+  const bool tree = b.parent != nullptr;
   int* lab = reinterpret_cast<int*>(sm);
   int16_t* roll = reinterpret_cast<int16_t*>(sm + al16(sizeof(int) * (size_t)n));
   int16_t* dep = roll + al16(sizeof(int16_t) * (size_t)n) / sizeof(int16_t);
   int* rstart = reinterpret_cast<int*>(reinterpret_cast<unsigned char*>(dep) + al16(sizeof(int16_t) * (size_t)n));
   uint8_t* rew = reinterpret_cast<uint8_t*>(rstart) + al16(sizeof(int) * (size_t)(n + 1));
   unsigned char* X = rew + al16((size_t)n);
+  // tree layout: parent (roll's place), subtree end and own statistics (rstart's place and
+  // the scratch region), all group-local; the group-math sums live in the workspace
+  int16_t* tpar = roll;
+  int16_t* tend = reinterpret_cast<int16_t*>(rstart);
+  int16_t* tcown = reinterpret_cast<int16_t*>(X);
+  int16_t* ttown = tcown + al16(sizeof(int16_t) * (size_t)n) / sizeof(int16_t);
 
   for (int i = tid; i < n; i += nt) {
     lab[i] = i;
     const int2 m = ws.state_meta[s0 + i];
-    roll[i] = (int16_t)(m.x - gi.r0);
     dep[i] = (int16_t)m.y;
+    if (tree) {
+      const int pp = ws.tree_par[s0 + i];
+      const int2 own = ws.tree_own[s0 + i];
+      tpar[i] = (int16_t)(pp < 0 ? -1 : pp - s0);
+      tend[i] = (int16_t)(ws.tree_end[s0 + i] - s0);
+      tcown[i] = (int16_t)own.x;
+      ttown[i] = (int16_t)own.y;
+    } else {
+      roll[i] = (int16_t)(m.x - gi.r0);
+    }
   }
-  for (int r = tid; r <= nr; r += nt) rstart[r] = b.rollout_step_off[gi.r0 + r] - s0;
-  for (int r = tid; r < nr; r += nt) rew[r] = b.reward[gi.r0 + r];
+  if (!tree) {
+    for (int r = tid; r <= nr; r += nt) rstart[r] = b.rollout_step_off[gi.r0 + r] - s0;
+    for (int r = tid; r < nr; r += nt) rew[r] = b.reward[gi.r0 + r];
+  }
   __syncthreads();
 
   // equivalence classes from the items' spanning forests, in the label forest lab
@@ -57,7 +75,7 @@ __global__ void __launch_bounds__(1024) groups_kernel(gpo_batch b, gpo_outputs o
   const int nit = gi.nblk + gi.noff;  // the group's diagonal items, then its off-diagonal ones
   auto item_at = [&](int k) { return k < gi.nblk ? gi.blk0 + k : gi.off0 + (k - gi.nblk); };
   int* ecnt = reinterpret_cast<int*>(X);
-  const bool cached = (size_t)nit * sizeof(int) <= group_scratch_bytes(n);
+  const bool cached = !tree && (size_t)nit * sizeof(int) <= group_scratch_bytes(n);
   if (cached)
     for (int k = tid; k < nit; k += nt) ecnt[k] = min(ws.edge_count[item_at(k)], kEdgeCap);
   __syncthreads();
@@ -102,22 +120,12 @@ __global__ void __launch_bounds__(1024) groups_kernel(gpo_batch b, gpo_outputs o
     __syncthreads();
   }
 
-  // eta(p(v), v) from the fp32 row statistics; zero rows give 0
-  auto eta = [&](int i) -> float {
+  // eta(p(v), v) from the compensated row statistics (pairs); zero rows give 0
+  const float2 zero2 = make_float2(0.f, 0.f);
+  auto eta = [&](int i) -> float2 {
     const int v = s0 + i;
-    float e = 0.f, n1 = 0.f, dot = 0.f;
-    if (dep[i] == 1) {
-      if (b.root_emb) {
-        n1 = ws.root_n2[g];
-        dot = ws.dotp[v];
-      }
-    } else {
-      n1 = ws.nrm2[v - 1];
-      dot = ws.dotp[v];
-    }
-    const float n2 = ws.nrm2[v];
-    if (n1 > 0.f && n2 > 0.f) e = dot * rsqrtf(n1 * n2);  // cos(p(v), v); a few ulp
-    return e > 0.f ? e : 0.f;
+    const float2 n1 = dep[i] == 1 ? (b.root_emb ? ws.x_root_n2[g] : zero2) : ws.x_n2[v - 1];
+    return ff_eta(ws.x_dot[v], n1, ws.x_n2[v]);
   };
   auto out = [&](int i, int label, float S, float acor, float E, float dual, unsigned char mask) {
     const int v = s0 + i;
@@ -129,6 +137,19 @@ __global__ void __launch_bounds__(1024) groups_kernel(gpo_batch b, gpo_outputs o
     if (o.class_id) o.class_id[v] = s0 + label;
     if (o.node_score) o.node_score[v] = S;
   };
+  if (tree) {
+    auto eta_t = [&](int i) -> float2 {
+      const int v = s0 + i;
+      const float2 n1 = tpar[i] < 0 ? (b.root_emb ? ws.x_root_n2[g] : zero2) : ws.x_n2[s0 + tpar[i]];
+      return ff_eta(ws.x_dot[v], n1, ws.x_n2[v]);
+    };
+    static_assert(tree_scratch_words(1) == 23 + 11 && tree_scratch_words(2) == 2 * 23 + 11,
+                  "workspace layout of the tree sums");
+    group_advantages_tree<kPer, int16_t>(n, nr, lab, tpar, dep, tend, tcown, ttown,
+                                         tree_scratch(ws.tree_x + (size_t)23 * s0 + (size_t)11 * g, n), p, tid, nt,
+                                         [] { __syncthreads(); }, eta_t, out);
+    return;  // the tree prep kernel wrote the first token of every edge
+  }
   __shared__ int s_rootc;
   group_advantages<kPer, false, int16_t>(n, nr, lab, roll, dep, rstart, rew, group_scratch_shared(X, n, &s_rootc), p,
                                          tid, nt, [] { __syncthreads(); }, eta, out);

@@ -86,6 +86,33 @@ __device__ __forceinline__ long long div_round(long long a, int k) {
 
 __host__ __device__ constexpr size_t al16(size_t x) { return (x + 15) & ~size_t(15); }
 
+// c + w a as a float pair (a, c integers below 2^24; w = wh + wl, the fp64 parameter to
+// about 2^-48): TwoProduct of wh a, TwoSum with c.
+__device__ __forceinline__ float2 lin_ff(int c, int a, float wh, float wl) {
+  const float fa = (float)a;
+  const float p = wh * fa;
+  const float e = fmaf(wh, fa, -p);
+  float h, t;
+  two_sum((float)c, p, h, t);
+  return make_float2(h, t + e + wl * fa);
+}
+
+// Eq. (combain) as a float pair: (c_own + w (C_Q - c_own)) / (t_own + w (T_Q - t_own)).
+// Numerator and denominator come out of the same operations, so a class whose leaves
+// share one reward gets exactly 1 (or exactly 0).
+__device__ __forceinline__ float2 score_ff(int c, int t, int C, int T, float wh, float wl) {
+  return ff_div(lin_ff(c, C - c, wh, wl), lin_ff(t, T - t, wh, wl));
+}
+
+// r_step = (S(v) - S(p(v))) (1 - eta) on the 2^-50 grid (|r| <= 1), from pair-valued
+// scores and eta: the pair arithmetic keeps r to ~2^-46 relative, well below the grid
+// of the exact group sums that follow.
+__device__ __forceinline__ long long step_reward_fixed(float2 S, float2 Sp, float2 eta) {
+  const float2 d = ff_add(S, make_float2(-Sp.x, -Sp.y));
+  const float2 r = ff_mul(d, ff_add(make_float2(1.0f, 0.0f), make_float2(-eta.x, -eta.y)));
+  return __float2ll_rn(r.x * 0x1p50f) + __float2ll_rn(r.y * 0x1p50f);
+}
+
 // Scratch arrays of group_advantages.  Class sums are indexed by the class root
 // (a local state index), correctness-group sums by the key (the class of the
 // parent, or n for the prompt root); the route sums reuse the class arrays.
@@ -165,7 +192,7 @@ __device__ __forceinline__ GroupScratch group_scratch_shared(unsigned char* X, i
 //   rew     [nr] rewards
 //   sc      scratch: separate layout zeroed by the caller (kZeroed), or the
 //           shared layout (!kZeroed)
-//   eta(i)  eta(p(v), v) of local state i (fp32, already clamped at 0)
+//   eta(i)  eta(p(v), v) of local state i as a float pair (already clamped at 0)
 //   out(i, label, S, acor, E, dual, mask) is called once per state by its owner
 //   sync()  barrier over the nt threads
 //
@@ -180,6 +207,7 @@ __device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const 
                                                  const int* rstart, const uint8_t* rew, const GroupScratch& sc,
                                                  const Params& p, int tid, int nt, Sync sync, Eta eta, Out out) {
   const float w = (float)p.w, eps = (float)p.eps;
+  const float wl = (float)(p.w - (double)w);  // w = w + wl to ~2^-48
   // ---- phase A: class sums C_Q (rewards), |Q|, sum l, sum l^2
   if (!kZeroed) {
     for (int i = tid; i < n; i += nt) {
@@ -207,22 +235,24 @@ __device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const 
   }
   for (int r = tid; r < nr; r += nt) atomicAdd(sc.rootc, (int)rew[r]);
   sync();
-  const float S_root = (float)*sc.rootc / (float)nr;
-  float S[kPer], aeff[kPer], r[kPer];
+  const float2 S_root = ff_div(make_float2((float)*sc.rootc, 0.f), make_float2((float)nr, 0.f));
+  float S[kPer], aeff[kPer];
+  long long rf[kPer];
   int key[kPer];
   bool route_end[kPer];
 #pragma unroll
   for (int k = 0; k < kPer; ++k) {
     const int i = tid + k * nt;
-    S[k] = aeff[k] = r[k] = 0.f;
+    S[k] = aeff[k] = 0.f;
+    rf[k] = 0;
     key[k] = n;
     route_end[k] = false;
     if (i >= n) continue;
     const int L = lb[k], Q = sc.ccnt[L], d = dep[i], c = rew[roll[i]];
-    // Eq. (combain): (c_own + w sum_{q != v} c_own(q)) / (t_own + w sum_{q != v} t_own(q)), t_own = 1.
-    // Correctly rounded, with numerator and denominator formed by the same fma, so that a
-    // class whose members share one reward gets S exactly 0 or 1 (as the exact formula).
-    S[k] = fmaf(w, (float)(sc.csum[L] - c), (float)c) / fmaf(w, (float)(Q - 1), 1.0f);
+    // Eq. (combain): (c_own + w sum_{q != v} c_own(q)) / (t_own + w sum_{q != v} t_own(q)), t_own = 1,
+    // as a float pair (a class whose members share one reward gets S exactly 0 or 1)
+    const float2 Sv = score_ff(c, 1, sc.csum[L], Q, w, wl);
+    S[k] = Sv.x;
     if (Q >= 2) {
       // Sbar_Q = mean of S over Q = C_Q / |Q| (every member has t_own = 1);
       // sum (l - mean)^2 = (Q sum l^2 - (sum l)^2) / Q with an exact integer numerator;
@@ -237,15 +267,13 @@ __device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const 
       route_end[k] = true;
       aeff[k] = g * (float)(sc.lsum[L] - Q * d);
     }
-    float Sp;
-    if (d == 1) {
-      Sp = S_root;
-    } else {
+    float2 Sp = S_root;
+    if (d != 1) {
       const int Lp = lab[i - 1];  // parent: the previous state of the same rollout (same reward c)
-      Sp = fmaf(w, (float)(sc.csum[Lp] - c), (float)c) / fmaf(w, (float)(sc.ccnt[Lp] - 1), 1.0f);
+      Sp = score_ff(c, 1, sc.csum[Lp], sc.ccnt[Lp], w, wl);
       key[k] = Lp;
     }
-    r[k] = (S[k] - Sp) * (1.0f - eta(i));
+    rf[k] = step_reward_fixed(Sv, Sp, eta(i));
   }
 
   // ---- phase B: correctness groups, key = class of p(v), n = the prompt root
@@ -254,13 +282,10 @@ __device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const 
     for (int i = tid; i < (kKeyWords) * (n + 1); i += nt) reinterpret_cast<int*>(sc.kcnt)[i] = 0;
     sync();
   }
-  long long rf[kPer];
 #pragma unroll
   for (int k = 0; k < kPer; ++k) {
-    rf[k] = 0;
     if (tid + k * nt < n) {
       // |r| <= 1 and a group holds at most 4096 edges: a 2^50 fixed point cannot overflow
-      rf[k] = __float2ll_rn(r[k] * 0x1p50f);
       atomicAdd(&sc.kcnt[key[k]], 1);
       red_chunks<kSumWords, 18>(&sc.ksum[kSumWords * key[k]], (unsigned long long)(rf[k] + (1ll << 50)));
     }
@@ -338,6 +363,237 @@ __device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const 
         }
         carry += tot;
         ccov = ccov || cb != 0;
+      }
+    }
+  }
+  sync();
+  const float lam = (float)p.lambda_eff;
+#pragma unroll
+  for (int k = 0; k < kPer; ++k) {
+    const int i = tid + k * nt;
+    if (i < n) out(i, lb[k], S[k], acor[k], sc.E[i], fmaf(lam, sc.E[i], acor[k]), sc.cov[i]);
+  }
+  sync();
+}
+
+// ---------------------------------------------------------------------------------
+// Tree layout (branching rollouts, parent pointers, states in depth-first pre-order):
+// the same quantities as group_advantages, with the provenance tree's own statistics
+//   c_own(v) = sum of R(z) over the leaves z of v's subtree, t_own(v) = their number
+//             (bottom-up along direct edges, Sec. 4.3), given by the caller;
+//   S(v)      (c_own + w (C_Q - c_own)) / (t_own + w (T_Q - t_own)), class sums
+//             C_Q, T_Q; S(root) = sum R / number of leaves                  (Eq. (combain))
+//   r_step    (S(v) - S(p(v))) (1 - eta(p(v), v))                          (Sec. 4.3)
+//   A_cor     edges grouped by the class of p(v), as in the chain layout    (Sec. 4.4)
+//   A_eff     per class |Q| >= 2: Sbar_Q (mean d - d_v) / (std(d) + eps) (the z-score of
+//             -l_v, l_v = d(v) - d(a_Q), does not depend on d(a_Q)); routed onto every
+//             edge of a_Q -> v, a_Q the deepest state that is a strict ancestor of every
+//             member.  In pre-order the lowest common ancestor of a set is that of its
+//             smallest and largest index, so a_Q follows from the class's label L (its
+//             smallest member) and its largest member h: walk up from L to the first
+//             state whose subtree reaches h; that state is a_Q unless it is L itself
+//             (then L is an ancestor of every member and a_Q = p(L)).
+//             The edge entering x carries the sum of A_eff(j) over the members j of
+//             its subtree whose a_Q lies strictly above x, summed in index order by one
+//             warp per x (work = sum of the depths; deterministic order).
+//   A_dual    A_cor + lambda_eff * routed A_eff                             (Sec. 4.5)
+
+// Sums of the tree variant.  Class arrays are indexed by the class root, key arrays by
+// the class of p(v) (n for the prompt root), both over n (+1) entries of the group.
+struct TreeScratch {
+  int* ccnt;        // [n]    |Q|
+  int* csum;        // [n]    C_Q = sum of the members' c_own
+  int* tsum;        // [n]    T_Q = sum of the members' t_own
+  int* lsum;        // [n]    sum of the members' depths
+  unsigned* l2;     // [n][2] sum of the squared depths, 2 x 13-bit chunks
+  int* hi;          // [n]    largest member
+  unsigned* ssum;   // [n][3] sum of S on the 2^-40 grid, 3 x 14-bit chunks
+  int* aqd;         // [n]    depth of a_Q
+  int* kcnt;        // [n+1]  edges per correctness group
+  unsigned* ksum;   // [n+1][kSumWords]
+  unsigned* kqh;    // [n+1][kSqhWords]
+  unsigned* kql;    // [n+1][kSqlWords]
+  float* aeff;      // [n]    A_eff of each state (0 unless |Q| >= 2)
+  int* rdep;        // [n]    depth of a_Q of the state's class, or a large value without a route
+  float* E;         // [n]    routed A_eff (over ccnt, written once the class sums are read)
+  unsigned char* cov;  // [n] covered by a route (over csum)
+  int* rootc;       // [1]    sum of the group's rewards
+  int nzero;        // words from ccnt that start at zero (class and key sums, rootc)
+};
+
+constexpr int kTreeClassWords = 11;
+constexpr int kTreeStateWords = 2;
+
+__host__ __device__ constexpr size_t tree_scratch_words(int n) {
+  return (size_t)kTreeClassWords * n + (size_t)kKeyWords * (n + 1) + 1 + (size_t)kTreeStateWords * n;
+}
+__host__ __device__ constexpr size_t tree_scratch_bytes(int n) { return al16(4 * tree_scratch_words(n)); }
+
+// Carves a tree scratch of tree_scratch_bytes(n) bytes (4-byte aligned).
+__device__ __forceinline__ TreeScratch tree_scratch(void* base, int n) {
+  TreeScratch t;
+  int* w = reinterpret_cast<int*>(base);
+  t.ccnt = w;
+  t.csum = w + n;
+  t.tsum = w + 2 * n;
+  t.lsum = w + 3 * n;
+  t.l2 = reinterpret_cast<unsigned*>(w + 4 * n);
+  t.hi = w + 6 * n;
+  t.ssum = reinterpret_cast<unsigned*>(w + 7 * n);
+  t.aqd = w + 10 * n;
+  int* k = w + kTreeClassWords * n;
+  t.kcnt = k;
+  t.ksum = reinterpret_cast<unsigned*>(k + (n + 1));
+  t.kqh = t.ksum + kSumWords * (n + 1);
+  t.kql = t.kqh + kSqhWords * (n + 1);
+  t.rootc = k + kKeyWords * (n + 1);
+  t.aeff = reinterpret_cast<float*>(t.rootc + 1);
+  t.rdep = reinterpret_cast<int*>(t.aeff + n);
+  t.E = reinterpret_cast<float*>(t.ccnt);
+  t.cov = reinterpret_cast<unsigned char*>(t.csum);
+  t.nzero = kTreeClassWords * n + kKeyWords * (n + 1) + 1;
+  return t;
+}
+
+// One group, nt cooperating threads (a multiple of 32; tid = thread index, lane = tid & 31
+// must be the hardware lane), kPer * nt >= n.
+//   lab    [n] union-find forest on entry (lab[x] <= x), class labels on exit
+//   par    [n] local parent, -1 for the prompt root (par[x] < x)
+//   dep    [n] depth (1 = child of the root);  end [n] local end of the subtree
+//   cown, town [n] own terminal statistics;  nleaf = number of leaves (> 0)
+//   sc     tree scratch (zeroed here), eta(i), out(...) and sync() as in group_advantages
+template <int kPer, class IdxT, class Sync, class Eta, class Out>
+__device__ __forceinline__ void group_advantages_tree(int n, int nleaf, int* lab, const IdxT* par, const IdxT* dep,
+                                                      const IdxT* end, const IdxT* cown, const IdxT* town,
+                                                      const TreeScratch& sc, const Params& p, int tid, int nt,
+                                                      Sync sync, Eta eta, Out out) {
+  const float w = (float)p.w, eps = (float)p.eps;
+  const float wl = (float)(p.w - (double)w);
+  for (int i = tid; i < sc.nzero; i += nt) sc.ccnt[i] = 0;
+  sync();
+  // ---- phase A: class sums
+  int lb[kPer];
+#pragma unroll
+  for (int k = 0; k < kPer; ++k) {
+    const int i = tid + k * nt;
+    lb[k] = 0;
+    if (i < n) {
+      lb[k] = uf_find(lab, i);
+      lab[i] = lb[k];
+      const int d = dep[i];
+      atomicAdd(&sc.ccnt[lb[k]], 1);
+      atomicAdd(&sc.csum[lb[k]], (int)cown[i]);
+      atomicAdd(&sc.tsum[lb[k]], (int)town[i]);
+      atomicAdd(&sc.lsum[lb[k]], d);
+      red_chunks<2, 13>(&sc.l2[2 * lb[k]], (unsigned long long)d * d);
+      atomicMax(&sc.hi[lb[k]], i);
+      if (par[i] < 0) atomicAdd(sc.rootc, (int)cown[i]);
+    }
+  }
+  sync();
+  // ---- phase A2: S, the parent's S, r_step; S and r into their sums; a_Q per class
+  const float2 S_root = ff_div(make_float2((float)*sc.rootc, 0.f), make_float2((float)nleaf, 0.f));
+  float S[kPer];
+  int key[kPer];
+  long long rf[kPer];
+#pragma unroll
+  for (int k = 0; k < kPer; ++k) {
+    const int i = tid + k * nt;
+    S[k] = 0.f;
+    key[k] = n;
+    rf[k] = 0;
+    if (i >= n) continue;
+    const int L = lb[k], c = cown[i], t = town[i];
+    // Eq. (combain) as a float pair: a class whose leaves share one reward gets S exactly 0 or 1
+    const float2 Sv = score_ff(c, t, sc.csum[L], sc.tsum[L], w, wl);
+    S[k] = Sv.x;
+    const int pp = par[i];
+    float2 Sp = S_root;
+    if (pp >= 0) {
+      const int Lp = lab[pp];  // the parent's S, recomputed alike
+      Sp = score_ff(cown[pp], town[pp], sc.csum[Lp], sc.tsum[Lp], w, wl);
+      key[k] = Lp;
+    }
+    rf[k] = step_reward_fixed(Sv, Sp, eta(i));
+    red_chunks<3, 14>(&sc.ssum[3 * L],
+                      (unsigned long long)(__float2ll_rn(Sv.x * 0x1p40f) + __float2ll_rn(Sv.y * 0x1p40f)));
+    atomicAdd(&sc.kcnt[key[k]], 1);
+    red_chunks<kSumWords, 18>(&sc.ksum[kSumWords * key[k]], (unsigned long long)(rf[k] + (1ll << 50)));
+    if (i == L && sc.ccnt[L] >= 2) {
+      const int h = sc.hi[L];
+      int x = L;
+      while (x >= 0 && end[x] <= h) x = par[x];
+      sc.aqd[L] = x == L ? (int)dep[L] - 1 : (x < 0 ? 0 : (int)dep[x]);
+    }
+  }
+  sync();
+  // ---- phase B2: exact group means and squared deviations; A_eff per state
+  float dv[kPer];
+#pragma unroll
+  for (int k = 0; k < kPer; ++k) {
+    const int i = tid + k * nt;
+    dv[k] = 0.f;
+    if (i >= n) continue;
+    const int cnt = sc.kcnt[key[k]];
+    const long long tot =
+        (long long)(sum_chunks<kSumWords, 18>(&sc.ksum[kSumWords * key[k]]) - ((unsigned long long)cnt << 50));
+    const long long mean = div_round(tot, cnt);
+    dv[k] = (float)(rf[k] - mean) * 0x1p-50f;
+    sq_add(&sc.kqh[kSqhWords * key[k]], &sc.kql[kSqlWords * key[k]], dv[k] * dv[k]);
+    const int L = lb[k], Q = sc.ccnt[L], d = dep[i];
+    float a = 0.f;
+    int rd = 0x7fffffff;
+    if (Q >= 2) {
+      // Sbar_Q = sum S / Q; sum (d - mean)^2 = (Q sum d^2 - (sum d)^2) / Q (exact numerator);
+      // A_eff = Sbar (mean d - d_v) / (sd + eps) = g (sum d - Q d_v), g = sum S / (Q^2 (sd + eps))
+      const long long ls = sc.lsum[L];
+      const float num = (float)((long long)Q * (long long)sum_chunks<2, 13>(&sc.l2[2 * L]) - ls * ls);
+      const float var = __fdividef(num, (float)Q * (float)(Q - p.ddof));
+      const float sd = var > 0.f ? var * rsqrtf(var) : 0.f;
+      const float ssum = (float)sum_chunks<3, 14>(&sc.ssum[3 * L]) * 0x1p-40f;
+      const float g = __fdividef(ssum, (float)Q * (float)Q * (sd + eps));
+      a = g * (float)(ls - (long long)Q * d);
+      rd = sc.aqd[L];
+    }
+    sc.aeff[i] = a;
+    sc.rdep[i] = rd;
+  }
+  sync();
+  // ---- phase B3: A_cor; phase C: routed A_eff (class sums are dead: E and cov overlay them)
+  float acor[kPer];
+#pragma unroll
+  for (int k = 0; k < kPer; ++k) {
+    acor[k] = 0.f;
+    const int K = key[k];
+    if (tid + k * nt < n && sc.kcnt[K] >= 2) {
+      const int cnt = sc.kcnt[K];
+      const long long qh = (long long)sum_chunks<kSqhWords, 13>(&sc.kqh[kSqhWords * K]);
+      const long long ql =
+          (long long)(sum_chunks<kSqlWords, 14>(&sc.kql[kSqlWords * K]) - ((unsigned long long)cnt << 39));
+      const float ss = (float)qh * 0x1p-36f + (float)ql * 0x1p-76f;
+      const float var = __fdividef(ss, (float)(cnt - p.ddof));
+      const float sd = var > 0.f ? var * rsqrtf(var) : 0.f;
+      acor[k] = dv[k] * __fdividef(1.0f, sd + eps);
+    }
+  }
+  {
+    const int lane = tid & 31, nw = nt >> 5;
+    for (int x = tid >> 5; x < n; x += nw) {
+      const int dx = dep[x], e = end[x];
+      float s = 0.f;
+      bool c = false;
+      for (int j = x + lane; j < e; j += 32) {
+        if (sc.rdep[j] < dx) {
+          s += sc.aeff[j];
+          c = true;
+        }
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+      c = __any_sync(0xffffffffu, c);
+      if (lane == 0) {
+        sc.E[x] = s;
+        sc.cov[x] = c ? 1 : 0;
       }
     }
   }

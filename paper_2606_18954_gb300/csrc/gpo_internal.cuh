@@ -63,6 +63,15 @@ struct Ws {
   float* e_eff;          // [N] routed efficiency advantage per edge
   uint8_t* e_mask;       // [N]
   int64_t* tok_start;    // [N] first token of each edge
+  // tree layout only (null otherwise)
+  int* tree_par;         // [N] parent (global index, -1 = the prompt root)
+  int* tree_end;         // [N] end of the state's subtree (global, exclusive)
+  int2* tree_own;        // [N] {c_own, t_own}: rewards and number of the leaves of the subtree
+  int* tree_x;           // [23 N + 11 G] group-math sums, tree_scratch of group g at 23 s0 + 11 g
+  // accurate row statistics (unevaluated float pairs hi + lo, see exact_stats_kernel)
+  float2* x_n2;          // [N] |z_v|^2
+  float2* x_dot;         // [N] <z_{p(v)}, z_v> (prompt embedding for a root child, 0 without one)
+  float2* x_root_n2;     // [G] |prompt embedding|^2
   int max_items;
 };
 
@@ -307,6 +316,75 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
 }
 
+// ------------------------------------------------------------------ float-float arithmetic
+// Unevaluated pairs hi + lo of fp32 numbers carry about 48 significant bits.  The
+// error-free transformations are Knuth's TwoSum and the fma-based TwoProduct (Ogita,
+// Rump and Oishi, "Accurate sum and dot product", SIAM J. Sci. Comput. 2005); the
+// pair operations follow Dekker's double-length arithmetic.  They are used where the
+// standardisation of Sec. 4.4 amplifies rounding: the cosine eta(p(v), v) and the
+// step reward r_step of nearly equal edges.
+
+// s + e = a + b exactly.
+__device__ __forceinline__ void two_sum(float a, float b, float& s, float& e) {
+  s = a + b;
+  const float bb = s - a;
+  e = (a - (s - bb)) + (b - bb);
+}
+
+// Adds x to the pair (hi, lo) (compensated summation: the rounding error of every
+// addition is collected in lo).
+__device__ __forceinline__ void ff_acc(float& hi, float& lo, float x) {
+  float s, e;
+  two_sum(hi, x, s, e);
+  hi = s;
+  lo += e;
+}
+
+// Pair sum (a.x + a.y) + (b.x + b.y).
+__device__ __forceinline__ float2 ff_add(float2 a, float2 b) {
+  float s, e;
+  two_sum(a.x, b.x, s, e);
+  e += a.y + b.y;
+  float h, l;
+  two_sum(s, e, h, l);
+  return make_float2(h, l);
+}
+
+// Pair product a * b.
+__device__ __forceinline__ float2 ff_mul(float2 a, float2 b) {
+  const float p = a.x * b.x;
+  const float e = fmaf(a.x, b.x, -p) + (a.x * b.y + a.y * b.x);
+  float h, l;
+  two_sum(p, e, h, l);
+  return make_float2(h, l);
+}
+
+// Pair quotient a / b (b.x > 0): one correction step of the fp32 quotient.
+__device__ __forceinline__ float2 ff_div(float2 a, float2 b) {
+  const float q = a.x / b.x;
+  const float r = fmaf(-q, b.x, a.x) + a.y - q * b.y;
+  float h, l;
+  two_sum(q, r / b.x, h, l);
+  return make_float2(h, l);
+}
+
+// Pair square root (a.x > 0): one correction step of the fp32 root.
+__device__ __forceinline__ float2 ff_sqrt(float2 a) {
+  const float s = sqrtf(a.x);
+  const float e = fmaf(-s, s, a.x) + a.y;
+  float h, l;
+  two_sum(s, e / (2.0f * s), h, l);
+  return make_float2(h, l);
+}
+
+// eta = max(0, dot / sqrt(np nv)) as a pair, from pair-valued dot and squared norms;
+// 0 when a norm is zero (a zero embedding has similarity 0 with every state).
+__device__ __forceinline__ float2 ff_eta(float2 dot, float2 np, float2 nv) {
+  if (!(np.x > 0.f) || !(nv.x > 0.f)) return make_float2(0.f, 0.f);
+  if (dot.x + dot.y <= 0.f) return make_float2(0.f, 0.f);
+  return ff_div(dot, ff_sqrt(ff_mul(np, nv)));
+}
+
 // ------------------------------------------------------------------ token spans
 
 // One warp writes value v to dst[ts, te): 16-byte stores in the aligned middle,
@@ -337,6 +415,9 @@ struct LaunchCtx {
 };
 
 cudaError_t launch_prep(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws);
+cudaError_t launch_exact_stats(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws);
+cudaError_t launch_tree_prep(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws);
+cudaError_t setup_tree_prep();
 cudaError_t launch_row_stats(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws);
 cudaError_t launch_root_stats(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws);
 cudaError_t launch_sim_tc(const LaunchCtx& lc, const CUtensorMap& map, const gpo_batch& b, const Sizes& sz,

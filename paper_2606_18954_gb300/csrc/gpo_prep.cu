@@ -60,11 +60,17 @@ __global__ void __launch_bounds__(kPlanThreads) prep_kernel(gpo_batch b, Sizes s
   const int32_t* go = b.group_rollout_off;
   const int32_t* so = b.rollout_step_off;
   const int64_t* to = b.rollout_token_off;
+  const bool tree = b.parent != nullptr;  // tree layout: tree_prep_kernel checks the groups and lays out their states
 
   if (tid == 0) {
     if (go[0] != 0 || go[sz.G] != sz.R) report(st, GPO_ERR_SHAPE, 0, 0);
-    if (so[0] != 0 || so[sz.R] != sz.N) report(st, GPO_ERR_SHAPE, 0, 1);
-    if (to[0] != 0 || to[sz.R] != sz.T) report(st, GPO_ERR_SHAPE, 0, 2);
+    if (tree) {
+      if (b.group_state_off[0] != 0 || b.group_state_off[sz.G] != sz.N) report(st, GPO_ERR_SHAPE, 0, 1);
+      if (b.group_token_off[0] != 0 || b.group_token_off[sz.G] != sz.T) report(st, GPO_ERR_SHAPE, 0, 2);
+    } else {
+      if (so[0] != 0 || so[sz.R] != sz.N) report(st, GPO_ERR_SHAPE, 0, 1);
+      if (to[0] != 0 || to[sz.R] != sz.T) report(st, GPO_ERR_SHAPE, 0, 2);
+    }
   }
   for (int g = tid; g < sz.G; g += nth) {
     const int a = go[g], c = go[g + 1];
@@ -76,7 +82,7 @@ __global__ void __launch_bounds__(kPlanThreads) prep_kernel(gpo_batch b, Sizes s
   }
   // one warp per rollout: its lanes stride over the rollout's steps
   const int lane = threadIdx.x & 31;
-  for (int r = tid >> 5; r < sz.R; r += nth >> 5) {
+  for (int r = tid >> 5; r < (tree ? 0 : sz.R); r += nth >> 5) {
     const int s = so[r], e = so[r + 1];
     if (s < 0 || e <= s || e > sz.N) {  // every rollout has at least one step
       if (lane == 0) report(st, GPO_ERR_SHAPE, 0, 4);
@@ -122,8 +128,12 @@ __global__ void __launch_bounds__(kPlanThreads) prep_kernel(gpo_batch b, Sizes s
     int cnt = 0, nb = 0, s0 = 0, n = 0;
     if (ok && g < sz.G) {
       const int r0 = go[g], r1 = go[g + 1];
-      s0 = so[r0];
-      n = so[r1] - s0;
+      s0 = tree ? b.group_state_off[g] : so[r0];
+      n = (tree ? b.group_state_off[g + 1] : so[r1]) - s0;
+      if (tree && (s0 < 0 || n < 0 || s0 + n > sz.N)) {  // reported by tree_prep_kernel
+        s0 = 0;
+        n = 0;
+      }
       if (n > sz.maxn || n > GPO_MAX_GROUP_STATES) report(st, GPO_ERR_UNSUPPORTED, 0, g);
       nb = blocks_for(n);
       cnt = nb + offdiag_for(n);
@@ -189,6 +199,158 @@ __global__ void __launch_bounds__(kPlanThreads) prep_kernel(gpo_batch b, Sizes s
   }
 }
 
+// ---------------------------------------------------------------------------
+// K0 (tree layout, before the planning kernel): one CTA per prompt group.  Checks the
+// group's offsets, parents (earlier states of the group, depth-first pre-order), step
+// lengths, leaf count and rewards; writes per state {group, depth}, the global parent,
+// the end of its subtree, its own terminal statistics (Sec. 4.3: c_own / t_own = the
+// rewards / the number of the leaves of its subtree, bottom-up along direct edges) and
+// the first token of its edge.
+constexpr int kTreeThreads = 1024;
+
+// Exclusive scan of (a, b) over the block; returns the block totals too.
+__device__ void block_excl_scan2(int& a, long long& b, int& ta, long long& tb, int* wa, long long* wb) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  int x = a;
+  long long y = b;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int u = __shfl_up_sync(0xffffffffu, x, o);
+    const long long v = __shfl_up_sync(0xffffffffu, y, o);
+    if (lane >= o) {
+      x += u;
+      y += v;
+    }
+  }
+  if (lane == 31) {
+    wa[wid] = x;
+    wb[wid] = y;
+  }
+  __syncthreads();
+  int pa = 0;
+  long long pb = 0;
+  ta = 0;
+  tb = 0;
+  for (int w = 0; w < nw; ++w) {
+    if (w < wid) {
+      pa += wa[w];
+      pb += wb[w];
+    }
+    ta += wa[w];
+    tb += wb[w];
+  }
+  a = pa + x - a;
+  b = pb + y - b;
+  __syncthreads();
+}
+
+__host__ __device__ inline size_t tree_prep_smem(int maxn) { return 4 * sizeof(int) * (size_t)(maxn < 1 ? 1 : maxn); }
+
+__global__ void __launch_bounds__(kTreeThreads) tree_prep_kernel(gpo_batch b, Sizes sz, Ws ws) {
+  extern __shared__ int tsm[];
+  __shared__ int s_wa[32];
+  __shared__ long long s_wb[32];
+  uint32_t* st = ws.status;
+  const int g = blockIdx.x, tid = threadIdx.x, nt = blockDim.x;
+  const int r0 = b.group_rollout_off[g], r1 = b.group_rollout_off[g + 1];
+  const int s0 = b.group_state_off[g], s1 = b.group_state_off[g + 1];
+  const int64_t t0 = b.group_token_off[g], t1 = b.group_token_off[g + 1];
+  if (r0 < 0 || r1 < r0 || r1 > sz.R || s0 < 0 || s1 < s0 || s1 > sz.N || t0 < 0 || t1 < t0 || t1 > sz.T ||
+      r1 - r0 > s1 - s0 || (s1 == s0 && (r1 != r0 || t1 != t0)) || (s1 > s0 && r1 == r0)) {
+    if (tid == 0) report(st, GPO_ERR_SHAPE, 0, 7);
+    return;
+  }
+  const int n = s1 - s0, nr = r1 - r0;
+  if (n == 0) return;
+  if (n > sz.maxn || n > GPO_MAX_GROUP_STATES) return;  // the planning kernel reports it
+  int* par = tsm;
+  int* end = tsm + n;
+  int* cown = tsm + 2 * n;
+  int* town = tsm + 3 * n;
+  bool bad = false;
+  for (int i = tid; i < n; i += nt) {
+    const int pp = b.parent[s0 + i], L = b.step_len[s0 + i];
+    par[i] = pp;
+    end[i] = i + 1;
+    cown[i] = town[i] = 0;
+    bad = bad || pp < -1 || pp >= i || L < 1;
+  }
+  if (__syncthreads_or(bad)) {
+    if (tid == 0) report(st, GPO_ERR_SHAPE, 0, 8);
+    return;
+  }
+  for (int i = tid; i < n; i += nt) {
+    const int pp = par[i];
+    if (pp >= 0) {  // pre-order: p(v) lies on the path from the root to the state before v
+      int x = i - 1;
+      while (x > pp) x = par[x];
+      bad = bad || x != pp;
+    }
+    int d = 1;
+    for (int x = pp; x >= 0; x = par[x]) {  // par[x] < x: at most i steps
+      ++d;
+      atomicMax(&end[x], i + 1);
+    }
+    ws.state_meta[s0 + i] = make_int2(g, d);
+    ws.tree_par[s0 + i] = pp < 0 ? -1 : s0 + pp;
+  }
+  if (__syncthreads_or(bad)) {
+    if (tid == 0) report(st, GPO_ERR_SHAPE, 0, 9);
+    return;
+  }
+  // leaves in state order are the group's rollouts; edge spans follow in state order.  Each
+  // thread takes a contiguous run of states; one block scan over the runs.
+  const int per = (n + nt - 1) / nt, a0 = min(n, tid * per), a1 = min(n, a0 + per);
+  int lc = 0;
+  long long tc = 0;
+  for (int i = a0; i < a1; ++i) {
+    lc += end[i] == i + 1;
+    tc += b.step_len[s0 + i];
+  }
+  int ltot;
+  long long ttot;
+  block_excl_scan2(lc, tc, ltot, ttot, s_wa, s_wb);
+  if (ltot != nr || ttot != t1 - t0) {
+    if (tid == 0) report(st, GPO_ERR_SHAPE, 0, 10);
+    return;
+  }
+  for (int i = a0; i < a1; ++i) {
+    ws.tok_start[s0 + i] = t0 + tc;
+    tc += b.step_len[s0 + i];
+    if (end[i] == i + 1) {
+      const int rw = b.reward[r0 + lc];
+      ++lc;
+      if (rw > 1) {
+        report(st, GPO_ERR_BAD_REWARD, 0, r0 + lc - 1);
+        bad = true;
+      } else {
+        for (int x = i; x >= 0; x = par[x]) {
+          atomicAdd(&cown[x], rw);
+          atomicAdd(&town[x], 1);
+        }
+      }
+    }
+  }
+  if (__syncthreads_or(bad)) return;
+  for (int i = tid; i < n; i += nt) {
+    ws.tree_end[s0 + i] = s0 + end[i];
+    ws.tree_own[s0 + i] = make_int2(cown[i], town[i]);
+  }
+}
+
+cudaError_t setup_tree_prep() {
+  return cudaFuncSetAttribute(tree_prep_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)tree_prep_smem(GPO_MAX_GROUP_STATES));
+}
+
+cudaError_t launch_tree_prep(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws) {
+  if (sz.G == 0) return cudaSuccess;
+  int threads = (sz.maxn + 31) & ~31;
+  threads = threads < 64 ? 64 : (threads > kTreeThreads ? kTreeThreads : threads);
+  tree_prep_kernel<<<sz.G, threads, tree_prep_smem(sz.maxn), lc.stream>>>(b, sz, ws);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_prep(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws) {
   const int64_t work = 32 * ((int64_t)sz.R + 1);  // a warp per rollout
   int blocks = (int)((work + kPlanThreads - 1) / kPlanThreads);
@@ -244,14 +406,14 @@ __global__ void __launch_bounds__(256) row_stats_kernel(gpo_batch b, Sizes sz, W
     if (job < sz.N) {
       row = job;
       rowp = b.emb;
-      const int2 m = ws.state_meta[job];
+      const int2 m = ws.state_meta[job];  // {rollout, depth}; tree layout: {group, depth}
       if (kRootsOnly && m.y > 1) continue;
       if (m.y > 1) {
         parp = b.emb;
-        prow = job - 1;
+        prow = b.parent ? ws.tree_par[job] : job - 1;
       } else if (b.root_emb) {
         parp = b.root_emb;
-        prow = ws.rollout_group[m.x];
+        prow = b.parent ? m.x : ws.rollout_group[m.x];
       }
     } else {
       row = job - sz.N;
@@ -409,7 +571,7 @@ cudaError_t launch_row_stats(const LaunchCtx& lc, const gpo_batch& b, const Size
   const int64_t cap = (int64_t)lc.num_sms * 8;
   if (blocks > cap) blocks = cap;
   const bool aligned16 = (reinterpret_cast<uintptr_t>(b.emb) & 15u) == 0 && sz.stride % 8 == 0 && sz.d % 8 == 0;
-  if (b.emb_dtype == GPO_EMB_BF16 && aligned16 && sz.d <= 8 * 32 * 8) {
+  if (b.emb_dtype == GPO_EMB_BF16 && aligned16 && sz.d <= 8 * 32 * 8 && !b.parent) {  // chain layout: p(v) = v - 1
     int64_t rblocks = ((int64_t)sz.N + 255) / 256;  // a warp per 32 rows
     if (rblocks < 1) rblocks = 1;
     if (rblocks > (int64_t)lc.num_sms * 8) rblocks = (int64_t)lc.num_sms * 8;
@@ -421,6 +583,181 @@ cudaError_t launch_row_stats(const LaunchCtx& lc, const gpo_batch& b, const Size
     row_stats_kernel<true, false><<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
   else
     row_stats_kernel<false, false><<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Accurate row statistics for eta(p(v), v) = max(0, cos(z_{p(v)}, z_v)) (Sec. 4.3): |z_v|^2
+// and <z_{p(v)}, z_v> as float pairs, one warp per state.  p(v) is the previous state of
+// the rollout (chain layout) or the parent (tree layout); a root child is dotted with its
+// group's prompt embedding when one is given.  bf16 products are exact in fp32, fp32
+// products are split exactly by TwoProduct, and every sum is compensated (Sum2), so the
+// cosine keeps ~1e-12 absolute accuracy even for nearly orthogonal rows, where a plain
+// fp32 (or tensor-core) accumulation loses it: the standardisation of Sec. 4.4 then
+// amplifies that loss in groups of nearly equal step rewards.
+// Nothing outside the arrays is read whatever the offsets hold: rollout and group come
+// from binary searches, and a parent outside [start of the group, v) counts as the root
+// (the validating kernels report such inputs).
+
+__device__ __forceinline__ int upper_idx(const int32_t* off, int n, int v) {  // last r < n with off[r] <= v
+  int lo = 0, hi = n - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (off[mid] <= v) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
+}
+
+template <bool kBf16>
+__device__ __forceinline__ void exact_pair_sums(const void* base, int64_t zrow, const void* pbase, int64_t prow,
+                                                bool has_p, int d, int lane, float2& n2, float2& dot) {
+  float nh = 0.f, nl = 0.f, dh = 0.f, dl = 0.f;
+  constexpr int kVec = kBf16 ? 8 : 4;  // elements per 16-byte chunk
+  const int nvec = d / kVec;
+  for (int c = lane; c < nvec; c += 32) {
+    float x[kVec], y[kVec];
+    if (kBf16) {
+      const uint4 u = *reinterpret_cast<const uint4*>(reinterpret_cast<const uint16_t*>(base) + zrow + 8 * c);
+      const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        x[2 * i] = __uint_as_float(w[i] << 16);
+        x[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+      }
+      if (has_p) {
+        const uint4 v = *reinterpret_cast<const uint4*>(reinterpret_cast<const uint16_t*>(pbase) + prow + 8 * c);
+        const uint32_t q[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          y[2 * i] = __uint_as_float(q[i] << 16);
+          y[2 * i + 1] = __uint_as_float(q[i] & 0xFFFF0000u);
+        }
+      }
+    } else {
+      const float4 u = *reinterpret_cast<const float4*>(reinterpret_cast<const float*>(base) + zrow + 4 * c);
+      x[0] = u.x; x[1] = u.y; x[2] = u.z; x[3] = u.w;
+      if (has_p) {
+        const float4 v = *reinterpret_cast<const float4*>(reinterpret_cast<const float*>(pbase) + prow + 4 * c);
+        y[0] = v.x; y[1] = v.y; y[2] = v.z; y[3] = v.w;
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < kVec; ++i) {
+      const float sq = x[i] * x[i];
+      ff_acc(nh, nl, sq);
+      if (!kBf16) nl += fmaf(x[i], x[i], -sq);  // TwoProduct error (bf16 squares are exact)
+      if (has_p) {
+        const float pr = x[i] * y[i];
+        ff_acc(dh, dl, pr);
+        if (!kBf16) dl += fmaf(x[i], y[i], -pr);
+      }
+    }
+  }
+  for (int k = nvec * kVec + lane; k < d; k += 32) {  // ragged tail of the row
+    const float x = kBf16 ? __uint_as_float((uint32_t)(reinterpret_cast<const uint16_t*>(base)[zrow + k]) << 16)
+                          : reinterpret_cast<const float*>(base)[zrow + k];
+    const float sq = x * x;
+    ff_acc(nh, nl, sq);
+    nl += fmaf(x, x, -sq);
+    if (has_p) {
+      const float y = kBf16 ? __uint_as_float((uint32_t)(reinterpret_cast<const uint16_t*>(pbase)[prow + k]) << 16)
+                            : reinterpret_cast<const float*>(pbase)[prow + k];
+      const float pr = x * y;
+      ff_acc(dh, dl, pr);
+      dl += fmaf(x, y, -pr);
+    }
+  }
+  // combine the lanes' pairs (fixed butterfly order: deterministic)
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float a = __shfl_xor_sync(0xffffffffu, nh, o), b = __shfl_xor_sync(0xffffffffu, nl, o);
+    const float c = __shfl_xor_sync(0xffffffffu, dh, o), e = __shfl_xor_sync(0xffffffffu, dl, o);
+    float s, t;
+    two_sum(nh, a, s, t);
+    nh = s;
+    nl = nl + b + t;
+    two_sum(dh, c, s, t);
+    dh = s;
+    dl = dl + e + t;
+  }
+  float h, l;
+  two_sum(nh, nl, h, l);
+  n2 = make_float2(h, l);
+  two_sum(dh, dl, h, l);
+  dot = make_float2(h, l);
+}
+
+template <bool kBf16>
+__global__ void __launch_bounds__(256) exact_stats_kernel(gpo_batch b, Sizes sz, Ws ws) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  const bool tree = b.parent != nullptr;
+  // the states and prompt embeddings of groups [g0, g1) (the whole batch but for range calls)
+  int v0 = 0, v1 = sz.N;
+  if (sz.g0 != 0 || sz.g1 != sz.G) {
+    const int32_t* go = b.group_rollout_off;
+    if (tree) {
+      v0 = b.group_state_off[sz.g0];
+      v1 = b.group_state_off[sz.g1];
+    } else {
+      const int ra = go[sz.g0], rb = go[sz.g1];
+      v0 = ra >= 0 && ra <= sz.R ? b.rollout_step_off[ra] : 0;
+      v1 = rb >= 0 && rb <= sz.R ? b.rollout_step_off[rb] : 0;
+    }
+    v0 = max(0, min(v0, sz.N));
+    v1 = max(v0, min(v1, sz.N));
+  }
+  const int nstate = v1 - v0, nroot = b.root_emb ? sz.g1 - sz.g0 : 0;
+  for (int64_t jj = warp; jj < (int64_t)nstate + nroot; jj += nwarps) {
+    const int64_t job = jj < nstate ? v0 + jj : sz.N + sz.g0 + (jj - nstate);
+    if (job >= sz.N) {  // |prompt embedding|^2
+      const int64_t g = job - sz.N;
+      float2 n2, dot;
+      exact_pair_sums<kBf16>(b.root_emb, g * sz.stride, nullptr, 0, false, sz.d, lane, n2, dot);
+      if (lane == 0) {
+        if (!isfinite(n2.x)) report(ws.status, GPO_ERR_NONFINITE, 3, (int)job);
+        ws.x_root_n2[g] = n2;
+      }
+      continue;
+    }
+    const int v = (int)job;
+    int prow = -1, g = -1;  // parent row, or the group whose prompt embedding is the parent
+    if (tree) {
+      if (sz.G > 0) {
+        g = upper_idx(b.group_state_off, sz.G, v);
+        const int s0 = b.group_state_off[g], pl = b.parent[v];
+        if (pl >= 0 && s0 >= 0 && (int64_t)s0 + pl < v) prow = s0 + pl;
+      }
+    } else if (sz.R > 0) {
+      const int r = upper_idx(b.rollout_step_off, sz.R, v);
+      if (v > b.rollout_step_off[r]) prow = v - 1;
+      else if (sz.G > 0) g = upper_idx(b.group_rollout_off, sz.G, r);
+    }
+    const bool root_parent = prow < 0 && b.root_emb && g >= 0;
+    const void* pbase = prow >= 0 ? b.emb : (root_parent ? b.root_emb : nullptr);
+    const int64_t poff = prow >= 0 ? (int64_t)prow * sz.stride : (root_parent ? (int64_t)g * sz.stride : 0);
+    float2 n2, dot;
+    exact_pair_sums<kBf16>(b.emb, (int64_t)v * sz.stride, pbase, poff, pbase != nullptr, sz.d, lane, n2, dot);
+    if (lane == 0) {
+      if (!isfinite(n2.x) || !isfinite(dot.x)) report(ws.status, GPO_ERR_NONFINITE, 3, v);
+      ws.x_n2[v] = n2;
+      ws.x_dot[v] = dot;
+    }
+  }
+}
+
+cudaError_t launch_exact_stats(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws) {
+  const int64_t jobs = (int64_t)sz.N + (b.root_emb ? sz.G : 0);  // at most (range calls take fewer)
+  if (jobs == 0) return cudaSuccess;
+  int64_t blocks = (jobs + 7) / 8;  // a warp per row
+  const int64_t cap = (int64_t)lc.num_sms * 16;
+  if (blocks > cap) blocks = cap;
+  if (b.emb_dtype == GPO_EMB_BF16)
+    exact_stats_kernel<true><<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
+  else
+    exact_stats_kernel<false><<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
   return cudaGetLastError();
 }
 

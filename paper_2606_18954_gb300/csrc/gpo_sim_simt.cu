@@ -49,10 +49,11 @@ __global__ void __launch_bounds__(kThreads) sim_simt_kernel(gpo_batch b, Sizes s
   __shared__ int lp[kSlots];
   __shared__ int cm_roll[kTileN], cm_depth[kTileN];
   __shared__ float cm_rn[kTileN];
-  __shared__ int rm_roll[kTileM], rm_depth[kTileM];
+  __shared__ int rm_roll[kTileM], rm_depth[kTileM], rm_end[kTileM];
   __shared__ float rm_rn[kTileM];
   __shared__ int edge_n;
   uint32_t* st = ws.status;
+  const bool tree = ws.tree_end != nullptr;
   const int nitems = (int)*((volatile uint32_t*)&st[kStItems]);
   if (aborted(st)) return;
   const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
@@ -78,6 +79,7 @@ __global__ void __launch_bounds__(kThreads) sim_simt_kernel(gpo_batch b, Sizes s
         rm_roll[r] = mt.x;
         rm_depth[r] = mt.y;
         rm_rn[r] = ws.rn[row];
+        rm_end[r] = tree ? ws.tree_end[row] : 0;
       } else {
         rm_roll[r] = -1;
       }
@@ -133,7 +135,8 @@ __global__ void __launch_bounds__(kThreads) sim_simt_kernel(gpo_batch b, Sizes s
       for (int j = 0; j < 16; ++j) {
         const int c = tx * 16 + j;
         const int col = item.col0 + c;
-        if (c >= item.ncols || col <= row || cm_roll[c] == rm_roll[r]) continue;
+        // comparable: not the row's own rollout (tree layout: outside the row's subtree)
+        if (c >= item.ncols || col <= row || (tree ? col < rm_end[r] : cm_roll[c] == rm_roll[r])) continue;
         if (rule == GPO_MERGE_SAME_DEPTH && cm_depth[c] != rm_depth[r]) continue;
         if (acc[i][j] * rm_rn[r] * cm_rn[c] >= kappa) {
           const int sc = (col < item.row0 + kTileM) ? col - item.row0 : kTileM + (col - item.col0);

@@ -56,6 +56,7 @@ struct __align__(8) SmemCtl {
   int overflow;                    // some warp found more pairs than its list holds
   int lp[kSlots];                  // label forest of the item's slots (rows, then columns)
   int cm_depth[kTileN];
+  int cm_par[kTileN];              // tree layout: parent (global) of each column state
   alignas(16) float cm_rn[kTileN];  // 1 / |z| of the item's columns
   uint32_t elist[kEpiWarps][kWarpEdges];  // slot pairs (row slot | column slot << 16)
 };
@@ -117,6 +118,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   constexpr uint32_t kCtlBytes = (sizeof(SmemCtl) + 15) & ~15u;
   unsigned char* tiles = smem_raw + (((sbase + kCtlBytes + 1023u) & ~1023u) - sbase);
   uint32_t* st = ws.status;
+  const bool tree = ws.tree_end != nullptr;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nitems = (int)*((volatile uint32_t*)&st[kStItems]);
@@ -244,19 +246,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int blk_row = gi.blk0 + (item.row0 - gi.s0) / kTileM;
       const int buf = m & 1;
       epi_sync();  // previous item finished with the metadata, lists and forest
-      for (int c = te; c < item.ncols; c += kEpiThreads) ctl->cm_depth[c] = ws.state_meta[item.col0 + c].y;
+      for (int c = te; c < item.ncols; c += kEpiThreads) {
+        ctl->cm_depth[c] = ws.state_meta[item.col0 + c].y;
+        if (tree) ctl->cm_par[c] = ws.tree_par[item.col0 + c];
+      }
       for (int c = item.ncols + te; c < kTileN; c += kEpiThreads) ctl->cm_rn[c] = 0.f;
       if (te == 0) {
         ctl->edge_n = 0;
         ctl->overflow = 0;
       }
-      // row constants: end of the row's rollout (in the chain layout the comparable columns
-      // right of row i are exactly those at or after it) and depth
+      // row constants: end of the row's rollout (tree layout: of its subtree; the comparable
+      // columns right of row i are exactly those at or after it) and depth
       const int row = item.row0 + t;
       int re = send, di = -1;
       if (row < send) {
         const int2 mt = ws.state_meta[row];
-        re = rollout_step_off[mt.x + 1];
+        re = tree ? ws.tree_end[row] : rollout_step_off[mt.x + 1];
         di = mt.y;
       }
       float thr = __int_as_float(0x7f800000);  // kappa |z_i|; +inf for a zero or absent row
@@ -304,7 +309,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             ws.rn[row] = rni;
             ctl->cm_rn[t] = rni;
             if (!isfinite(dg)) report(st, GPO_ERR_NONFINITE, 1, row);
-            if (t + 1 < item.ncols && ctl->cm_depth[t + 1] > 1) ws.dotp[row + 1] = up;
+            if (!tree && t + 1 < item.ncols && ctl->cm_depth[t + 1] > 1) ws.dotp[row + 1] = up;
           }
           __threadfence();
         }
@@ -327,8 +332,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_wait_ld();
         // <z of the block's last row, z of the next block's first row>: the parent dot of
         // the next block's first state when it continues the same rollout
-        if (ch == 0 && q == 3 && lane == 31 && item.col0 == item.row0 + kTileM && ctl->cm_depth[0] > 1)
+        if (!tree && ch == 0 && q == 3 && lane == 31 && item.col0 == item.row0 + kTileM && ctl->cm_depth[0] > 1)
           ws.dotp[item.col0] = __uint_as_float(r[0]);
+        if (tree) {
+          // tree layout: <z_{p(v)}, z_v> of every child v of this row in the chunk (each
+          // (parent, child) pair lies in exactly one item's upper part)
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            const int c = ch * 32 + j;
+            if (c < item.ncols && ctl->cm_par[c] == row) ws.dotp[item.col0 + c] = __uint_as_float(r[j]);
+          }
+        }
         uint32_t mp[4] = {0u, 0u, 0u, 0u};
         const float4* rn4 = reinterpret_cast<const float4*>(ctl->cm_rn + ch * 32);
 #pragma unroll

@@ -42,8 +42,10 @@ rollout by rollout, step by step):
 Trees: the root expands b_1 children; a state at layer h < H ends its branch
 early with probability p_stop, else expands b_{h+1} children; states of layer H
 are terminal.  Structure first (pre-order), then step lengths, embeddings (the
-same centroid recipe with n_max = H), leaf rewards and the margin filter over
-the pairs not in an ancestor-descendant relation.
+same centroid recipe with n_max = max(H, K/2): the band advances by at most two
+centroids per layer, so neighbouring layers share centroids and classes span
+depths, as in the chain workloads), leaf rewards and the margin filter over the
+pairs not in an ancestor-descendant relation.
 """
 from __future__ import annotations
 
@@ -322,6 +324,7 @@ def make_tree_batch(spec: TreeSpec, seed: Optional[int] = None, margin_check: bo
         seed = config_seed(spec.name)
     rng = np.random.default_rng(seed)
     H, G, d = len(spec.schedule), spec.groups, spec.d
+    n_band = max(H, spec.centroids // 2)  # depth span of the centroid bands
     pars, lens, store, planted, rewards, nleaf, nstate = [], [], [], [], [], [], []
     resampled = 0
     for g in range(G):
@@ -335,7 +338,7 @@ def make_tree_batch(spec: TreeSpec, seed: Optional[int] = None, margin_check: bo
         end = subtree_end(par)
         leaves = int(np.sum(end == np.arange(1, n + 1)))
         lens.append(rng.integers(spec.lengths[1], spec.lengths[2] + 1, size=n).astype(np.int32))
-        z, cid = _draw_states(rng, spec, cents, dep, H)
+        z, cid = _draw_states(rng, spec, cents, dep, n_band)
         s, e = _round(spec, z)
         rewards.extend((rng.random(leaves) < p).astype(np.uint8).tolist())
         if margin_check:
@@ -345,7 +348,7 @@ def make_tree_batch(spec: TreeSpec, seed: Optional[int] = None, margin_check: bo
                 r = rows[:, None]
                 return ((idx[None, :] >= end[r]) | (r >= end[idx][None, :])) & (r != idx[None, :])
 
-            resampled += _margin_filter(rng, spec, cents, H, s, e, cid, None, dep, comparable)
+            resampled += _margin_filter(rng, spec, cents, n_band, s, e, cid, None, dep, comparable)
         pars.append(par)
         store.append(s)
         planted.append(cid)
