@@ -40,7 +40,21 @@ WORKLOADS = {
             "64 centroids/prompt, sigma 0.06",
     "full": "full batch: 512 prompts x 16 rollouts, ~20 steps, lognormal lengths (median 4k, cap 16k), "
             "bf16 d=1024, 48 centroids/prompt",
+    "tree": "branching rollouts (tree layout): 128 prompts, branching schedule {2,5,4,2,2} (<= 292 states and "
+            "160 leaves per prompt), edges of 64-512 tokens, bf16 d=1024, 32 centroids/prompt, sigma 0.08, "
+            "rewards Bernoulli(Beta(2,2))",
 }
+
+
+def make_workload(name, seed_offset=0):
+    from paper_2606_18954_gb300 import workloads as W
+    if name in W.TREE_CONFIGS:
+        return W.make_tree_batch(W.TREE_CONFIGS[name], seed=W.config_seed(name) + seed_offset)
+    return W.make_batch(W.CONFIGS[name], seed=W.config_seed(name) + seed_offset)
+
+
+def batch_tokens(b):
+    return int(b["total_tokens"]) if b.get("parent") is not None else int(b["rollout_token_off"][-1])
 
 
 def load_peaks():
@@ -58,17 +72,25 @@ def algorithmic(b):
     N = len(b["step_len"])
     R = len(b["reward"])
     G = len(b["group_rollout_off"]) - 1
-    T = int(b["rollout_token_off"][-1])
+    T = batch_tokens(b)
     d = b["emb"].shape[1]
     esz = 2 if b["emb_dtype"] == "bf16" else 4
     zb = N * d * esz
-    so, go = b["rollout_step_off"], b["group_rollout_off"]
-    ng = (so[go[1:]] - so[go[:-1]]).astype(np.float64)
+    tree = b.get("parent") is not None
+    if tree:
+        ng = np.diff(b["group_state_off"]).astype(np.float64)
+        meta = 4 * N + 16 * (G + 1)  # parents + group rollout / state / token offsets
+    else:
+        so, go = b["rollout_step_off"], b["group_rollout_off"]
+        ng = (so[go[1:]] - so[go[:-1]]).astype(np.float64)
+        meta = 12 * R
     flops = float(d * (ng ** 2).sum())  # comparable upper triangle: 2 d n^2 / 2 per group
-    path_bytes = zb + 4 * N + 12 * R + R + 4 * T
+    path_bytes = zb + 4 * N + meta + R + 4 * T
     stages = {
+        "exact_stats": (zb + 16 * N, 0.0),
+        "tree_prep": (meta + 4 * N + R + 24 * N, 0.0),
         "prep": (4 * (G + 1) + 12 * (R + 1) + 4 * N + R + 8 * N + 4 * R, 0.0),
-        "row_stats": (zb + 8 * N + 12 * N, 0.0),
+        "row_stats": (zb + 8 * N, 0.0),
         "similarity": (zb + 12 * N, flops),
         "groups": (8 * N + R + 12 * R + 4 * N + 17 * N + 8 * N, 0.0),
         "tokens": (4 * T + 8 * N + 4 * N + 4 * N, 0.0),
@@ -159,7 +181,8 @@ def traffic_for(kernel_file, workload):
         return None, "no capture"
 
 
-STAGE_SOURCE = {"prep": "gpo_prep.cu", "row_stats": "gpo_prep.cu", "similarity": "gpo_sim_tc.cu",
+STAGE_SOURCE = {"prep": "gpo_prep.cu", "tree_prep": "gpo_prep.cu", "exact_stats": "gpo_prep.cu",
+                "row_stats": "gpo_prep.cu", "similarity": "gpo_sim_tc.cu",
                 "groups": "gpo_group.cu", "tokens": "gpo_prep.cu", "fused": "gpo_fused.cu"}
 
 
@@ -173,7 +196,7 @@ def cpu_baseline(b, budget_s=6.0, max_groups=None):
     if max_groups is not None and G > max_groups:
         sub = W.sub_batch(b, range(max_groups))
         sample = f"the first {max_groups} of {G} groups"
-    T = int(sub["rollout_token_off"][-1])
+    T = batch_tokens(sub)
     params = dict(kappa=b["kappa"], w=b["w"], lambda_eff=b["lambda_eff"])
     oracle.run(W.sub_batch(sub, [0]), params, threads=1)  # build + warm
     times = []
@@ -201,7 +224,7 @@ def run_reference(args):
         return 0
     from paper_2606_18954_gb300 import workloads as W
     import oracle
-    b = W.make_batch(W.CONFIGS[args.config])
+    b = make_workload(args.config)
     cores = len(os.sched_getaffinity(0))
     G = len(b["group_rollout_off"]) - 1
     max_groups = {"wide": 2, "full": 64}.get(args.config)
@@ -209,7 +232,7 @@ def run_reference(args):
     if max_groups and G > max_groups:
         sub = W.sub_batch(b, range(max_groups))
         sample = f"the first {max_groups} of {G} groups per step"
-    T = int(sub["rollout_token_off"][-1])
+    T = batch_tokens(sub)
     params = dict(kappa=b["kappa"], w=b["w"], lambda_eff=b["lambda_eff"])
     for _ in range(args.warmup):
         oracle.run(sub, params, threads=cores, want={"adv"})
@@ -246,8 +269,7 @@ def run_ours(args):
         torch.cuda.set_device(0)
     dev = torch.device("cuda", torch.cuda.current_device())
     P.build()
-    spec = W.CONFIGS[args.config]
-    b = W.make_batch(spec, seed=W.config_seed(args.config) + rank)
+    b = make_workload(args.config, rank)
     alg = algorithmic(b)
     db = P.Batch.from_arrays(b, device=dev)
     gp = P.GraphPO(kappa=b["kappa"], w=b["w"], lambda_eff=b["lambda_eff"])
@@ -315,7 +337,8 @@ def run_ours(args):
     hb = P.Batch.from_arrays(b, device="cpu", pin=True)
     host_out = torch.empty(alg["T"], dtype=torch.float32, pin_memory=True)
     h2d = sum(t.numel() * t.element_size() for t in (hb.group_rollout_off, hb.rollout_step_off, hb.step_len,
-                                                      hb.rollout_token_off, hb.emb, hb.reward))
+                                                      hb.rollout_token_off, hb.emb, hb.reward, hb.parent,
+                                                      hb.group_state_off, hb.group_token_off) if t is not None)
     for _ in range(max(1, args.warmup // 2)):
         gp.compute_host(hb, out=host_out)
     e2e_ms = []
@@ -356,7 +379,8 @@ def run_ours(args):
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": WORKLOADS[args.config], "groups": alg["G"], "rollouts": alg["R"],
                    "states": alg["N"], "tokens": alg["T"], "d": int(b["emb"].shape[1]),
-                   "emb_dtype": b["emb_dtype"], "merge_rule": "noncausal", "kappa": b["kappa"], "w": b["w"],
+                   "emb_dtype": b["emb_dtype"], "layout": "tree" if b.get("parent") is not None else "chain",
+                   "merge_rule": "noncausal", "kappa": b["kappa"], "w": b["w"],
                    "lambda_eff": b["lambda_eff"], "l2": "flushed by a 256 MiB write before every timed step",
                    "seed": W.config_seed(args.config)},
         "graphs_per_s": ws_n * alg["G"] / (ms / 1e3),

@@ -65,7 +65,7 @@ int64_t max_items_for(int64_t N, int64_t G, int64_t maxn) {
 }
 
 struct Layout {
-  size_t status, items, blk_ready, groups, state_meta, rollout_group, nrm2, dotp, rn, root_n2, edge_count,
+  size_t status, items, blk_ready, groups, state_meta, nrm2, rn, edge_count,
       edges, e_adv, e_cor, e_eff, e_mask, tok_start, tree_par, tree_end, tree_own, tree_x, x_n2, x_dot, x_root_n2,
       total;
   int max_items;
@@ -91,11 +91,8 @@ bool layout(const gpo_batch& b, Layout& L) {
   L.blk_ready = take(sizeof(int) * mi);  // indexed by the diagonal items' positions
   L.groups = take(sizeof(GroupInfo) * G);
   L.state_meta = take(sizeof(int2) * N);
-  L.rollout_group = take(sizeof(int) * R);
   L.nrm2 = take(sizeof(float) * N);
-  L.dotp = take(sizeof(float) * N);
   L.rn = take(sizeof(float) * N);
-  L.root_n2 = take(sizeof(float) * G);
   L.edge_count = take(sizeof(int) * mi);
   L.edges = take(sizeof(int2) * (size_t)kEdgeCap * mi);
   L.e_adv = take(sizeof(float) * N);
@@ -125,11 +122,8 @@ Ws workspace_views(void* base, const Layout& L) {
   w.blk_ready = reinterpret_cast<int*>(p + L.blk_ready);
   w.groups = reinterpret_cast<GroupInfo*>(p + L.groups);
   w.state_meta = reinterpret_cast<int2*>(p + L.state_meta);
-  w.rollout_group = reinterpret_cast<int*>(p + L.rollout_group);
   w.nrm2 = reinterpret_cast<float*>(p + L.nrm2);
-  w.dotp = reinterpret_cast<float*>(p + L.dotp);
   w.rn = reinterpret_cast<float*>(p + L.rn);
-  w.root_n2 = reinterpret_cast<float*>(p + L.root_n2);
   w.edge_count = reinterpret_cast<int*>(p + L.edge_count);
   w.edges = reinterpret_cast<int2*>(p + L.edges);
   w.e_adv = reinterpret_cast<float*>(p + L.e_adv);

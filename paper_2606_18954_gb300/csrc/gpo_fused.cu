@@ -14,16 +14,16 @@
 //                   if a group needs more, blocks >= 1 go first, block 0 second
 //                   (Sec. 4.2: sim of every comparable pair)
 //   warps 4..       TMEM drain of each pass (three (large) or one (small) warps per
-//                   accumulator lane quarter, splitting the 32-column chunks): the diagonal and
-//                   super-diagonal entries give |z_i|^2 and <z_i, z_{i+1}> (the
-//                   norms of the cosine and eta(p(v), v)); then every comparable
-//                   pair (different rollout; optionally same depth) with
+//                   accumulator lane quarter, splitting the 32-column chunks): the diagonal
+//                   entries give |z_i|^2 (the norms of the threshold test); then every
+//                   comparable pair (not ancestor-related; optionally same depth) with
 //                   cos = acc / (|z_i||z_j|) >= kappa goes to an edge list; the
 //                   accumulator is released and the listed pairs are united in a
 //                   shared-memory union-find forest (Alg. S.1)
 //   warps 2..       per-group validation, graph reward and dual-group advantage
-//                   (gpo_group_math.cuh) and the token scatter (Sec. 4.5),
-//                   overlapping the next group's loads and MMAs
+//                   (gpo_group_math.cuh; eta(p(v), v) from the compensated row
+//                   statistics of exact_stats, run just before) and the token scatter
+//                   (Sec. 4.5), overlapping the next group's loads and MMAs
 // Group ranges are assigned round-robin to CTAs.  Every wait is bounded.
 #include "gpo_group_math.cuh"
 

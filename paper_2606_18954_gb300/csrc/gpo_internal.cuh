@@ -51,11 +51,8 @@ struct Ws {
   int* blk_ready;        // [max_items]: at a diagonal item's position, set once it has written its norms
   GroupInfo* groups;     // [G]
   int2* state_meta;      // [N] {rollout, depth}
-  int* rollout_group;    // [R]
-  float* nrm2;           // [N] squared norm (fp32 accumulation)
-  float* dotp;           // [N] <z_{p(v)}, z_v> (root embedding for depth 1 if given)
+  float* nrm2;           // [N] squared norm (fp32 accumulation; the threshold test)
   float* rn;             // [N] 1/|z| (0 for a zero row)
-  float* root_n2;        // [G]
   int* edge_count;       // [max_items]
   int2* edges;           // [max_items * kEdgeCap]
   float* e_adv;          // [N] A_dual per edge
@@ -385,6 +382,128 @@ __device__ __forceinline__ float2 ff_eta(float2 dot, float2 np, float2 nv) {
   return ff_div(dot, ff_sqrt(ff_mul(np, nv)));
 }
 
+// Two fp32 lanes per instruction (sm_100 and later): a pair (lo, hi) in one 64-bit
+// register.  Used where compensated sums must keep pace with the tile stream.
+__device__ __forceinline__ uint64_t f2add(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2sub(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2mul(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+// The two bf16 of a 32-bit word as fp32 lanes (low half first).
+__device__ __forceinline__ uint64_t bf16x2_f32x2(uint32_t w) {
+  return ((uint64_t)(w & 0xFFFF0000u) << 32) | (uint64_t)(w << 16);
+}
+// Compensated accumulation (TwoSum per lane) of x into (s, e).
+__device__ __forceinline__ void f2_acc(uint64_t& s, uint64_t& e, uint64_t x) {
+  const uint64_t t = f2add(s, x);
+  const uint64_t bb = f2sub(t, s);
+  e = f2add(e, f2add(f2sub(s, f2sub(t, bb)), f2sub(x, bb)));
+  s = t;
+}
+// The float pair of a two-lane compensated sum.
+__device__ __forceinline__ float2 f2_finish(uint64_t s, uint64_t e) {
+  const float s0 = __uint_as_float((uint32_t)s), s1 = __uint_as_float((uint32_t)(s >> 32));
+  const float e0 = __uint_as_float((uint32_t)e), e1 = __uint_as_float((uint32_t)(e >> 32));
+  float h, t;
+  two_sum(s0, s1, h, t);
+  float hh, ll;
+  two_sum(h, t + e0 + e1, hh, ll);
+  return make_float2(hh, ll);
+}
+
+// One warp: |z|^2 of the row at element offset zrow of `base` and, if has_p, its dot with
+// the row at poff of `pbase`, as float pairs.  bf16 products are exact in fp32, fp32
+// products are split by TwoProduct, sums are compensated (Sum2) per lane and the lanes'
+// pairs combined in a fixed butterfly (deterministic).  Rows start on 16-byte boundaries.
+template <bool kBf16>
+__device__ __forceinline__ void exact_pair_sums(const void* base, int64_t zrow, const void* pbase, int64_t prow,
+                                                bool has_p, int d, int lane, float2& n2, float2& dot) {
+  float nh = 0.f, nl = 0.f, dh = 0.f, dl = 0.f;
+  constexpr int kVec = kBf16 ? 8 : 4;  // elements per 16-byte chunk
+  const int nvec = d / kVec;
+  for (int c = lane; c < nvec; c += 32) {
+    float x[kVec], y[kVec];
+    if (kBf16) {
+      const uint4 u = *reinterpret_cast<const uint4*>(reinterpret_cast<const uint16_t*>(base) + zrow + 8 * c);
+      const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        x[2 * i] = __uint_as_float(w[i] << 16);
+        x[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+      }
+      if (has_p) {
+        const uint4 v = *reinterpret_cast<const uint4*>(reinterpret_cast<const uint16_t*>(pbase) + prow + 8 * c);
+        const uint32_t q[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          y[2 * i] = __uint_as_float(q[i] << 16);
+          y[2 * i + 1] = __uint_as_float(q[i] & 0xFFFF0000u);
+        }
+      }
+    } else {
+      const float4 u = *reinterpret_cast<const float4*>(reinterpret_cast<const float*>(base) + zrow + 4 * c);
+      x[0] = u.x; x[1] = u.y; x[2] = u.z; x[3] = u.w;
+      if (has_p) {
+        const float4 v = *reinterpret_cast<const float4*>(reinterpret_cast<const float*>(pbase) + prow + 4 * c);
+        y[0] = v.x; y[1] = v.y; y[2] = v.z; y[3] = v.w;
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < kVec; ++i) {
+      const float sq = x[i] * x[i];
+      ff_acc(nh, nl, sq);
+      if (!kBf16) nl += fmaf(x[i], x[i], -sq);  // TwoProduct error (bf16 squares are exact)
+      if (has_p) {
+        const float pr = x[i] * y[i];
+        ff_acc(dh, dl, pr);
+        if (!kBf16) dl += fmaf(x[i], y[i], -pr);
+      }
+    }
+  }
+  for (int k = nvec * kVec + lane; k < d; k += 32) {  // ragged tail of the row
+    const float x = kBf16 ? __uint_as_float((uint32_t)(reinterpret_cast<const uint16_t*>(base)[zrow + k]) << 16)
+                          : reinterpret_cast<const float*>(base)[zrow + k];
+    const float sq = x * x;
+    ff_acc(nh, nl, sq);
+    nl += fmaf(x, x, -sq);
+    if (has_p) {
+      const float y = kBf16 ? __uint_as_float((uint32_t)(reinterpret_cast<const uint16_t*>(pbase)[prow + k]) << 16)
+                            : reinterpret_cast<const float*>(pbase)[prow + k];
+      const float pr = x * y;
+      ff_acc(dh, dl, pr);
+      dl += fmaf(x, y, -pr);
+    }
+  }
+  // combine the lanes' pairs (fixed butterfly order: deterministic)
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float a = __shfl_xor_sync(0xffffffffu, nh, o), b = __shfl_xor_sync(0xffffffffu, nl, o);
+    const float c = __shfl_xor_sync(0xffffffffu, dh, o), e = __shfl_xor_sync(0xffffffffu, dl, o);
+    float s, t;
+    two_sum(nh, a, s, t);
+    nh = s;
+    nl = nl + b + t;
+    two_sum(dh, c, s, t);
+    dh = s;
+    dl = dl + e + t;
+  }
+  float h, l;
+  two_sum(nh, nl, h, l);
+  n2 = make_float2(h, l);
+  two_sum(dh, dl, h, l);
+  dot = make_float2(h, l);
+}
+
 // ------------------------------------------------------------------ token spans
 
 // One warp writes value v to dst[ts, te): 16-byte stores in the aligned middle,
@@ -419,7 +538,6 @@ cudaError_t launch_exact_stats(const LaunchCtx& lc, const gpo_batch& b, const Si
 cudaError_t launch_tree_prep(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws);
 cudaError_t setup_tree_prep();
 cudaError_t launch_row_stats(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws);
-cudaError_t launch_root_stats(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws);
 cudaError_t launch_sim_tc(const LaunchCtx& lc, const CUtensorMap& map, const gpo_batch& b, const Sizes& sz,
                           const Ws& ws, const Params& p);
 cudaError_t launch_sim_simt(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws,

@@ -74,11 +74,7 @@ __global__ void __launch_bounds__(kPlanThreads) prep_kernel(gpo_batch b, Sizes s
   }
   for (int g = tid; g < sz.G; g += nth) {
     const int a = go[g], c = go[g + 1];
-    if (a < 0 || c < a || c > sz.R) {
-      report(st, GPO_ERR_SHAPE, 0, 3);
-      continue;
-    }
-    for (int r = a; r < c; ++r) ws.rollout_group[r] = g;
+    if (a < 0 || c < a || c > sz.R) report(st, GPO_ERR_SHAPE, 0, 3);
   }
   // one warp per rollout: its lanes stride over the rollout's steps
   const int lane = threadIdx.x & 31;
@@ -360,10 +356,9 @@ cudaError_t launch_prep(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz
 }
 
 // ---------------------------------------------------------------------------
-// K1a: per state, |z_v|^2 and <z_{p(v)}, z_v> with fp32 accumulation (one warp
-// per row: lane partial sums over a strided set of elements, then a shuffle
-// tree).  p(v) is the previous state of the rollout, or the prompt embedding
-// for the first step when one is given.  Extra warps compute |root|^2.
+// K1a (CUDA-core similarity only): |z_v|^2 and 1/|z_v| with fp32 accumulation for the
+// threshold test, one warp per row (lane partial sums over a strided set of elements, then
+// a shuffle tree).  eta takes its norms from exact_stats instead.
 
 template <bool kBf16>
 __device__ __forceinline__ void load8(const void* base, int64_t elem, float (&x)[8]) {
@@ -389,200 +384,50 @@ __device__ __forceinline__ float load1(const void* base, int64_t elem) {
   return reinterpret_cast<const float*>(base)[elem];
 }
 
-// kRootsOnly: only what the tcgen05 similarity kernel does not produce itself, i.e. the
-// dots of first steps with the prompt embeddings and |root|^2.
-template <bool kBf16, bool kRootsOnly>
+template <bool kBf16, bool kVec>
 __global__ void __launch_bounds__(256) row_stats_kernel(gpo_batch b, Sizes sz, Ws ws) {
   if (aborted(ws.status)) return;
   const int lane = threadIdx.x & 31;
   const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  const int nroot = b.root_emb ? sz.G : 0;
-  const int d = sz.d, nvec = d / 8;
-  for (int64_t job = warp; job < (int64_t)sz.N + nroot; job += nwarps) {
-    const void* rowp;
-    const void* parp = nullptr;
-    int64_t row, prow = 0;
-    if (job < sz.N) {
-      row = job;
-      rowp = b.emb;
-      const int2 m = ws.state_meta[job];  // {rollout, depth}; tree layout: {group, depth}
-      if (kRootsOnly && m.y > 1) continue;
-      if (m.y > 1) {
-        parp = b.emb;
-        prow = b.parent ? ws.tree_par[job] : job - 1;
-      } else if (b.root_emb) {
-        parp = b.root_emb;
-        prow = b.parent ? m.x : ws.rollout_group[m.x];
-      }
-    } else {
-      row = job - sz.N;
-      rowp = b.root_emb;
-    }
-    const int64_t rb = row * sz.stride, pb = prow * sz.stride;
-    float s2 = 0.f, sd = 0.f;
+  const int d = sz.d, nvec = kVec ? d / 8 : 0;
+  for (int64_t row = warp; row < sz.N; row += nwarps) {
+    const int64_t rb = row * sz.stride;
+    float s2 = 0.f;
 #pragma unroll 2
     for (int k = lane; k < nvec; k += 32) {
       float x[8];
-      load8<kBf16>(rowp, rb + 8 * k, x);
-      if (parp) {
-        float y[8];
-        load8<kBf16>(parp, pb + 8 * k, y);
-#pragma unroll
-        for (int i = 0; i < 8; ++i) sd = fmaf(x[i], y[i], sd);
-      }
+      load8<kBf16>(b.emb, rb + 8 * k, x);
 #pragma unroll
       for (int i = 0; i < 8; ++i) s2 = fmaf(x[i], x[i], s2);
     }
     for (int k = nvec * 8 + lane; k < d; k += 32) {
-      const float x = load1<kBf16>(rowp, rb + k);
+      const float x = load1<kBf16>(b.emb, rb + k);
       s2 = fmaf(x, x, s2);
-      if (parp) sd = fmaf(x, load1<kBf16>(parp, pb + k), sd);
     }
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      s2 += __shfl_xor_sync(0xffffffffu, s2, o);
-      sd += __shfl_xor_sync(0xffffffffu, sd, o);
-    }
+    for (int o = 16; o > 0; o >>= 1) s2 += __shfl_xor_sync(0xffffffffu, s2, o);
     if (lane == 0) {
-      if (!isfinite(s2) || !isfinite(sd)) report(ws.status, GPO_ERR_NONFINITE, 1, (int)job);
-      if (job < sz.N) {
-        if (!kRootsOnly) {
-          ws.nrm2[row] = s2;
-          ws.rn[row] = s2 > 0.f ? 1.0f / sqrtf(s2) : 0.f;
-        }
-        ws.dotp[row] = sd;
-      } else {
-        ws.root_n2[row] = s2;
-      }
+      if (!isfinite(s2)) report(ws.status, GPO_ERR_NONFINITE, 1, (int)row);
+      ws.nrm2[row] = s2;
+      ws.rn[row] = s2 > 0.f ? 1.0f / sqrtf(s2) : 0.f;
     }
   }
-}
-
-// bf16 rows of d = 8 * 32 * kNV elements at most: one warp walks a run of 32
-// consecutive rows (one coalesced metadata load for the run), holds a whole row in
-// registers (kNV 16-byte chunks per lane) and keeps it as the parent of the next
-// row, so every row is read once.  The prompt rows (|root|^2) and the dots of first
-// steps against them come from the generic kernel's formula with plain loads.
-template <int kNV>
-__global__ void __launch_bounds__(256) row_stats_run_kernel(gpo_batch b, Sizes sz, Ws ws) {
-  if (aborted(ws.status)) return;
-  const int lane = threadIdx.x & 31;
-  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  const int nvec = sz.d / 8;
-  const uint4* Z = reinterpret_cast<const uint4*>(b.emb);
-  const int64_t rs = sz.stride / 8;  // row stride in 16-byte chunks
-  auto load_row = [&](int64_t r, uint4 (&x)[kNV]) {
-#pragma unroll
-    for (int c = 0; c < kNV; ++c) {
-      const int k = lane + 32 * c;
-      x[c] = k < nvec ? Z[r * rs + k] : make_uint4(0u, 0u, 0u, 0u);
-    }
-  };
-  auto dot2 = [](uint32_t a, uint32_t b) {  // two bf16 pairs, fp32 products
-    return __uint_as_float(a << 16) * __uint_as_float(b << 16) +
-           __uint_as_float(a & 0xFFFF0000u) * __uint_as_float(b & 0xFFFF0000u);
-  };
-  for (int64_t base = warp * 32; base < sz.N; base += nwarps * 32) {
-    const int64_t nrun = min((int64_t)32, (int64_t)sz.N - base);
-    const int2 m = lane < nrun ? ws.state_meta[base + lane] : make_int2(0, 1);
-    uint4 prev[kNV], cur[kNV], nxt[kNV];
-    const int d0 = __shfl_sync(0xffffffffu, m.y, 0);
-    if (d0 > 1) load_row(base - 1, prev);
-    load_row(base, nxt);
-    for (int i = 0; i < nrun; ++i) {
-      const int dep = __shfl_sync(0xffffffffu, m.y, i);
-      const int rol = __shfl_sync(0xffffffffu, m.x, i);
-#pragma unroll
-      for (int c = 0; c < kNV; ++c) cur[c] = nxt[c];
-      if (i + 1 < nrun) load_row(base + i + 1, nxt);  // next row in flight during this one
-      float s2 = 0.f, sd = 0.f;
-#pragma unroll
-      for (int c = 0; c < kNV; ++c) {
-        const uint32_t w[4] = {cur[c].x, cur[c].y, cur[c].z, cur[c].w};
-#pragma unroll
-        for (int h = 0; h < 4; ++h) {
-          const float lo = __uint_as_float(w[h] << 16), hi = __uint_as_float(w[h] & 0xFFFF0000u);
-          s2 = fmaf(lo, lo, s2);
-          s2 = fmaf(hi, hi, s2);
-        }
-      }
-      if (dep > 1) {
-#pragma unroll
-        for (int c = 0; c < kNV; ++c) {
-          sd += dot2(cur[c].x, prev[c].x) + dot2(cur[c].y, prev[c].y);
-          sd += dot2(cur[c].z, prev[c].z) + dot2(cur[c].w, prev[c].w);
-        }
-      } else if (b.root_emb) {
-        const uint16_t* R = reinterpret_cast<const uint16_t*>(b.root_emb) + (int64_t)ws.rollout_group[rol] * sz.stride;
-        const uint16_t* X = reinterpret_cast<const uint16_t*>(b.emb) + (base + i) * sz.stride;
-        for (int k = lane; k < sz.d; k += 32)
-          sd = fmaf(__uint_as_float((uint32_t)X[k] << 16), __uint_as_float((uint32_t)R[k] << 16), sd);
-      }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        s2 += __shfl_xor_sync(0xffffffffu, s2, o);
-        sd += __shfl_xor_sync(0xffffffffu, sd, o);
-      }
-      if (lane == 0) {
-        const int64_t row = base + i;
-        if (!isfinite(s2) || !isfinite(sd)) report(ws.status, GPO_ERR_NONFINITE, 1, (int)row);
-        ws.nrm2[row] = s2;
-        ws.dotp[row] = sd;
-        ws.rn[row] = s2 > 0.f ? 1.0f / sqrtf(s2) : 0.f;
-      }
-#pragma unroll
-      for (int c = 0; c < kNV; ++c) prev[c] = cur[c];
-    }
-  }
-  // |root|^2 of every prompt embedding
-  if (b.root_emb) {
-    const uint16_t* R = reinterpret_cast<const uint16_t*>(b.root_emb);
-    for (int64_t g = warp; g < sz.G; g += nwarps) {
-      float s2 = 0.f;
-      for (int k = lane; k < sz.d; k += 32) {
-        const float x = __uint_as_float((uint32_t)R[g * sz.stride + k] << 16);
-        s2 = fmaf(x, x, s2);
-      }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) s2 += __shfl_xor_sync(0xffffffffu, s2, o);
-      if (lane == 0) {
-        if (!isfinite(s2)) report(ws.status, GPO_ERR_NONFINITE, 1, (int)(sz.N + g));
-        ws.root_n2[g] = s2;
-      }
-    }
-  }
-}
-
-cudaError_t launch_root_stats(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws) {
-  const int64_t jobs = (int64_t)sz.N + sz.G;
-  if (!b.root_emb || jobs == 0) return cudaSuccess;
-  int64_t blocks = (jobs * 32 + 255) / 256;
-  if (blocks > (int64_t)lc.num_sms * 8) blocks = (int64_t)lc.num_sms * 8;
-  row_stats_kernel<true, true><<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
-  return cudaGetLastError();
 }
 
 cudaError_t launch_row_stats(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws) {
-  const int64_t jobs = (int64_t)sz.N + (b.root_emb ? sz.G : 0);
-  if (jobs == 0) return cudaSuccess;
-  int64_t blocks = (jobs * 32 + 255) / 256;
+  if (sz.N == 0) return cudaSuccess;
+  int64_t blocks = ((int64_t)sz.N * 32 + 255) / 256;
   const int64_t cap = (int64_t)lc.num_sms * 8;
   if (blocks > cap) blocks = cap;
-  const bool aligned16 = (reinterpret_cast<uintptr_t>(b.emb) & 15u) == 0 && sz.stride % 8 == 0 && sz.d % 8 == 0;
-  if (b.emb_dtype == GPO_EMB_BF16 && aligned16 && sz.d <= 8 * 32 * 8 && !b.parent) {  // chain layout: p(v) = v - 1
-    int64_t rblocks = ((int64_t)sz.N + 255) / 256;  // a warp per 32 rows
-    if (rblocks < 1) rblocks = 1;
-    if (rblocks > (int64_t)lc.num_sms * 8) rblocks = (int64_t)lc.num_sms * 8;
-    if (sz.d <= 8 * 32 * 4)
-      row_stats_run_kernel<4><<<(int)rblocks, 256, 0, lc.stream>>>(b, sz, ws);
-    else
-      row_stats_run_kernel<8><<<(int)rblocks, 256, 0, lc.stream>>>(b, sz, ws);
-  } else if (b.emb_dtype == GPO_EMB_BF16)
-    row_stats_kernel<true, false><<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
-  else
-    row_stats_kernel<false, false><<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
+  const bool vec = (reinterpret_cast<uintptr_t>(b.emb) & 15u) == 0 && sz.stride % 8 == 0 && sz.d % 8 == 0;
+  if (b.emb_dtype == GPO_EMB_BF16) {
+    if (vec) row_stats_kernel<true, true><<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
+    else row_stats_kernel<true, false><<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
+  } else {
+    if (vec) row_stats_kernel<false, true><<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
+    else row_stats_kernel<false, false><<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
+  }
   return cudaGetLastError();
 }
 
@@ -607,85 +452,6 @@ __device__ __forceinline__ int upper_idx(const int32_t* off, int n, int v) {  //
     else hi = mid - 1;
   }
   return lo;
-}
-
-template <bool kBf16>
-__device__ __forceinline__ void exact_pair_sums(const void* base, int64_t zrow, const void* pbase, int64_t prow,
-                                                bool has_p, int d, int lane, float2& n2, float2& dot) {
-  float nh = 0.f, nl = 0.f, dh = 0.f, dl = 0.f;
-  constexpr int kVec = kBf16 ? 8 : 4;  // elements per 16-byte chunk
-  const int nvec = d / kVec;
-  for (int c = lane; c < nvec; c += 32) {
-    float x[kVec], y[kVec];
-    if (kBf16) {
-      const uint4 u = *reinterpret_cast<const uint4*>(reinterpret_cast<const uint16_t*>(base) + zrow + 8 * c);
-      const uint32_t w[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        x[2 * i] = __uint_as_float(w[i] << 16);
-        x[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
-      }
-      if (has_p) {
-        const uint4 v = *reinterpret_cast<const uint4*>(reinterpret_cast<const uint16_t*>(pbase) + prow + 8 * c);
-        const uint32_t q[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          y[2 * i] = __uint_as_float(q[i] << 16);
-          y[2 * i + 1] = __uint_as_float(q[i] & 0xFFFF0000u);
-        }
-      }
-    } else {
-      const float4 u = *reinterpret_cast<const float4*>(reinterpret_cast<const float*>(base) + zrow + 4 * c);
-      x[0] = u.x; x[1] = u.y; x[2] = u.z; x[3] = u.w;
-      if (has_p) {
-        const float4 v = *reinterpret_cast<const float4*>(reinterpret_cast<const float*>(pbase) + prow + 4 * c);
-        y[0] = v.x; y[1] = v.y; y[2] = v.z; y[3] = v.w;
-      }
-    }
-#pragma unroll
-    for (int i = 0; i < kVec; ++i) {
-      const float sq = x[i] * x[i];
-      ff_acc(nh, nl, sq);
-      if (!kBf16) nl += fmaf(x[i], x[i], -sq);  // TwoProduct error (bf16 squares are exact)
-      if (has_p) {
-        const float pr = x[i] * y[i];
-        ff_acc(dh, dl, pr);
-        if (!kBf16) dl += fmaf(x[i], y[i], -pr);
-      }
-    }
-  }
-  for (int k = nvec * kVec + lane; k < d; k += 32) {  // ragged tail of the row
-    const float x = kBf16 ? __uint_as_float((uint32_t)(reinterpret_cast<const uint16_t*>(base)[zrow + k]) << 16)
-                          : reinterpret_cast<const float*>(base)[zrow + k];
-    const float sq = x * x;
-    ff_acc(nh, nl, sq);
-    nl += fmaf(x, x, -sq);
-    if (has_p) {
-      const float y = kBf16 ? __uint_as_float((uint32_t)(reinterpret_cast<const uint16_t*>(pbase)[prow + k]) << 16)
-                            : reinterpret_cast<const float*>(pbase)[prow + k];
-      const float pr = x * y;
-      ff_acc(dh, dl, pr);
-      dl += fmaf(x, y, -pr);
-    }
-  }
-  // combine the lanes' pairs (fixed butterfly order: deterministic)
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const float a = __shfl_xor_sync(0xffffffffu, nh, o), b = __shfl_xor_sync(0xffffffffu, nl, o);
-    const float c = __shfl_xor_sync(0xffffffffu, dh, o), e = __shfl_xor_sync(0xffffffffu, dl, o);
-    float s, t;
-    two_sum(nh, a, s, t);
-    nh = s;
-    nl = nl + b + t;
-    two_sum(dh, c, s, t);
-    dh = s;
-    dl = dl + e + t;
-  }
-  float h, l;
-  two_sum(nh, nl, h, l);
-  n2 = make_float2(h, l);
-  two_sum(dh, dl, h, l);
-  dot = make_float2(h, l);
 }
 
 template <bool kBf16>
@@ -748,9 +514,142 @@ __global__ void __launch_bounds__(256) exact_stats_kernel(gpo_batch b, Sizes sz,
   }
 }
 
+// bf16 rows (16-byte aligned, d a multiple of 32): a warp takes 8 consecutive rows, lane
+// 4 r + j summing quarter j of row base + r in 16-byte chunks, four chunks in flight.  In the
+// chain layout the parent of a row is the row before, whose chunk the lane 4 below already
+// holds (a shuffle); the first row's parent chunk, a tree parent or a prompt embedding is
+// loaded.  Compensated sums per lane, two fp32 lanes per instruction (f2_acc), then a fixed
+// butterfly over the 4 quarters: the accuracy of exact_stats_kernel with every row read once.
+__global__ void __launch_bounds__(256) exact_stats_lane_kernel(gpo_batch b, Sizes sz, Ws ws) {
+  const int lane = threadIdx.x & 31, r = lane >> 2, j = lane & 3;
+  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  const bool tree = b.parent != nullptr;
+  const int nq = sz.d / 32;          // 16-byte chunks per quarter
+  const int64_t rs = sz.stride / 8;  // row stride in 16-byte chunks
+  const uint4* Z = reinterpret_cast<const uint4*>(b.emb);
+  const uint4* RZ = reinterpret_cast<const uint4*>(b.root_emb);
+  int v0 = 0, v1 = sz.N;  // states of groups [g0, g1)
+  if (sz.g0 != 0 || sz.g1 != sz.G) {
+    if (tree) {
+      v0 = b.group_state_off[sz.g0];
+      v1 = b.group_state_off[sz.g1];
+    } else {
+      const int ra = b.group_rollout_off[sz.g0], rb = b.group_rollout_off[sz.g1];
+      v0 = ra >= 0 && ra <= sz.R ? b.rollout_step_off[ra] : 0;
+      v1 = rb >= 0 && rb <= sz.R ? b.rollout_step_off[rb] : 0;
+    }
+    v0 = max(0, min(v0, sz.N));
+    v1 = max(v0, min(v1, sz.N));
+  }
+  auto finish4 = [&](uint64_t s, uint64_t e) -> float2 {  // the 4 quarters' pairs, fixed order
+    float2 P = f2_finish(s, e);
+#pragma unroll
+    for (int o = 1; o < 4; o <<= 1) {
+      const float a = __shfl_xor_sync(0xffffffffu, P.x, o), c = __shfl_xor_sync(0xffffffffu, P.y, o);
+      float t, u;
+      two_sum(P.x, a, t, u);
+      P.x = t;
+      P.y = P.y + c + u;
+    }
+    float h, l;
+    two_sum(P.x, P.y, h, l);
+    return make_float2(h, l);
+  };
+  for (int64_t base = v0 + warp * 8; base < v1; base += nwarps * 8) {
+    const int64_t v = base + r;
+    const bool live = v < v1;
+    // parent: p >= 0 a state row, -2 - g the prompt embedding of group g, -1 none
+    int p = -1;
+    if (live) {
+      int g = -1;
+      if (tree) {
+        if (sz.G > 0) {
+          g = upper_idx(b.group_state_off, sz.G, (int)v);
+          const int s0 = b.group_state_off[g], pl = b.parent[v];
+          if (pl >= 0 && s0 >= 0 && (int64_t)s0 + pl < v) p = s0 + pl;
+        }
+      } else if (sz.R > 0) {
+        const int ro = upper_idx(b.rollout_step_off, sz.R, (int)v);
+        if (v > b.rollout_step_off[ro]) p = (int)v - 1;
+        else if (sz.G > 0) g = upper_idx(b.group_rollout_off, sz.G, ro);
+      }
+      if (p < 0 && b.root_emb && g >= 0) p = -2 - g;
+    }
+    // the parent chunk comes from the lane 4 below when it holds the parent's row
+    const bool from_left = p >= 0 && p == v - 1 && r > 0;
+    const uint4* pb = p >= 0 ? Z + (int64_t)p * rs : (p <= -2 ? RZ + (int64_t)(-2 - p) * rs : nullptr);
+    const uint4* zb = Z + (live ? v : base) * rs;
+    uint64_t ns = 0ull, ne = 0ull, ds = 0ull, de = 0ull;
+    constexpr int kU = 4;  // chunks loaded ahead of their arithmetic (memory-level parallelism)
+    for (int c0 = 0; c0 < nq; c0 += kU) {
+      uint4 x[kU], y[kU];
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        const int k = j * nq + c0 + u;
+        x[u] = live && c0 + u < nq ? zb[k] : make_uint4(0u, 0u, 0u, 0u);
+        y[u] = (!from_left && pb && c0 + u < nq) ? pb[k] : make_uint4(0u, 0u, 0u, 0u);
+      }
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        uint4 t;
+        t.x = __shfl_up_sync(0xffffffffu, x[u].x, 4);
+        t.y = __shfl_up_sync(0xffffffffu, x[u].y, 4);
+        t.z = __shfl_up_sync(0xffffffffu, x[u].z, 4);
+        t.w = __shfl_up_sync(0xffffffffu, x[u].w, 4);
+        if (from_left) y[u] = t;
+        const uint32_t xw[4] = {x[u].x, x[u].y, x[u].z, x[u].w}, yw[4] = {y[u].x, y[u].y, y[u].z, y[u].w};
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+          const uint64_t xx = bf16x2_f32x2(xw[h]), yy = bf16x2_f32x2(yw[h]);
+          f2_acc(ns, ne, f2mul(xx, xx));  // bf16 products are exact in fp32
+          f2_acc(ds, de, f2mul(xx, yy));
+        }
+      }
+    }
+    const float2 n2 = finish4(ns, ne);
+    float2 dot = finish4(ds, de);
+    if (p == -1) dot = make_float2(0.f, 0.f);
+    if (live && j == 0) {
+      if (!isfinite(n2.x) || !isfinite(dot.x)) report(ws.status, GPO_ERR_NONFINITE, 3, (int)v);
+      ws.x_n2[v] = n2;
+      ws.x_dot[v] = dot;
+    }
+  }
+}
+
+// |prompt embedding|^2 of groups [g0, g1), one warp each (the streamed kernel covers the states).
+__global__ void __launch_bounds__(256) root_norms_kernel(gpo_batch b, Sizes sz, Ws ws) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t g = sz.g0 + warp; g < sz.g1; g += nwarps) {
+    float2 n2, dot;
+    exact_pair_sums<true>(b.root_emb, g * sz.stride, nullptr, 0, false, sz.d, lane, n2, dot);
+    if (lane == 0) {
+      if (!isfinite(n2.x)) report(ws.status, GPO_ERR_NONFINITE, 3, (int)(sz.N + g));
+      ws.x_root_n2[g] = n2;
+    }
+  }
+}
+
 cudaError_t launch_exact_stats(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws) {
   const int64_t jobs = (int64_t)sz.N + (b.root_emb ? sz.G : 0);  // at most (range calls take fewer)
   if (jobs == 0) return cudaSuccess;
+  const bool aligned16 = (reinterpret_cast<uintptr_t>(b.emb) & 15u) == 0 && sz.stride % 8 == 0 && sz.d % 8 == 0 &&
+                         (!b.root_emb || (reinterpret_cast<uintptr_t>(b.root_emb) & 15u) == 0);
+  if (b.emb_dtype == GPO_EMB_BF16 && aligned16 && sz.d % 32 == 0) {
+    int64_t blocks = ((int64_t)sz.N + 63) / 64;  // a warp per 8 rows
+    const int64_t bcap = (int64_t)lc.num_sms * 32;
+    blocks = blocks < 1 ? 1 : (blocks > bcap ? bcap : blocks);
+    exact_stats_lane_kernel<<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
+    if (b.root_emb && sz.g1 > sz.g0) {
+      int64_t rblocks = ((int64_t)(sz.g1 - sz.g0) + 7) / 8;
+      if (rblocks > (int64_t)lc.num_sms * 8) rblocks = (int64_t)lc.num_sms * 8;
+      root_norms_kernel<<<(int)rblocks, 256, 0, lc.stream>>>(b, sz, ws);
+    }
+    return cudaGetLastError();
+  }
   int64_t blocks = (jobs + 7) / 8;  // a warp per row
   const int64_t cap = (int64_t)lc.num_sms * 16;
   if (blocks > cap) blocks = cap;

@@ -8,9 +8,9 @@
 // Work items: per 128-row block of a group, a diagonal item (the block against
 // itself) and off-diagonal items (the block against up to 256 later columns), so
 // each unordered pair is visited once.  A group's diagonal items precede its
-// off-diagonal ones in the list.  A diagonal item takes the block's norms from the
-// diagonal of its Gram tile (|z_i|^2, and <z_i, z_{i+1}> from the super-diagonal),
-// writes them to the workspace and raises the block's ready flag; an off-diagonal
+// off-diagonal ones in the list.  A diagonal item takes the block's squared norms from
+// the diagonal of its Gram tile (for the threshold test; eta uses the compensated
+// statistics), writes them to the workspace and raises the block's ready flag; an off-diagonal
 // item waits (bounded) for the flags of its row and column blocks before its
 // epilogue reads them.  Every wait is on an item earlier in the list, diagonal items
 // never wait, and each CTA takes its items in list order, so every wait ends.
@@ -56,7 +56,6 @@ struct __align__(8) SmemCtl {
   int overflow;                    // some warp found more pairs than its list holds
   int lp[kSlots];                  // label forest of the item's slots (rows, then columns)
   int cm_depth[kTileN];
-  int cm_par[kTileN];              // tree layout: parent (global) of each column state
   alignas(16) float cm_rn[kTileN];  // 1 / |z| of the item's columns
   uint32_t elist[kEpiWarps][kWarpEdges];  // slot pairs (row slot | column slot << 16)
 };
@@ -248,7 +247,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       epi_sync();  // previous item finished with the metadata, lists and forest
       for (int c = te; c < item.ncols; c += kEpiThreads) {
         ctl->cm_depth[c] = ws.state_meta[item.col0 + c].y;
-        if (tree) ctl->cm_par[c] = ws.tree_par[item.col0 + c];
       }
       for (int c = item.ncols + te; c < kTileN; c += kEpiThreads) ctl->cm_rn[c] = 0.f;
       if (te == 0) {
@@ -285,31 +283,23 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (epi_any(!got)) break;
       tc_fence_after();
       if (diag) {
-        // the block's norms: diagonal and super-diagonal of its Gram tile, read by one warp
-        // per lane quarter; published before the flag that releases the block
+        // the block's squared norms (threshold test): the diagonal of its Gram tile, read by
+        // one warp per lane quarter; published before the flag that releases the block
         if (rep == 0 && q * 32 < item.ncols) {
           const uint32_t base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * kTileN + q * 32);
           uint32_t r[32];
           tmem_ld_32x32b_x32(base, r);
           tmem_wait_ld();
-          float dg = 0.f, up = 0.f;
+          float dg = 0.f;
 #pragma unroll
-          for (int k = 0; k < 32; ++k) {
+          for (int k = 0; k < 32; ++k)
             if (k == lane) dg = __uint_as_float(r[k]);
-            if (k == lane + 1) up = __uint_as_float(r[k]);
-          }
-          if (q * 32 + 32 < item.ncols) {
-            tmem_ld_32x32b_x32(base + 32u, r);
-            tmem_wait_ld();
-            if (lane == 31) up = __uint_as_float(r[0]);
-          }
           if (t < item.ncols) {
             const float rni = dg > 0.f ? 1.0f / sqrtf(dg) : 0.f;
             ws.nrm2[row] = dg;
             ws.rn[row] = rni;
             ctl->cm_rn[t] = rni;
             if (!isfinite(dg)) report(st, GPO_ERR_NONFINITE, 1, row);
-            if (!tree && t + 1 < item.ncols && ctl->cm_depth[t + 1] > 1) ws.dotp[row + 1] = up;
           }
           __threadfence();
         }
@@ -332,17 +322,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_wait_ld();
         // <z of the block's last row, z of the next block's first row>: the parent dot of
         // the next block's first state when it continues the same rollout
-        if (!tree && ch == 0 && q == 3 && lane == 31 && item.col0 == item.row0 + kTileM && ctl->cm_depth[0] > 1)
-          ws.dotp[item.col0] = __uint_as_float(r[0]);
-        if (tree) {
-          // tree layout: <z_{p(v)}, z_v> of every child v of this row in the chunk (each
-          // (parent, child) pair lies in exactly one item's upper part)
-#pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            const int c = ch * 32 + j;
-            if (c < item.ncols && ctl->cm_par[c] == row) ws.dotp[item.col0 + c] = __uint_as_float(r[j]);
-          }
-        }
         uint32_t mp[4] = {0u, 0u, 0u, 0u};
         const float4* rn4 = reinterpret_cast<const float4*>(ctl->cm_rn + ch * 32);
 #pragma unroll
