@@ -454,6 +454,20 @@ __device__ __forceinline__ int upper_idx(const int32_t* off, int n, int v) {  //
   return lo;
 }
 
+// The same as upper_idx, for a value common to the warp: rounds of 32 probes (one
+// coalesced load per round, log32(n) rounds) instead of log2(n) dependent loads.
+__device__ __forceinline__ int warp_upper_idx(const int32_t* off, int n, int v, int lane) {
+  int lo = 0, hi = n;  // the answer lies in [lo, hi)
+  while (hi - lo > 1) {
+    const int step = (hi - lo + 31) / 32;  // probes at lo, lo + step, ...
+    const int k = lo + lane * step;
+    const uint32_t m = __ballot_sync(0xffffffffu, k < hi && off[k] <= v);
+    lo += (m ? 31 - __clz(m) : 0) * step;
+    hi = min(hi, lo + step);
+  }
+  return lo;
+}
+
 template <bool kBf16>
 __global__ void __launch_bounds__(256) exact_stats_kernel(gpo_batch b, Sizes sz, Ws ws) {
   const int lane = threadIdx.x & 31;
@@ -559,20 +573,38 @@ __global__ void __launch_bounds__(256) exact_stats_lane_kernel(gpo_batch b, Size
   for (int64_t base = v0 + warp * 8; base < v1; base += nwarps * 8) {
     const int64_t v = base + r;
     const bool live = v < v1;
+    // the rollout (chain) or group (tree) of the warp's first row by a 32-ary search, then each
+    // row's from a window of 32 offsets and one ballot per row
+    const int32_t* off = tree ? b.group_state_off : b.rollout_step_off;
+    const int cnt = tree ? sz.G : sz.R;
+    int k_row = 0, start = 0;
+    if (cnt > 0) {
+      const int k0 = warp_upper_idx(off, cnt, (int)base, lane);
+      const int win = k0 + lane < cnt ? off[k0 + lane] : 0x7fffffff;
+      for (int q = 0; q < 8; ++q) {
+        const int vq = (int)min(base + q, (int64_t)v1 - 1);
+        const uint32_t m = __ballot_sync(0xffffffffu, win <= vq);
+        int k = k0 + (m ? 31 - __clz(m) : 0);
+        if (m == 0xffffffffu)
+          while (k + 1 < cnt && off[k + 1] <= vq) ++k;
+        const int st_k = k - k0 < 32 ? __shfl_sync(0xffffffffu, win, (k - k0) & 31) : off[k];
+        if (q == r) {
+          k_row = k;
+          start = st_k;
+        }
+      }
+    }
     // parent: p >= 0 a state row, -2 - g the prompt embedding of group g, -1 none
     int p = -1;
-    if (live) {
+    if (live && cnt > 0) {
       int g = -1;
       if (tree) {
-        if (sz.G > 0) {
-          g = upper_idx(b.group_state_off, sz.G, (int)v);
-          const int s0 = b.group_state_off[g], pl = b.parent[v];
-          if (pl >= 0 && s0 >= 0 && (int64_t)s0 + pl < v) p = s0 + pl;
-        }
-      } else if (sz.R > 0) {
-        const int ro = upper_idx(b.rollout_step_off, sz.R, (int)v);
-        if (v > b.rollout_step_off[ro]) p = (int)v - 1;
-        else if (sz.G > 0) g = upper_idx(b.group_rollout_off, sz.G, ro);
+        g = k_row;
+        const int pl = b.parent[v];
+        if (pl >= 0 && start >= 0 && (int64_t)start + pl < v) p = start + pl;
+      } else {
+        if (v > start) p = (int)v - 1;
+        else if (b.root_emb && sz.G > 0) g = upper_idx(b.group_rollout_off, sz.G, k_row);
       }
       if (p < 0 && b.root_emb && g >= 0) p = -2 - g;
     }
