@@ -56,7 +56,7 @@ _OUT_FIELDS = [
     ("root_score", np.float64, "G"), ("eta", np.float64, "N"), ("step_reward", np.float64, "N"),
     ("a_cor", np.float64, "N"), ("a_eff_node", np.float64, "N"), ("e_eff", np.float64, "N"),
     ("edge_adv", np.float64, "N"), ("edge_eff_mask", np.uint8, "N"),
-    ("cor_group_size", np.int32, "N"),
+    ("cor_group_size", np.int32, "N"), ("eff_tree", np.float64, "G"), ("eff_graph", np.float64, "G"),
 ]
 
 

@@ -18,6 +18,12 @@
  *             to every generated edge on the route a_Q -> v.
  *   Sec. 4.5  A_dual(e) = A_cor(e) + lambda_eff * A_eff(e); every token of an
  *             edge carries the edge's advantage.
+ *   Eq. (eq1) exploration efficiency Eff = (tokens of correct steps) / (tokens of
+ *             all steps); a step (p(v), v) is correct when a correct final
+ *             answer can be reached from v: along direct edges (tree reading,
+ *             c_own(v) > 0; in the chain layout this is the paper's chain case,
+ *             the whole trajectory counted as one step), or along direct edges
+ *             and equivalences of the merged graph (graph reading).
  *
  * The same definitions serve both input layouts (oracle.h): in the chain layout
  * every rollout is a path from the root, in the tree layout the provenance
@@ -230,10 +236,11 @@ static int run_group(const oracle_batch* b, const oracle_params* p, oracle_outpu
   int* cnt = malloc(sizeof(int) * n);
   int* tmp = malloc(sizeof(int) * n);
   double* xs = malloc(sizeof(double) * n);
+  unsigned char* reach = calloc(n, 1);
   if (!G.parent || !G.depth || !G.rollout || !G.terminal || !G.child_off || !G.child_list ||
       !G.z || !G.nrm || !G.adj || !G.label || !G.mem_off || !G.mem_list || !c_own || !t_own ||
       !S || !eta || !r || !a_cor || !gsize || !a_eff || !e_eff || !emask || !queue || !order ||
-      !cnt || !tmp || !xs)
+      !cnt || !tmp || !xs || !reach)
     return ORACLE_ERR_NOMEM; /* the process is about to fail anyway; no cleanup */
 
   /* --- the rollout graph: root v0 plus one node per generated step (Sec. 4.2) --- */
@@ -405,6 +412,38 @@ static int run_group(const oracle_batch* b, const oracle_params* p, oracle_outpu
     }
   }
 
+  /* --- exploration efficiency, Eq. (eq1) --- */
+  if (o->eff_tree || o->eff_graph) {
+    /* graph reading: a class reaches a correct answer if one of its members is a correct
+       terminal, or a member has a child whose class reaches one; breadth-first search
+       backwards over the quotient graph's edges class(child) -> class(parent) */
+    int qh = 0, qt = 0;
+    for (int i = 1; i < n; ++i)
+      if (G.terminal[i] && b->reward[G.rollout[i]] && !reach[G.label[i]]) {
+        reach[G.label[i]] = 1;
+        queue[qt++] = G.label[i];
+      }
+    while (qh < qt) {
+      const int L = queue[qh++];
+      for (int i = 1; i < n; ++i) {
+        const int u = G.parent[i];
+        if (G.label[i] == L && u > 0 && !reach[G.label[u]]) {
+          reach[G.label[u]] = 1;
+          queue[qt++] = G.label[u];
+        }
+      }
+    }
+    double tok = 0.0, good_tree = 0.0, good_graph = 0.0;
+    for (int i = 1; i < n; ++i) {
+      const double len = (double)b->step_len[s0 + i - 1];
+      tok += len;
+      if (c_own[i] > 0.0) good_tree += len; /* a correct terminal lies below v */
+      if (reach[G.label[i]]) good_graph += len;
+    }
+    if (o->eff_tree) o->eff_tree[g] = tok > 0.0 ? good_tree / tok : 0.0;
+    if (o->eff_graph) o->eff_graph[g] = tok > 0.0 ? good_graph / tok : 0.0;
+  }
+
   /* --- outputs: per state / edge, then every token of the edge (Sec. 4.5) --- */
   if (o->root_score) o->root_score[g] = S[0];
   for (int i = 1; i < n; ++i) {
@@ -442,7 +481,7 @@ static int run_group(const oracle_batch* b, const oracle_params* p, oracle_outpu
   free(G.child_list); free(G.z); free(G.nrm); free(G.adj); free(G.label); free(G.mem_off);
   free(G.mem_list); free(c_own); free(t_own); free(S); free(eta); free(r); free(a_cor);
   free(gsize); free(a_eff); free(e_eff); free(emask); free(queue); free(order); free(cnt);
-  free(tmp); free(xs);
+  free(tmp); free(xs); free(reach);
   return ORACLE_OK;
 }
 

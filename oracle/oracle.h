@@ -92,6 +92,9 @@ typedef struct {
   double* edge_adv;       /* [N] A_dual of edge (p(v), v) */
   uint8_t* edge_eff_mask; /* [N] */
   int32_t* cor_group_size;/* [N] size of the correctness group holding the edge */
+  double* eff_tree;       /* [G] exploration efficiency Eff, Eq. (eq1): a step is correct when a
+                             correct terminal is reachable from it along direct edges */
+  double* eff_graph;      /* [G] the same with reachability in the merged (quotient) graph */
 } oracle_outputs;
 
 /* Runs the whole path on `num_threads` host threads (groups are independent).

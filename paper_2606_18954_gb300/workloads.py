@@ -495,3 +495,34 @@ def summary(batch: dict) -> dict:
     return dict(groups=G, rollouts=R, states=N, tokens=T, d=int(batch["emb"].shape[1]),
                 dtype=batch["emb_dtype"], max_states_per_group=max(ng) if ng else 0,
                 mean_states_per_group=(sum(ng) / G) if G else 0.0)
+
+
+# ---- per-token log-probabilities for the policy loss (GraphPO Sec. 4.5) -------------
+#
+# Recipe (seed 20261202 + 100 + k by default): old log-probs -|N(0, 1.5)| - 0.01 (a
+# sampled token's log-probability under the behaviour policy), new log-probs = old +
+# N(0, 0.15) (a policy a few optimiser steps later: about a fifth of the tokens leave
+# the clip range [0.8, 1.2]), reference log-probs = new + N(0, 0.1); all float32.
+# Margin: tokens whose ratio exp(new - old) (fp64 on the float32 values) lies within
+# 1e-4 of a clip bound are redrawn, so that the clip decision is unambiguous in fp32.
+LOGP_SEED_OFFSET = 100
+
+
+def make_logprobs(T: int, seed: int, clip_low: float = 0.2, clip_high: float = 0.2, margin: float = 1e-4,
+                  spread: float = 0.15) -> dict:
+    rng = np.random.default_rng(seed)
+    old = (-np.abs(rng.normal(0.0, 1.5, T)) - 0.01).astype(np.float32)
+    new = (old.astype(np.float64) + rng.normal(0.0, spread, T)).astype(np.float32)
+    bounds = (1.0 - clip_low, 1.0 + clip_high)
+    for _ in range(100):
+        r = np.exp(new.astype(np.float64) - old.astype(np.float64))
+        bad = np.zeros(T, dtype=bool)
+        for c in bounds:
+            bad |= np.abs(r - c) < margin
+        if not bad.any():
+            break
+        new[bad] = (old[bad].astype(np.float64) + rng.normal(0.0, spread, int(bad.sum()))).astype(np.float32)
+    else:
+        raise RuntimeError("log-prob margin filter did not converge")
+    ref = (new.astype(np.float64) + rng.normal(0.0, 0.1, T)).astype(np.float32)
+    return dict(logp=new, old_logp=old, ref_logp=ref)
