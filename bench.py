@@ -228,6 +228,42 @@ def cpu_baseline(b, budget_s=6.0, max_groups=None):
             "graphs_per_s": (len(sub["group_rollout_off"]) - 1) / t}
 
 
+def time_token_loss(P, gp, b, db, alg, flush, stream, args):
+    """The policy loss (GraphPO Sec. 4.5 objective, dual form, edge normalisation, no KL term)
+    on the batch's per-edge A_dual from the path and seeded log-probabilities, timed like the
+    path (L2 flushed before every launch, CUDA events on the launching stream).  Algorithmic
+    bytes per launch: log-probs, old log-probs and the gradient (12 bytes per token) plus
+    every edge's first token, weight and advantage (16 bytes per edge)."""
+    import torch
+    from paper_2606_18954_gb300 import workloads as W
+    T, N = alg["T"], alg["N"]
+    nodes = gp.alloc_outputs(db, nodes=True)
+    gp.compute_into(db, nodes, stream=stream)
+    lp = W.make_logprobs(T, W.BASE_SEED + W.LOGP_SEED_OFFSET)
+    logp = torch.from_numpy(lp["logp"]).to(db.step_len.device)
+    old = torch.from_numpy(lp["old_logp"]).to(db.step_len.device)
+    plan = gp.loss_plan(db, stream=stream)
+    out = None
+    for _ in range(args.warmup):
+        out = gp.token_loss(db, plan, logp, old, edge_adv=nodes["edge_adv"], out=out, stream=stream)
+    gp.check(stream)
+    times = []
+    for _ in range(args.steps):
+        flush.zero_()
+        s = torch.cuda.Event(enable_timing=True)
+        e = torch.cuda.Event(enable_timing=True)
+        s.record(stream)
+        gp.token_loss(db, plan, logp, old, edge_adv=nodes["edge_adv"], out=out, stream=stream)
+        e.record(stream)
+        e.synchronize()
+        times.append(s.elapsed_time(e))
+    gp.check(stream)
+    ms = statistics.mean(times)
+    return {"ms": ms, "tokens_per_s": T / (ms / 1e3), "form": "dual", "norm": "edge", "beta_kl": 0.0,
+            "loss": float(out["loss"].cpu()[0]), "launches_per_step": 1,
+            "bytes": 12 * T + 16 * N}
+
+
 def dist_env():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     return ws, int(os.environ.get("RANK", "0")), int(os.environ.get("LOCAL_RANK", "0"))
@@ -372,6 +408,8 @@ def run_ours(args):
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         e2e_t = float(t.item())
 
+    loss = None if args.no_loss else time_token_loss(P, gp, b, db, alg, flush, stream, args)
+
     if rank != 0:
         return 0
     hbm, tc, tc_sus, peak_src = load_peaks()
@@ -414,6 +452,14 @@ def run_ours(args):
         "clocks": clk.summary(),
         "gpu_launches": nst * args.steps,
     }
+    if loss is not None:
+        lb = loss.pop("bytes")
+        achieved = lb / (loss["ms"] / 1e3) / 1e9
+        traffic, tnote = traffic_for("gpo_loss.cu", args.config)
+        loss["roofline"] = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
+                            "traffic": traffic, "traffic_note": tnote, "algorithmic_bytes": lb,
+                            "peak_source": f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured" else "fallback"}
+        line["token_loss"] = loss
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(b, max_groups={"wide": 2, "full": 64}.get(args.config))
     print(json.dumps(line), flush=True)
@@ -428,6 +474,7 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--config", choices=list(WORKLOADS), default="math")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-loss", action="store_true", help="skip the policy-loss measurement")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)

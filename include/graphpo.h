@@ -145,6 +145,18 @@ typedef struct {
   int32_t* class_id;  /* [N] optional: smallest state index of the state's class */
   float* node_score;  /* [N] optional: pooled score S(v) */
   float* edge_adv;    /* [N] optional: A_dual of the edge entering each state */
+  /* Per-edge components, the inputs of the split loss form (gpo_token_loss): */
+  float* edge_cor;       /* [N] optional: A_cor of the edge entering each state */
+  float* edge_eff;       /* [N] optional: efficiency advantage routed through that edge (no lambda) */
+  uint8_t* edge_eff_mask;/* [N] optional: 1 where some route a_Q -> v covers that edge */
+  /* Exploration efficiency, GraphPO Eq. (eq1): tokens of the steps from which a correct
+   * final answer can be reached / tokens of all steps of the group (0 for a group without
+   * states).  Tree reading: a correct terminal lies below the step's state (c_own > 0; in
+   * the chain layout: the rollout is correct, each trajectory counted as one step).  Graph
+   * reading: reachable along direct edges and through merged states (a class reaches a
+   * correct answer when a member is, or has a child whose class is, such a state). */
+  float* group_eff;       /* [G] optional: tree reading */
+  float* group_eff_graph; /* [G] optional: graph reading */
 } gpo_outputs;
 
 typedef struct gpo_ctx gpo_ctx;
@@ -219,6 +231,83 @@ gpo_status gpo_stage_times(gpo_ctx* ctx, float* ms, const char** names, int capa
  * behave as for gpo_compute. */
 #define GPO_NOALLOC_SCRATCH_BYTES ((size_t)32 << 20)
 gpo_status gpo_compute_noalloc(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* out, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * Policy loss on per-token log-probabilities (GraphPO Sec. 4.5: the objective
+ * J_GraphPO, DAPO's clipped surrogate on the graph advantage averaged over each
+ * edge's tokens and each prompt graph's edges; Algorithm S.1 Stage 4: the split
+ * form with separate correctness and efficiency terms).  The paper has no
+ * counterpart of the plan; the loss itself is what a trainer minimises after
+ * gpo_compute, once per optimiser step.
+ *
+ *   J = 1/G' sum_g 1/|E_g| sum_{e in E_g} 1/|e| sum_{t in e} (f_t - beta k_t)
+ *                                                       (GPO_LOSS_NORM_EDGE)
+ *   J = 1/T sum_t (f_t - beta k_t)                      (GPO_LOSS_NORM_TOKEN: DAPO's token mean)
+ *   phi(A) = min(r_t A, clip(r_t, 1 - clip_low, 1 + clip_high) A),
+ *   r_t = exp(logp_t - old_logp_t)
+ *   dual form:  f_t = phi(A_dual(e))                      (gpo_outputs.edge_adv)
+ *   split form: f_t = phi(A_cor(e)) + lambda_eff m_eff(e) phi(A_eff(e))
+ *               (gpo_outputs.edge_cor, edge_eff, edge_eff_mask)
+ *   k_t = exp(x) - x - 1, x = ref_logp_t - logp_t (the k3 estimate of KL(pi_theta || pi_ref))
+ *   loss = -J;  grad_logp[t] = d loss / d logp_t, taken where the min picks the
+ *   unclipped term (r A <= clip(r) A) and 0 where the clipped term is smaller
+ *
+ * G' = groups with at least one state, |E_g| = the states of group g (one direct
+ * edge enters each state), |e| = step_len of the edge's state, e the edge holding
+ * token t in the batch's token layout (that of gpo_compute's per-token outputs).
+ * The entropy bonus of Algorithm S.1 needs the whole vocabulary distribution and
+ * is left to the caller.
+ */
+typedef enum { GPO_LOSS_DUAL = 0, GPO_LOSS_SPLIT = 1 } gpo_loss_form;
+typedef enum { GPO_LOSS_NORM_EDGE = 0, GPO_LOSS_NORM_TOKEN = 1 } gpo_loss_norm;
+
+typedef struct {
+  double clip_low;   /* in [0, 1): lower clip bound 1 - clip_low (the paper: 0.2) */
+  double clip_high;  /* >= 0: upper clip bound 1 + clip_high (the paper: 0.2; DAPO raises it) */
+  double beta_kl;    /* >= 0: weight of the KL estimate (0: ref_logp is not read) */
+  double lambda_eff; /* >= 0: split form's weight of the efficiency term */
+  int32_t form;      /* gpo_loss_form */
+  int32_t norm;      /* gpo_loss_norm */
+} gpo_loss_params;
+
+typedef struct {
+  const float* logp;          /* [T] log pi_theta of every token, 16-byte aligned */
+  const float* old_logp;      /* [T] log pi_theta_old (the sampling policy), 16-byte aligned */
+  const float* ref_logp;      /* [T] log pi_ref, 16-byte aligned; read only when beta_kl > 0 */
+  const float* edge_adv;      /* [N] dual form: A_dual of the edge entering each state */
+  const float* edge_cor;      /* [N] split form: A_cor */
+  const float* edge_eff;      /* [N] split form: routed A_eff (no lambda) */
+  const uint8_t* edge_eff_mask; /* [N] split form: m_eff */
+} gpo_loss_inputs;
+
+#define GPO_LOSS_NSTATS 4
+typedef struct {
+  float* loss;       /* [1] required: -J */
+  float* grad_logp;  /* [T] optional: d loss / d logp, 16-byte aligned */
+  double* stats;     /* [GPO_LOSS_NSTATS] optional: the policy term sum w f, the KL term sum w k
+                        (0 when beta_kl = 0), the number of tokens whose (first) surrogate took
+                        the clipped branch, the token mean of r */
+} gpo_loss_outputs;
+
+/* Bytes of a loss plan for batches of this shape (reads the host-side sizes only). */
+gpo_status gpo_loss_plan_size(const gpo_batch* batch, size_t* bytes);
+
+/* Builds a loss plan (the first token and the weight of every edge, the first edge of
+ * every token tile) from the batch's structure: the offsets and step_len (embeddings and
+ * rewards are not read).  `plan`: device memory of gpo_loss_plan_size bytes, 256-byte
+ * aligned, owned by the caller.  Asynchronous on `stream`; layout errors the kernels find
+ * (as for gpo_compute) are returned by gpo_sync_status, and gpo_token_loss calls on that
+ * plan then leave their outputs unwritten.  A plan serves every gpo_token_loss call on
+ * the same batch structure.  It also holds those calls' reduction scratch: calls that
+ * share a plan must be ordered on the GPU. */
+gpo_status gpo_loss_plan(gpo_ctx* ctx, const gpo_batch* batch, void* plan, size_t plan_bytes, void* stream);
+
+/* Enqueues the loss, its gradient and statistics on `stream` (one kernel; the token
+ * tiles' reductions are combined in a fixed order, so results are deterministic).
+ * Host-checked: parameters, NULL inputs for the chosen form, alignment
+ * (GPO_ERR_UNSUPPORTED), plan size. */
+gpo_status gpo_token_loss(gpo_ctx* ctx, const gpo_batch* batch, void* plan, const gpo_loss_params* params,
+                          const gpo_loss_inputs* in, const gpo_loss_outputs* out, void* stream);
 
 /* Library version string. */
 const char* gpo_version(void);

@@ -53,12 +53,35 @@ class CBatch(ctypes.Structure):
 class COutputs(ctypes.Structure):
     _fields_ = [("adv", ctypes.c_void_p), ("adv_cor", ctypes.c_void_p), ("adv_eff", ctypes.c_void_p),
                 ("eff_mask", ctypes.c_void_p), ("class_id", ctypes.c_void_p),
-                ("node_score", ctypes.c_void_p), ("edge_adv", ctypes.c_void_p)]
+                ("node_score", ctypes.c_void_p), ("edge_adv", ctypes.c_void_p), ("edge_cor", ctypes.c_void_p),
+                ("edge_eff", ctypes.c_void_p), ("edge_eff_mask", ctypes.c_void_p), ("group_eff", ctypes.c_void_p),
+                ("group_eff_graph", ctypes.c_void_p)]
 
+OUTPUT_NAMES = ("adv", "adv_cor", "adv_eff", "eff_mask", "class_id", "node_score", "edge_adv", "edge_cor", "edge_eff",
+                "edge_eff_mask", "group_eff", "group_eff_graph")
+
+
+class LossParams(ctypes.Structure):
+    _fields_ = [("clip_low", ctypes.c_double), ("clip_high", ctypes.c_double), ("beta_kl", ctypes.c_double),
+                ("lambda_eff", ctypes.c_double), ("form", ctypes.c_int32), ("norm", ctypes.c_int32)]
+
+
+class LossInputs(ctypes.Structure):
+    _fields_ = [(k, ctypes.c_void_p) for k in ("logp", "old_logp", "ref_logp", "edge_adv", "edge_cor", "edge_eff",
+                                                "edge_eff_mask")]
+
+
+class LossOutputs(ctypes.Structure):
+    _fields_ = [("loss", ctypes.c_void_p), ("grad_logp", ctypes.c_void_p), ("stats", ctypes.c_void_p)]
+
+
+LOSS_FORMS = {"dual": 0, "split": 1}
+LOSS_NORMS = {"edge": 0, "token": 1}
+LOSS_NSTATS = 4
 
 EXPORTS = ["gpo_create", "gpo_workspace_size", "gpo_compute", "gpo_sync_status", "gpo_status_string",
            "gpo_last_error", "gpo_version", "gpo_destroy", "gpo_enable_timing", "gpo_stage_times", "gpo_compute_noalloc",
-           "gpo_compute_groups"]
+           "gpo_compute_groups", "gpo_loss_plan_size", "gpo_loss_plan", "gpo_token_loss"]
 
 FUSED_MAX_STATES = 384  # largest group the group-resident path (and gpo_compute_groups) serves
 
@@ -111,6 +134,15 @@ def load(build_if_missing: bool = False):
         L.gpo_stage_times.argtypes = [ctypes.c_void_p, ctypes.POINTER(ctypes.c_float),
                                       ctypes.POINTER(ctypes.c_char_p), ctypes.c_int, ctypes.POINTER(ctypes.c_int)]
         L.gpo_stage_times.restype = ctypes.c_int
+        L.gpo_loss_plan_size.argtypes = [ctypes.POINTER(CBatch), ctypes.POINTER(ctypes.c_size_t)]
+        L.gpo_loss_plan_size.restype = ctypes.c_int
+        L.gpo_loss_plan.argtypes = [ctypes.c_void_p, ctypes.POINTER(CBatch), ctypes.c_void_p, ctypes.c_size_t,
+                                    ctypes.c_void_p]
+        L.gpo_loss_plan.restype = ctypes.c_int
+        L.gpo_token_loss.argtypes = [ctypes.c_void_p, ctypes.POINTER(CBatch), ctypes.c_void_p,
+                                     ctypes.POINTER(LossParams), ctypes.POINTER(LossInputs),
+                                     ctypes.POINTER(LossOutputs), ctypes.c_void_p]
+        L.gpo_token_loss.restype = ctypes.c_int
         _lib = L
         return L
 
@@ -121,7 +153,7 @@ def _ptr(t) -> Optional[int]:
 
 def _c_outputs(out: dict) -> COutputs:
     return COutputs(*[_ptr(out.get(k)) if out.get(k) is not None and out[k].numel() else None
-                      for k in ("adv", "adv_cor", "adv_eff", "eff_mask", "class_id", "node_score", "edge_adv")])
+                      for k in OUTPUT_NAMES])
 
 
 @dataclasses.dataclass
@@ -271,10 +303,13 @@ class GraphPO:
             self._ws = torch.empty(max(need, 256), dtype=torch.uint8, device=batch.emb.device)
         return self._ws
 
-    def alloc_outputs(self, batch: Batch, components=False, nodes=False) -> dict:
+    def alloc_outputs(self, batch: Batch, components=False, nodes=False, edges=False, efficiency=False) -> dict:
+        """Output tensors: per-token A_dual always; `components` adds per-token A_cor, A_eff and
+        m_eff; `nodes` class ids, S(v) and per-edge A_dual; `edges` per-edge A_cor, A_eff and
+        m_eff (the split loss form's inputs); `efficiency` Eff per group in both readings."""
         import torch
         dev = batch.emb.device
-        T, N = batch.total_tokens, batch.num_states
+        T, N, G = batch.total_tokens, batch.num_states, batch.num_groups
         out = {"adv": torch.empty(max(T, 1), dtype=torch.float32, device=dev)[:T]}
         if components:
             out["adv_cor"] = torch.empty(max(T, 1), dtype=torch.float32, device=dev)[:T]
@@ -284,6 +319,13 @@ class GraphPO:
             out["class_id"] = torch.empty(max(N, 1), dtype=torch.int32, device=dev)[:N]
             out["node_score"] = torch.empty(max(N, 1), dtype=torch.float32, device=dev)[:N]
             out["edge_adv"] = torch.empty(max(N, 1), dtype=torch.float32, device=dev)[:N]
+        if edges:
+            out["edge_cor"] = torch.empty(max(N, 1), dtype=torch.float32, device=dev)[:N]
+            out["edge_eff"] = torch.empty(max(N, 1), dtype=torch.float32, device=dev)[:N]
+            out["edge_eff_mask"] = torch.empty(max(N, 1), dtype=torch.uint8, device=dev)[:N]
+        if efficiency:
+            out["group_eff"] = torch.empty(max(G, 1), dtype=torch.float32, device=dev)[:G]
+            out["group_eff_graph"] = torch.empty(max(G, 1), dtype=torch.float32, device=dev)[:G]
         return out
 
     def compute_into(self, batch: Batch, out: dict, workspace=None, stream=None) -> None:
@@ -311,9 +353,63 @@ class GraphPO:
         if code != GPO_OK:
             raise GraphPOError(code, self.last_error())
 
-    def __call__(self, batch: Batch, components=False, nodes=False, stream=None) -> dict:
-        out = self.alloc_outputs(batch, components, nodes)
+    def __call__(self, batch: Batch, components=False, nodes=False, edges=False, efficiency=False,
+                 stream=None) -> dict:
+        out = self.alloc_outputs(batch, components, nodes, edges, efficiency)
         self.compute_into(batch, out, stream=stream)
+        return out
+
+    # ---- policy loss (gpo_loss_plan / gpo_token_loss)
+
+    def loss_plan(self, batch: Batch, plan=None, stream=None):
+        """Builds (into `plan`, a uint8 device tensor, allocated if None) the loss plan of the
+        batch's structure and returns it; enqueued on the current stream."""
+        import torch
+        if stream is None:
+            stream = torch.cuda.current_stream(batch.step_len.device)
+        cb = batch.c_struct()
+        n = ctypes.c_size_t()
+        code = self._lib.gpo_loss_plan_size(ctypes.byref(cb), ctypes.byref(n))
+        if code != GPO_OK:
+            raise GraphPOError(code, "gpo_loss_plan_size")
+        if plan is None or plan.numel() < n.value:
+            plan = torch.empty(max(n.value, 256), dtype=torch.uint8, device=batch.step_len.device)
+        code = self._lib.gpo_loss_plan(self._h, ctypes.byref(cb), plan.data_ptr(), plan.numel(),
+                                       ctypes.c_void_p(stream.cuda_stream))
+        if code != GPO_OK:
+            raise GraphPOError(code, self.last_error())
+        return plan
+
+    def token_loss(self, batch: Batch, plan, logp, old_logp, ref_logp=None, edge_adv=None, edge_cor=None,
+                   edge_eff=None, edge_eff_mask=None, clip_low=0.2, clip_high=0.2, beta_kl=0.0, lambda_eff=1.0,
+                   form="dual", norm="edge", grad=True, stats=True, out=None, stream=None) -> dict:
+        """gpo_token_loss: returns {"loss": [1] float32, "grad_logp": [T] float32 (if grad),
+        "stats": [4] float64 (if stats)} as device tensors (or fills `out`)."""
+        import torch
+        dev = logp.device
+        if stream is None:
+            stream = torch.cuda.current_stream(dev)
+        T = batch.total_tokens
+        if out is None:
+            out = {"loss": torch.empty(1, dtype=torch.float32, device=dev)}
+            if grad:
+                out["grad_logp"] = torch.empty(max(T, 4), dtype=torch.float32, device=dev)[:T]
+            if stats:
+                out["stats"] = torch.empty(LOSS_NSTATS, dtype=torch.float64, device=dev)
+        lp = LossParams(float(clip_low), float(clip_high), float(beta_kl), float(lambda_eff), LOSS_FORMS[form],
+                        LOSS_NORMS[norm])
+
+        def pt(t):
+            return None if t is None or t.numel() == 0 else t.data_ptr()
+
+        li = LossInputs(pt(logp), pt(old_logp), pt(ref_logp), pt(edge_adv), pt(edge_cor), pt(edge_eff),
+                        pt(edge_eff_mask))
+        lo = LossOutputs(pt(out["loss"]), pt(out.get("grad_logp")), pt(out.get("stats")))
+        cb = batch.c_struct()
+        code = self._lib.gpo_token_loss(self._h, ctypes.byref(cb), plan.data_ptr(), ctypes.byref(lp),
+                                        ctypes.byref(li), ctypes.byref(lo), ctypes.c_void_p(stream.cuda_stream))
+        if code != GPO_OK:
+            raise GraphPOError(code, self.last_error())
         return out
 
     def enable_timing(self, on: bool = True) -> None:

@@ -252,7 +252,7 @@ gpo_status gpo_create(gpo_ctx** out, const gpo_params* params) {
     }
   }
   if (setup_sim_tc() != cudaSuccess || setup_groups() != cudaSuccess || setup_fused() != cudaSuccess ||
-      setup_tree_prep() != cudaSuccess ||
+      setup_tree_prep() != cudaSuccess || setup_loss() != cudaSuccess ||
       cudaMallocHost(&c->host_status, sizeof(uint32_t) * kStatusWords) != cudaSuccess) {
     cudaGetLastError();
     delete c;
@@ -409,6 +409,182 @@ gpo_status gpo_compute_groups(gpo_ctx* ctx, const gpo_batch* batch, const gpo_ou
                    (long long)(first_group + num_groups), (long long)batch->num_groups), GPO_ERR_INVALID_ARG;
   return compute_impl(ctx, batch, out, workspace, workspace_bytes, first_group, first_group + num_groups,
                       clear_status != 0, stream);
+}
+
+}  // extern "C"
+
+namespace {
+
+struct LossLayout {
+  size_t head, start, w, tile_edge, partial, total;
+  int64_t ntiles;
+};
+
+bool loss_layout(const gpo_batch& b, LossLayout& L) {
+  const int64_t N = b.num_states, T = b.total_tokens;
+  L.ntiles = (T + kLossTile - 1) / kLossTile;
+  if (N >= ((int64_t)1 << 31) - 1) return false;
+  size_t o = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = o;
+    o = up(o + bytes);
+    return at;
+  };
+  L.head = take(kLossPlanHead);
+  L.start = take(sizeof(int64_t) * (size_t)(N + 1));
+  L.w = take(sizeof(float) * (size_t)(N > 0 ? N : 1));
+  L.tile_edge = take(sizeof(int32_t) * (size_t)(L.ntiles + 1));
+  L.partial = take(sizeof(double) * 4 * (size_t)kLossMaxBlocks);
+  L.total = o;
+  return true;
+}
+
+LossPlan loss_views(void* base, const LossLayout& L) {
+  unsigned char* p = static_cast<unsigned char*>(base);
+  LossPlan lp;
+  lp.status = reinterpret_cast<uint32_t*>(p + L.head);
+  lp.dims = reinterpret_cast<int64_t*>(p + L.head + 128);
+  lp.start = reinterpret_cast<int64_t*>(p + L.start);
+  lp.w = reinterpret_cast<float*>(p + L.w);
+  lp.tile_edge = reinterpret_cast<int32_t*>(p + L.tile_edge);
+  lp.partial = reinterpret_cast<double*>(p + L.partial);
+  lp.ntiles = L.ntiles;
+  return lp;
+}
+
+Sizes loss_sizes(const gpo_batch& b) {
+  Sizes sz;
+  sz.G = b.num_groups;
+  sz.R = b.num_rollouts;
+  sz.N = b.num_states;
+  sz.d = b.d;
+  sz.T = b.total_tokens;
+  sz.stride = b.emb_row_stride;
+  sz.maxn = b.max_states_per_group;
+  sz.g0 = 0;
+  sz.g1 = b.num_groups;
+  return sz;
+}
+
+// The structure the loss reads: sizes and offsets (embeddings and rewards are not needed).
+gpo_status check_loss_batch(gpo_ctx* c, const gpo_batch* b) {
+  if (!b) return set_msg(c, "batch is NULL"), GPO_ERR_INVALID_ARG;
+  if (b->num_groups < 0 || b->num_rollouts < 0 || b->num_states < 0 || b->total_tokens < 0)
+    return set_msg(c, "negative size"), GPO_ERR_INVALID_ARG;
+  if (b->num_states == 0 && b->total_tokens != 0) return set_msg(c, "tokens without states"), GPO_ERR_SHAPE;
+  if (b->num_groups == 0 && (b->num_states != 0 || b->num_rollouts != 0))
+    return set_msg(c, "states without groups"), GPO_ERR_SHAPE;
+  if (b->parent) {
+    if (!b->group_rollout_off || !b->group_state_off || !b->group_token_off)
+      return set_msg(c, "tree layout: an offset array is NULL"), GPO_ERR_INVALID_ARG;
+  } else if (b->group_state_off || b->group_token_off) {
+    return set_msg(c, "group_state_off / group_token_off given without parent"), GPO_ERR_INVALID_ARG;
+  } else if (!b->group_rollout_off || !b->rollout_step_off || !b->rollout_token_off) {
+    return set_msg(c, "offset array is NULL"), GPO_ERR_INVALID_ARG;
+  }
+  if (b->num_states > 0 && !b->step_len) return set_msg(c, "step_len is NULL"), GPO_ERR_INVALID_ARG;
+  return GPO_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+gpo_status gpo_loss_plan_size(const gpo_batch* batch, size_t* bytes) {
+  if (!batch || !bytes) return GPO_ERR_INVALID_ARG;
+  LossLayout L;
+  if (batch->num_states < 0 || batch->total_tokens < 0 || !loss_layout(*batch, L)) return GPO_ERR_INVALID_ARG;
+  *bytes = L.total;
+  return GPO_OK;
+}
+
+gpo_status gpo_loss_plan(gpo_ctx* ctx, const gpo_batch* batch, void* plan, size_t plan_bytes, void* stream) {
+  if (!ctx) return GPO_ERR_INVALID_ARG;
+  ctx->msg[0] = 0;
+  gpo_status s = check_loss_batch(ctx, batch);
+  if (s != GPO_OK) return s;
+  LossLayout L;
+  if (!loss_layout(*batch, L)) return set_msg(ctx, "batch too large"), GPO_ERR_UNSUPPORTED;
+  if (!plan || !aligned(plan, kAlign) || plan_bytes < L.total)
+    return set_msg(ctx, "the plan needs %zu bytes, 256-byte aligned", L.total), GPO_ERR_WORKSPACE;
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev != ctx->device)
+    return set_msg(ctx, "current device differs from the context's"), GPO_ERR_INVALID_ARG;
+  const LossPlan lp = loss_views(plan, L);
+  LaunchCtx lc;
+  lc.stream = static_cast<cudaStream_t>(stream);
+  lc.num_sms = ctx->num_sms;
+  cudaError_t e = cudaMemsetAsync(lp.status, 0, kLossPlanHead, lc.stream);
+  if (e == cudaSuccess) e = launch_loss_plan(lc, *batch, loss_sizes(*batch), lp);
+  ctx->nstages = 0;
+  ctx->last_status = lp.status;
+  if (e != cudaSuccess) return set_msg(ctx, "launch failed: %s", cudaGetErrorString(e)), GPO_ERR_CUDA;
+  return GPO_OK;
+}
+
+gpo_status gpo_token_loss(gpo_ctx* ctx, const gpo_batch* batch, void* plan, const gpo_loss_params* params,
+                          const gpo_loss_inputs* in, const gpo_loss_outputs* out, void* stream) {
+  if (!ctx) return GPO_ERR_INVALID_ARG;
+  ctx->msg[0] = 0;
+  gpo_status s = check_loss_batch(ctx, batch);
+  if (s != GPO_OK) return s;
+  if (!params || !in || !out) return set_msg(ctx, "params, inputs or outputs NULL"), GPO_ERR_INVALID_ARG;
+  const gpo_loss_params& p = *params;
+  if (!(p.clip_low >= 0.0 && p.clip_low < 1.0) || !(p.clip_high >= 0.0) || !std::isfinite(p.clip_high) ||
+      !(p.beta_kl >= 0.0) || !std::isfinite(p.beta_kl) || !(p.lambda_eff >= 0.0) || !std::isfinite(p.lambda_eff) ||
+      (p.form != GPO_LOSS_DUAL && p.form != GPO_LOSS_SPLIT) || (p.norm != GPO_LOSS_NORM_EDGE && p.norm != GPO_LOSS_NORM_TOKEN))
+    return set_msg(ctx, "loss parameters out of range"), GPO_ERR_INVALID_ARG;
+  const bool split = p.form == GPO_LOSS_SPLIT, kl = p.beta_kl > 0.0;
+  const int64_t T = batch->total_tokens, N = batch->num_states;
+  if (!out->loss) return set_msg(ctx, "loss output is NULL"), GPO_ERR_INVALID_ARG;
+  if (T > 0 && (!in->logp || !in->old_logp || (kl && !in->ref_logp)))
+    return set_msg(ctx, "log-probabilities NULL"), GPO_ERR_INVALID_ARG;
+  if (N > 0 && (split ? (!in->edge_cor || !in->edge_eff || !in->edge_eff_mask) : !in->edge_adv))
+    return set_msg(ctx, "per-edge advantages of the %s form NULL", split ? "split" : "dual"), GPO_ERR_INVALID_ARG;
+  if (!aligned(in->logp, 16) || !aligned(in->old_logp, 16) || (kl && !aligned(in->ref_logp, 16)) ||
+      !aligned(out->grad_logp, 16))
+    return set_msg(ctx, "per-token arrays must be 16-byte aligned"), GPO_ERR_UNSUPPORTED;
+  LossLayout L;
+  if (!loss_layout(*batch, L)) return set_msg(ctx, "batch too large"), GPO_ERR_UNSUPPORTED;
+  if (!plan || !aligned(plan, kAlign)) return set_msg(ctx, "plan NULL or misaligned"), GPO_ERR_WORKSPACE;
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev != ctx->device)
+    return set_msg(ctx, "current device differs from the context's"), GPO_ERR_INVALID_ARG;
+  const LossPlan lp = loss_views(plan, L);
+  LossArgs a;
+  a.logp = in->logp;
+  a.old_logp = in->old_logp;
+  a.ref_logp = kl ? in->ref_logp : nullptr;
+  a.adv = split ? in->edge_cor : in->edge_adv;
+  a.eff = split ? in->edge_eff : nullptr;
+  a.mask = split ? in->edge_eff_mask : nullptr;
+  a.loss = out->loss;
+  a.grad = out->grad_logp;
+  a.stats = out->stats;
+  a.lo = (float)(1.0 - p.clip_low);
+  a.hi = (float)(1.0 + p.clip_high);
+  a.beta = (float)p.beta_kl;
+  a.lambda = (float)p.lambda_eff;
+  a.norm_token = p.norm == GPO_LOSS_NORM_TOKEN;
+  a.split = split;
+  a.kl = kl;
+  a.N = (int)N;
+  a.T = T;
+  LaunchCtx lc;
+  lc.stream = static_cast<cudaStream_t>(stream);
+  lc.num_sms = ctx->num_sms;
+  int ns = 0;
+  cudaError_t e = cudaSuccess;
+  if (ctx->timing) e = cudaEventRecord(ctx->ev[0], lc.stream);
+  if (e == cudaSuccess) e = launch_token_loss(lc, lp, a);
+  if (e == cudaSuccess && ctx->timing) {
+    ctx->stage_name[ns] = "token_loss";
+    e = cudaEventRecord(ctx->ev[++ns], lc.stream);
+  }
+  ctx->nstages = ns;
+  ctx->last_status = lp.status;
+  if (e != cudaSuccess) return set_msg(ctx, "launch failed: %s", cudaGetErrorString(e)), GPO_ERR_CUDA;
+  return GPO_OK;
 }
 
 gpo_status gpo_enable_timing(gpo_ctx* ctx, int enable) {

@@ -129,6 +129,7 @@ struct __align__(16) GroupSmem {
   int64_t tstart[kMaxN];
   uint8_t rew[kMaxN];
   uint8_t emask[kMaxN];
+  unsigned long long esum[3];  // exploration efficiency: token sums
   int flags;             // bit 0: group invalid
   int overflow;          // some warp found more pairs than its part of elist holds
   Plan plan;
@@ -152,6 +153,7 @@ struct __align__(8) Ctl {
 
 constexpr uint32_t kCtlOff = (sizeof(GroupSmem) + 15) & ~15u;
 constexpr uint32_t kTilesOff = kCtlOff + ((sizeof(Ctl) + 15) & ~15u);
+static_assert(kTilesOff + 1023 + kRingBytes <= 232448, "fused kernel exceeds 227 KB of shared memory");
 
 __device__ __forceinline__ void bar_group() { asm volatile("bar.sync %0, %1;" ::"n"(kBarGroup), "n"(kGThreads) : "memory"); }
 __device__ __forceinline__ void bar_epi() { asm volatile("bar.sync %0, %1;" ::"n"(kBarEpi), "n"(kEpiThreads) : "memory"); }
@@ -459,6 +461,10 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
                                 ((nr == 0 && n > 0) || (n == 0 && b.group_token_off[g + 1] != b.group_token_off[g]));
           if (!in_range || nr > n || (nr > 0 && n == 0) || tree_bad) report(st, GPO_ERR_SHAPE, 2, g);
           else if (n > kMaxN || n > sz.maxn) report(st, GPO_ERR_UNSUPPORTED, 2, g);
+          else if (n == 0) {  // a group without states: Eff 0 (no tokens)
+            if (o.group_eff) o.group_eff[g] = 0.f;
+            if (o.group_eff_graph) o.group_eff_graph[g] = 0.f;
+          }
         }
         continue;
       }
@@ -700,6 +706,9 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
           if (o.edge_adv) o.edge_adv[v] = dual;
           if (o.class_id) o.class_id[v] = s0 + label;
           if (o.node_score) o.node_score[v] = S;
+          if (o.edge_cor) o.edge_cor[v] = acor;
+          if (o.edge_eff) o.edge_eff[v] = E;
+          if (o.edge_eff_mask) o.edge_eff_mask[v] = mask;
         };
         if (tree) {
           auto eta_t = [&](int i) -> float2 {
@@ -714,6 +723,15 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
         } else {
           group_advantages<1, true>(n, nr, gs->lab, gs->roll, gs->dep, gs->rstart, gs->rew,
                                     group_scratch_sep(gs->X, n), p, gt, kGThreads, [] { bar_group(); }, eta, out);
+        }
+        // ---- exploration efficiency, Eq. (eq1) (the threshold norms' array is free here)
+        if (o.group_eff || o.group_eff_graph) {
+          auto own = [&](int i) { return tree ? gs->cown[i] > 0 : gs->rew[gs->roll[i]] != 0; };
+          auto par = [&](int i) { return tree ? gs->par[i] : (gs->dep[i] == 1 ? -1 : i - 1); };
+          auto len = [&](int i) { return gs->slen[i]; };
+          group_efficiency(n, gs->lab, reinterpret_cast<int*>(gs->n2), gs->esum, gt, kGThreads, own, par, len,
+                           [] { bar_group(); }, [](bool f) { return bar_any<kBarGroup, kGThreads>(f); },
+                           o.group_eff ? o.group_eff + g : nullptr, o.group_eff_graph ? o.group_eff_graph + g : nullptr);
         }
         // ---- every token of an edge carries the edge's advantage (Sec. 4.5).  State-major:
         //      each half-warp takes a state, its 16 lanes write the whole 16-byte chunks of the

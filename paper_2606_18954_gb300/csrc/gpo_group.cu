@@ -14,6 +14,9 @@ constexpr int kMaxRounds = 64;  // hook-and-shortcut rounds before falling back 
 
 // Shared memory: labels, rollout/depth per state (16-bit: a group holds at most
 // 4096 states), rollout offsets, rewards, then the scratch of group_advantages.
+// X also holds the tree's own statistics (2 al16(2n) <= 4n + 30 bytes) followed by the
+// efficiency marks (4n): within group_scratch_bytes(n) >= 4 kKeyWords (n + 1) + 32
+static_assert(kKeyWords >= 2, "efficiency marks after the tree's own statistics");
 __host__ __device__ inline size_t group_smem(int n) {
   return al16(sizeof(int) * (size_t)n) + 2 * al16(sizeof(int16_t) * (size_t)n) + al16(sizeof(int) * (size_t)(n + 1)) +
          al16((size_t)n) + group_scratch_bytes(n) + 64;
@@ -27,7 +30,13 @@ __global__ void __launch_bounds__(1024) groups_kernel(gpo_batch b, gpo_outputs o
   const int g = blockIdx.x;
   const GroupInfo gi = ws.groups[g];
   const int n = gi.n, s0 = gi.s0, nr = gi.nr, nt = blockDim.x, tid = threadIdx.x;
-  if (nr == 0 || n == 0 || n > sz.maxn) return;
+  if (nr == 0 || n == 0 || n > sz.maxn) {
+    if (n == 0 && tid == 0) {  // a group without states: Eff 0 (no tokens)
+      if (o.group_eff) o.group_eff[g] = 0.f;
+      if (o.group_eff_graph) o.group_eff_graph[g] = 0.f;
+    }
+    return;
+  }
 
   const bool tree = b.parent != nullptr;
   int* lab = reinterpret_cast<int*>(sm);
@@ -136,6 +145,21 @@ __global__ void __launch_bounds__(1024) groups_kernel(gpo_batch b, gpo_outputs o
     if (o.edge_adv) o.edge_adv[v] = dual;
     if (o.class_id) o.class_id[v] = s0 + label;
     if (o.node_score) o.node_score[v] = S;
+    if (o.edge_cor) o.edge_cor[v] = acor;
+    if (o.edge_eff) o.edge_eff[v] = E;
+    if (o.edge_eff_mask) o.edge_eff_mask[v] = mask;
+  };
+  // exploration efficiency, Eq. (eq1), once the classes are final; `mark` is scratch that
+  // the group math no longer needs
+  __shared__ unsigned long long s_eff[3];
+  auto efficiency = [&](int* mark) {
+    if (!o.group_eff && !o.group_eff_graph) return;
+    auto own = [&](int i) { return tree ? tcown[i] > 0 : rew[roll[i]] != 0; };
+    auto par = [&](int i) { return tree ? (int)tpar[i] : (dep[i] == 1 ? -1 : i - 1); };
+    auto len = [&](int i) { return b.step_len[s0 + i]; };
+    group_efficiency(n, lab, mark, s_eff, tid, nt, own, par, len, [] { __syncthreads(); },
+                     [](bool f) { return __syncthreads_or(f) != 0; }, o.group_eff ? o.group_eff + g : nullptr,
+                     o.group_eff_graph ? o.group_eff_graph + g : nullptr);
   };
   if (tree) {
     auto eta_t = [&](int i) -> float2 {
@@ -148,11 +172,14 @@ __global__ void __launch_bounds__(1024) groups_kernel(gpo_batch b, gpo_outputs o
     group_advantages_tree<kPer, int16_t>(n, nr, lab, tpar, dep, tend, tcown, ttown,
                                          tree_scratch(ws.tree_x + (size_t)23 * s0 + (size_t)11 * g, n), p, tid, nt,
                                          [] { __syncthreads(); }, eta_t, out);
+    // the own statistics take 2 al16(2n) bytes at the start of X
+    efficiency(reinterpret_cast<int*>(X + 2 * al16(sizeof(int16_t) * (size_t)n)));
     return;  // the tree prep kernel wrote the first token of every edge
   }
   __shared__ int s_rootc;
   group_advantages<kPer, false, int16_t>(n, nr, lab, roll, dep, rstart, rew, group_scratch_shared(X, n, &s_rootc), p,
                                          tid, nt, [] { __syncthreads(); }, eta, out);
+  efficiency(reinterpret_cast<int*>(X));
 
   // first token of every edge: one warp per rollout, an exclusive scan of the step lengths
   {

@@ -607,4 +607,78 @@ __device__ __forceinline__ void group_advantages_tree(int n, int nleaf, int* lab
   sync();
 }
 
+// ---------------------------------------------------------------------------------
+// Exploration efficiency, Eq. (eq1): the share of a group's step tokens spent on
+// steps from which a correct final answer can be reached.
+//   tree reading   own(i): a correct leaf lies below state i (c_own > 0; in the chain
+//                  layout the rollout is correct, the paper's chain case)
+//   graph reading  reachable through direct edges and merged states: a class reaches a
+//                  correct answer if one of its members does by the tree reading or a
+//                  member's child's class does; the least fixed point, by rounds that mark
+//                  the class of p(v) for every v whose class is marked (at most n + 1
+//                  rounds: each round before the last marks a new class)
+// lab      [n] final class labels
+// mark     [n] scratch words; sums: 3 scratch 64-bit words
+// par(i)   group-local parent of state i, or -1 for the prompt root
+// len(i)   tokens of the edge entering state i
+// any(f)   barrier over the nt threads that returns whether any thread passed true
+// Writes eff_tree / eff_graph (NULL: skipped) from thread 0; results are exact token
+// counts divided once.
+template <class Own, class Par, class Len, class Sync, class Any>
+__device__ __forceinline__ void group_efficiency(int n, const int* lab, int* mark, unsigned long long* sums, int tid,
+                                                 int nt, Own own, Par par, Len len, Sync sync, Any any,
+                                                 float* eff_tree, float* eff_graph) {
+  const int lane = tid & 31;
+  auto warp_sum = [&](unsigned long long x) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+    return x;
+  };
+  for (int i = tid; i < n; i += nt) mark[i] = 0;
+  if (tid < 3) sums[tid] = 0ull;
+  sync();
+  unsigned long long tot = 0, good = 0;
+  for (int i = tid; i < n; i += nt) {
+    const unsigned long long l = (unsigned long long)(unsigned)len(i);
+    tot += l;
+    if (own(i)) {
+      good += l;
+      mark[lab[i]] = 1;  // every such class is in the fixed point (a correct leaf lies below)
+    }
+  }
+  tot = warp_sum(tot);
+  good = warp_sum(good);
+  if (lane == 0) {
+    atomicAdd(&sums[0], tot);
+    atomicAdd(&sums[1], good);
+  }
+  sync();
+  if (eff_graph) {
+    bool changed = true;
+    for (int round = 0; round <= n && changed; ++round) {
+      bool ch = false;
+      for (int i = tid; i < n; i += nt) {
+        const int pp = par(i);
+        if (pp >= 0 && mark[lab[i]] && !mark[lab[pp]]) {
+          mark[lab[pp]] = 1;
+          ch = true;
+        }
+      }
+      changed = any(ch);
+    }
+    unsigned long long gg = 0;
+    for (int i = tid; i < n; i += nt)
+      if (mark[lab[i]]) gg += (unsigned long long)(unsigned)len(i);
+    gg = warp_sum(gg);
+    if (lane == 0) atomicAdd(&sums[2], gg);
+    sync();
+  }
+  if (tid == 0) {
+    const double t = (double)sums[0];
+    if (eff_tree) *eff_tree = t > 0.0 ? (float)((double)sums[1] / t) : 0.f;
+    if (eff_graph) *eff_graph = t > 0.0 ? (float)((double)sums[2] / t) : 0.f;
+  }
+  sync();
+}
+
 }  // namespace gpo

@@ -558,4 +558,43 @@ cudaError_t setup_groups();
 size_t sim_tc_smem_bytes();
 size_t groups_smem_bytes(int maxn);
 
+// ------------------------------------------------------------------ policy loss
+
+constexpr int kLossTile = 4096;        // tokens per tile of the loss kernel
+constexpr int kLossMaxBlocks = 1024;   // CTAs of one loss launch at most (reduction scratch)
+constexpr int kLossPlanHead = 256;     // bytes: status words, then the group count and the ticket
+constexpr int kLossWordGroups = kStatusWords, kLossWordTicket = kStatusWords + 1;
+
+// Device views of a loss plan (gpo_loss_plan), laid out on the host.
+struct LossPlan {
+  uint32_t* status;      // [kStatusWords], then [kLossWordGroups] groups with states, [kLossWordTicket]
+  int64_t* dims;         // [2] N and T of the batch the plan was built for (in the head, at byte 128)
+  int64_t* start;        // [N+1] first token of every edge, start[N] = T
+  float* w;              // [N] 1 / (G' |E_g| |e|) of the edge's tokens (first the group's |E_g|)
+  int32_t* tile_edge;    // [ntiles+1] edge holding each tile's first token; [ntiles] = N - 1
+  double* partial;       // [kLossMaxBlocks * 4] per-CTA sums of one loss launch
+  int64_t ntiles;
+};
+
+struct LossArgs {
+  const float* logp;
+  const float* old_logp;
+  const float* ref_logp;
+  const float* adv;      // dual: A_dual; split: A_cor
+  const float* eff;      // split: routed A_eff
+  const uint8_t* mask;   // split: m_eff
+  float* loss;
+  float* grad;
+  double* stats;
+  float lo, hi, beta, lambda;
+  int norm_token;        // 1: weights 1/T
+  int split, kl;
+  int N;
+  int64_t T;
+};
+
+cudaError_t launch_loss_plan(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const LossPlan& lp);
+cudaError_t launch_token_loss(const LaunchCtx& lc, const LossPlan& lp, const LossArgs& a);
+cudaError_t setup_loss();
+
 }  // namespace gpo

@@ -56,6 +56,9 @@ def test_binding_structs_match_header():
     assert [f for f, _ in B.Params._fields_] == struct_fields("gpo_params")
     assert [f for f, _ in B.CBatch._fields_] == struct_fields("gpo_batch")
     assert [f for f, _ in B.COutputs._fields_] == struct_fields("gpo_outputs")
+    assert [f for f, _ in B.LossParams._fields_] == struct_fields("gpo_loss_params")
+    assert [f for f, _ in B.LossInputs._fields_] == struct_fields("gpo_loss_inputs")
+    assert [f for f, _ in B.LossOutputs._fields_] == struct_fields("gpo_loss_outputs")
     assert sorted(B.EXPORTS) == declared_functions()
 
 
