@@ -526,3 +526,58 @@ def make_logprobs(T: int, seed: int, clip_low: float = 0.2, clip_high: float = 0
         raise RuntimeError("log-prob margin filter did not converge")
     ref = (new.astype(np.float64) + rng.normal(0.0, 0.1, T)).astype(np.float32)
     return dict(logp=new, old_logp=old, ref_logp=ref)
+
+
+# ---- layer-by-layer views of a branching batch (per-layer merge, GraphPO Sec. 4.2) -----
+
+
+def tree_depths(batch: dict) -> np.ndarray:
+    """Depth of every state of a tree-layout batch (1 = child of the prompt root)."""
+    par, gs = batch["parent"], batch["group_state_off"]
+    dep = np.zeros(len(par), dtype=np.int64)
+    for g in range(len(gs) - 1):
+        s0 = int(gs[g])
+        for v in range(s0, int(gs[g + 1])):
+            dep[v] = 1 if par[v] < 0 else dep[s0 + par[v]] + 1
+    return dep
+
+
+def truncate_tree(batch: dict, layer: int) -> dict:
+    """The batch as it stands after layer `layer` is sampled: the states of depth <= layer
+    (pre-order is kept, parents renumbered), their edges' tokens, the leaves of that tree
+    as its rollouts with placeholder rewards 0 (no answer is verified yet), and `active`:
+    1 on the states of depth `layer` that the full batch expands further."""
+    par, gs = batch["parent"], batch["group_state_off"]
+    dep = tree_depths(batch)
+    has_child = np.zeros(len(par), dtype=bool)
+    for g in range(len(gs) - 1):
+        s0 = int(gs[g])
+        for v in range(s0, int(gs[g + 1])):
+            if par[v] >= 0:
+                has_child[s0 + par[v]] = True
+    keep = dep <= layer
+    new_par, new_gs, new_go, new_gt, leaves = [], [0], [0], [0], 0
+    for g in range(len(gs) - 1):
+        s0, s1 = int(gs[g]), int(gs[g + 1])
+        idx = np.nonzero(keep[s0:s1])[0]
+        local = -np.ones(s1 - s0, dtype=np.int64)
+        local[idx] = np.arange(len(idx))
+        p = par[s0:s1][idx]
+        new_par.append(np.where(p < 0, -1, local[np.maximum(p, 0)]).astype(np.int32))
+        child = np.zeros(len(idx), dtype=bool)
+        q = new_par[-1]
+        child[q[q >= 0]] = True
+        nl = int((~child).sum())
+        leaves += nl
+        new_gs.append(new_gs[-1] + len(idx))
+        new_go.append(new_go[-1] + nl)
+        new_gt.append(new_gt[-1] + int(batch["step_len"][s0:s1][idx].astype(np.int64).sum()))
+    states = np.nonzero(keep)[0]
+    out = {k: v for k, v in batch.items() if k not in ("planted_centroid",)}
+    out.update(parent=np.concatenate(new_par) if new_par else np.zeros(0, np.int32),
+               group_state_off=np.asarray(new_gs, np.int32), group_rollout_off=np.asarray(new_go, np.int32),
+               group_token_off=np.asarray(new_gt, np.int64), total_tokens=int(new_gt[-1]),
+               step_len=batch["step_len"][states].astype(np.int32), emb=np.ascontiguousarray(batch["emb"][states]),
+               reward=np.zeros(leaves, np.uint8), source_states=states,
+               active=((dep[states] == layer) & has_child[states]).astype(np.uint8), layer=layer)
+    return out
