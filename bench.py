@@ -264,6 +264,42 @@ def time_token_loss(P, gp, b, db, alg, flush, stream, args):
             "bytes": 12 * T + 16 * N}
 
 
+def time_layer_budget(P, b, flush, stream, args):
+    """Per-layer graph construction (gpo_layer_budget: classes of the states sampled so far
+    and next-layer budgets, GraphPO Sec. 4.2) after the second-to-last layer of a branching
+    batch, timed like the path.  Algorithmic bytes per call: the embeddings of the states
+    sampled so far, their parents and step lengths, the budgets out."""
+    import torch
+    from paper_2606_18954_gb300 import workloads as W
+    H = len(b["spec"].schedule)
+    t = W.truncate_tree(b, H - 1)
+    db = P.Batch.from_arrays(t, device=stream.device)
+    act = torch.as_tensor(t["active"], device=stream.device)
+    gp = P.GraphPO(kappa=b["kappa"], w=b["w"], lambda_eff=b["lambda_eff"])
+    ws = gp.workspace(db)
+    out = None
+    for _ in range(args.warmup):
+        out = gp.layer_budget(db, H - 1, b["spec"].schedule[H - 1], act, out=out, workspace=ws, stream=stream)
+    gp.check(stream)
+    times = []
+    for _ in range(args.steps):
+        flush.zero_()
+        s = torch.cuda.Event(enable_timing=True)
+        e = torch.cuda.Event(enable_timing=True)
+        s.record(stream)
+        gp.layer_budget(db, H - 1, b["spec"].schedule[H - 1], act, out=out, workspace=ws, stream=stream)
+        e.record(stream)
+        e.synchronize()
+        times.append(s.elapsed_time(e))
+    gp.check(stream)
+    N = len(t["step_len"])
+    esz = 2 if t["emb_dtype"] == "bf16" else 4
+    nbytes = N * t["emb"].shape[1] * esz + 4 * N + 4 * N + 4 * N + N
+    ms = statistics.mean(times)
+    return {"ms": ms, "layer": H - 1, "states": N, "frontier": int((W.tree_depths(t) == H - 1).sum()), "active": int(t["active"].sum()),
+            "states_per_s": N / (ms / 1e3), "bytes": nbytes, "b_next": int(b["spec"].schedule[H - 1])}
+
+
 def dist_env():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     return ws, int(os.environ.get("RANK", "0")), int(os.environ.get("LOCAL_RANK", "0"))
@@ -409,6 +445,7 @@ def run_ours(args):
         e2e_t = float(t.item())
 
     loss = None if args.no_loss else time_token_loss(P, gp, b, db, alg, flush, stream, args)
+    layer = time_layer_budget(P, b, flush, stream, args) if b.get("parent") is not None else None
 
     if rank != 0:
         return 0
@@ -460,6 +497,12 @@ def run_ours(args):
                             "traffic": traffic, "traffic_note": tnote, "algorithmic_bytes": lb,
                             "peak_source": f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured" else "fallback"}
         line["token_loss"] = loss
+    if layer is not None:
+        lb = layer.pop("bytes")
+        achieved = lb / (layer["ms"] / 1e3) / 1e9
+        layer["roofline"] = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
+                             "algorithmic_bytes": lb, "launches": "fused kernel alone (no row statistics)"}
+        line["layer_budget"] = layer
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(b, max_groups={"wide": 2, "full": 64}.get(args.config))
     print(json.dumps(line), flush=True)

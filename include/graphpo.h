@@ -232,6 +232,33 @@ gpo_status gpo_stage_times(gpo_ctx* ctx, float* ms, const char** names, int capa
 #define GPO_NOALLOC_SCRATCH_BYTES ((size_t)32 << 20)
 gpo_status gpo_compute_noalloc(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* out, void* stream);
 
+/* Next-layer budgets of layer-by-layer graph construction (GraphPO Sec. 4.2: a path
+ * that reaches an existing equivalence class has its next-layer budget halved, keeping
+ * at least one continuation, and the saved budget is reallocated; Algorithm S.1 Stage 1:
+ * after layer h is sampled, every non-causal pair is linked and the saved budget goes
+ * to the active frontier states that are not redundant).
+ *
+ * `batch`: the tree layout of the states sampled so far (depth <= layer), its leaves
+ * as the rollouts (their rewards are not used but must be 0 or 1); the similarity part
+ * runs as in gpo_compute (same parameters, workspace size and checks).
+ * Per group:
+ *   frontier   the states of depth `layer` with active[v] != 0 (active NULL: all)
+ *   redundant  a frontier state whose class holds a state registered before it: one of
+ *              an earlier layer, or one of the same layer with a smaller index
+ *   budget[v]  b_next for a non-redundant frontier state, max(1, b_next / 2) for a
+ *              redundant one, 0 for every other state; the saved budget (the redundant
+ *              count times b_next - max(1, b_next / 2)) is split over the k non-redundant
+ *              frontier states: saved / k each plus one for the first saved % k of them
+ *              by index (with k = 0 it is not spent)
+ *   class_id   optional [N]: the classes of all states sampled so far (as gpo_compute)
+ * After the last layer the classes equal those of gpo_compute on the whole batch (every
+ * non-causal pair has been compared once).  1 <= layer, 1 <= b_next <= 65536; the chain
+ * layout gives GPO_ERR_UNSUPPORTED.  Asynchronous; device-side errors via
+ * gpo_sync_status as for gpo_compute. */
+gpo_status gpo_layer_budget(gpo_ctx* ctx, const gpo_batch* batch, int32_t layer, int32_t b_next,
+                            const uint8_t* active, int32_t* budget, int32_t* class_id, void* workspace,
+                            size_t workspace_bytes, void* stream);
+
 /* ---------------------------------------------------------------------------
  * Policy loss on per-token log-probabilities (GraphPO Sec. 4.5: the objective
  * J_GraphPO, DAPO's clipped surrogate on the graph advantage averaged over each

@@ -81,7 +81,7 @@ LOSS_NSTATS = 4
 
 EXPORTS = ["gpo_create", "gpo_workspace_size", "gpo_compute", "gpo_sync_status", "gpo_status_string",
            "gpo_last_error", "gpo_version", "gpo_destroy", "gpo_enable_timing", "gpo_stage_times", "gpo_compute_noalloc",
-           "gpo_compute_groups", "gpo_loss_plan_size", "gpo_loss_plan", "gpo_token_loss"]
+           "gpo_compute_groups", "gpo_loss_plan_size", "gpo_loss_plan", "gpo_token_loss", "gpo_layer_budget"]
 
 FUSED_MAX_STATES = 384  # largest group the group-resident path (and gpo_compute_groups) serves
 
@@ -134,6 +134,10 @@ def load(build_if_missing: bool = False):
         L.gpo_stage_times.argtypes = [ctypes.c_void_p, ctypes.POINTER(ctypes.c_float),
                                       ctypes.POINTER(ctypes.c_char_p), ctypes.c_int, ctypes.POINTER(ctypes.c_int)]
         L.gpo_stage_times.restype = ctypes.c_int
+        L.gpo_layer_budget.argtypes = [ctypes.c_void_p, ctypes.POINTER(CBatch), ctypes.c_int32, ctypes.c_int32,
+                                       ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
+                                       ctypes.c_size_t, ctypes.c_void_p]
+        L.gpo_layer_budget.restype = ctypes.c_int
         L.gpo_loss_plan_size.argtypes = [ctypes.POINTER(CBatch), ctypes.POINTER(ctypes.c_size_t)]
         L.gpo_loss_plan_size.restype = ctypes.c_int
         L.gpo_loss_plan.argtypes = [ctypes.c_void_p, ctypes.POINTER(CBatch), ctypes.c_void_p, ctypes.c_size_t,
@@ -357,6 +361,31 @@ class GraphPO:
                  stream=None) -> dict:
         out = self.alloc_outputs(batch, components, nodes, edges, efficiency)
         self.compute_into(batch, out, stream=stream)
+        return out
+
+    # ---- per-layer graph construction (gpo_layer_budget)
+
+    def layer_budget(self, batch: Batch, layer: int, b_next: int, active=None, classes: bool = False,
+                     out=None, workspace=None, stream=None) -> dict:
+        """Next-layer budgets (int32 [N]) and optionally the class ids after layer `layer` of a
+        tree-layout batch holding the states sampled so far; enqueued on the current stream."""
+        import torch
+        dev = batch.emb.device
+        if stream is None:
+            stream = torch.cuda.current_stream(dev)
+        N = batch.num_states
+        if out is None:
+            out = {"budget": torch.empty(max(N, 1), dtype=torch.int32, device=dev)[:N]}
+            if classes:
+                out["class_id"] = torch.empty(max(N, 1), dtype=torch.int32, device=dev)[:N]
+        ws = self.workspace(batch) if workspace is None else workspace
+        cb = batch.c_struct()
+        ptr = lambda t: None if t is None or t.numel() == 0 else t.data_ptr()
+        code = self._lib.gpo_layer_budget(self._h, ctypes.byref(cb), int(layer), int(b_next), ptr(active),
+                                          ptr(out["budget"]), ptr(out.get("class_id")), ws.data_ptr(), ws.numel(),
+                                          ctypes.c_void_p(stream.cuda_stream))
+        if code != GPO_OK:
+            raise GraphPOError(code, self.last_error())
         return out
 
     # ---- policy loss (gpo_loss_plan / gpo_token_loss)

@@ -284,14 +284,23 @@ gpo_status gpo_workspace_size(const gpo_ctx* ctx, const gpo_batch* batch, size_t
 
 namespace {
 
+// Next-layer budget request of gpo_layer_budget (mode 1 of the kernels).
+struct BudgetReq {
+  int layer, b_next;
+  const uint8_t* active;
+  int32_t* budget;
+};
+
 // The path for groups [g0, g1) of the batch; clears the status words first if `clear`.
+// With `bud`, the classes and the next-layer budgets instead of the advantages.
 gpo_status compute_impl(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* out, void* workspace,
-                        size_t workspace_bytes, int64_t g0, int64_t g1, bool clear, void* stream) {
+                        size_t workspace_bytes, int64_t g0, int64_t g1, bool clear, void* stream,
+                        const BudgetReq* bud = nullptr) {
   if (!ctx) return GPO_ERR_INVALID_ARG;
   ctx->msg[0] = 0;
   gpo_status s = check_batch(ctx, batch);
   if (s != GPO_OK) return s;
-  s = check_outputs(ctx, batch, out);
+  s = bud ? GPO_OK : check_outputs(ctx, batch, out);
   if (s != GPO_OK) return s;
   Layout L;
   if (!layout(*batch, L)) return set_msg(ctx, "batch too large"), GPO_ERR_UNSUPPORTED;
@@ -320,6 +329,11 @@ gpo_status compute_impl(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs*
   pp.eps = p.std_eps;
   pp.ddof = p.std_ddof;
   pp.rule = p.merge_rule;
+  pp.mode = bud ? 1 : 0;
+  pp.layer = bud ? bud->layer : 0;
+  pp.b_next = bud ? bud->b_next : 0;
+  pp.active = bud ? bud->active : nullptr;
+  pp.budget = bud ? bud->budget : nullptr;
   const Ws ws = workspace_views(workspace, L);
   LaunchCtx lc;
   lc.stream = static_cast<cudaStream_t>(stream);
@@ -367,7 +381,7 @@ gpo_status compute_impl(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs*
   if (g1 <= g0) {
     // nothing to compute (a call that only clears the status words)
   } else if (fused) {
-    if (e == cudaSuccess) e = stage("exact_stats", launch_exact_stats(lc, b, sz, ws));
+    if (e == cudaSuccess && !bud) e = stage("exact_stats", launch_exact_stats(lc, b, sz, ws));
     if (e == cudaSuccess) e = stage("fused", launch_fused(lc, map, map32, b, *out, sz, ws, pp));
   } else {
   if (e == cudaSuccess && b.parent) e = stage("tree_prep", launch_tree_prep(lc, b, sz, ws));
@@ -375,12 +389,12 @@ gpo_status compute_impl(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs*
   if (e == cudaSuccess && sz.N > 0) {
     // eta takes compensated norms and parent dots (exact_stats); the fp32 norms of the
     // threshold test come from the Gram tiles (tcgen05) or from row_stats (CUDA cores)
-    e = stage("exact_stats", launch_exact_stats(lc, b, sz, ws));
+    if (!bud) e = stage("exact_stats", launch_exact_stats(lc, b, sz, ws));
     if (e == cudaSuccess && !use_tc) e = stage("row_stats", launch_row_stats(lc, b, sz, ws));
     if (e == cudaSuccess)
       e = stage("similarity", use_tc ? launch_sim_tc(lc, map, b, sz, ws, pp) : launch_sim_simt(lc, b, sz, ws, pp));
     if (e == cudaSuccess) e = stage("groups", launch_groups(lc, b, *out, sz, ws, pp));
-    if (e == cudaSuccess) e = stage("tokens", launch_tokens(lc, b, *out, sz, ws));
+    if (e == cudaSuccess && !bud) e = stage("tokens", launch_tokens(lc, b, *out, sz, ws));
   }
   }
   ctx->nstages = ns;
@@ -397,6 +411,21 @@ gpo_status gpo_compute(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* 
                        size_t workspace_bytes, void* stream) {
   if (!ctx || !batch) return GPO_ERR_INVALID_ARG;
   return compute_impl(ctx, batch, out, workspace, workspace_bytes, 0, batch->num_groups, true, stream);
+}
+
+gpo_status gpo_layer_budget(gpo_ctx* ctx, const gpo_batch* batch, int32_t layer, int32_t b_next, const uint8_t* active,
+                            int32_t* budget, int32_t* class_id, void* workspace, size_t workspace_bytes, void* stream) {
+  if (!ctx || !batch) return GPO_ERR_INVALID_ARG;
+  ctx->msg[0] = 0;
+  if (!batch->parent) return set_msg(ctx, "next-layer budgets need the tree layout"), GPO_ERR_UNSUPPORTED;
+  if (layer < 1 || b_next < 1 || b_next > (1 << 16))
+    return set_msg(ctx, "layer must be >= 1 and b_next in [1, 65536]"), GPO_ERR_INVALID_ARG;
+  if (batch->num_states > 0 && !budget) return set_msg(ctx, "budget output is NULL"), GPO_ERR_INVALID_ARG;
+  gpo_outputs o;
+  memset(&o, 0, sizeof o);
+  o.class_id = class_id;
+  const BudgetReq req = {layer, b_next, active, budget};
+  return compute_impl(ctx, batch, &o, workspace, workspace_bytes, 0, batch->num_groups, true, stream, &req);
 }
 
 gpo_status gpo_compute_groups(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* out, int64_t first_group,

@@ -689,8 +689,19 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
       }
       if (bar_any<kBarGroup, kGThreads>(fail)) break;
 
+      // ---- next-layer budgets of a branching group (gpo_layer_budget)
+      if (valid && p.mode == 1) {
+        auto active = [&](int i) { return p.active == nullptr || p.active[s0 + i] != 0; };
+        auto put = [&](int i, int label, int bud) {
+          p.budget[s0 + i] = bud;
+          if (o.class_id) o.class_id[s0 + i] = s0 + label;
+        };
+        group_budget(n, gs->lab, gs->dep, p.layer, p.b_next, reinterpret_cast<int*>(gs->n2),
+                     reinterpret_cast<int*>(gs->esum), reinterpret_cast<int*>(gs->elist), gt, kGThreads,
+                     active, [] { bar_group(); }, put);
+      }
       // ---- graph reward and dual-group advantage of every edge
-      if (valid) {
+      else if (valid) {
         // eta(p(v), v) from the compensated row statistics (pairs; see exact_stats_kernel)
         auto eta = [&](int i) -> float2 {
           const float2 z = make_float2(0.f, 0.f);

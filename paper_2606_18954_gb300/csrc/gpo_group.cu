@@ -129,6 +129,19 @@ __global__ void __launch_bounds__(1024) groups_kernel(gpo_batch b, gpo_outputs o
     __syncthreads();
   }
 
+  if (p.mode == 1) {  // next-layer budgets (gpo_layer_budget; tree layout only)
+    __shared__ int s_bud[2 + 32];
+    auto active = [&](int i) { return p.active == nullptr || p.active[s0 + i] != 0; };
+    auto put = [&](int i, int label, int bud) {
+      p.budget[s0 + i] = bud;
+      if (o.class_id) o.class_id[s0 + i] = s0 + label;
+    };
+    // the own statistics take 2 al16(2n) bytes at the start of X
+    group_budget(n, lab, dep, p.layer, p.b_next, reinterpret_cast<int*>(X + 2 * al16(sizeof(int16_t) * (size_t)n)),
+                 s_bud, s_bud + 2, tid, nt, active, [] { __syncthreads(); }, put);
+    return;
+  }
+
   // eta(p(v), v) from the compensated row statistics (pairs); zero rows give 0
   const float2 zero2 = make_float2(0.f, 0.f);
   auto eta = [&](int i) -> float2 {

@@ -681,4 +681,72 @@ __device__ __forceinline__ void group_efficiency(int n, const int* lab, int* mar
   sync();
 }
 
+// ---------------------------------------------------------------------------------
+// Next-layer budgets after layer `layer` of a branching group (Sec. 4.2: a path that
+// reaches an existing equivalence class has its next-layer budget halved, keeping at
+// least one continuation, and the saved budget goes to other paths; Algorithm S.1
+// Stage 1 reallocates it to the active frontier states that are not redundant).
+//   frontier   states of depth `layer` with active(i)
+//   redundant  a frontier state whose class holds a state registered before it: one of
+//              an earlier layer, or one of the same layer with a smaller index
+//   budget     b_next for a non-redundant frontier state, max(1, b_next / 2) for a
+//              redundant one, 0 elsewhere; the saved budget S (redundant count x
+//              (b_next - max(1, b_next / 2))) is split over the k non-redundant frontier
+//              states: S / k each and one more for the first S % k of them by index
+// lab    [n] union-find forest of the classes (flattened here)
+// first  [n] scratch; cnt: 2 scratch words; wt: one scratch word per warp of the nt threads
+// out(i, label, budget) is called once per state.
+template <class IdxT, class Active, class Sync, class Out>
+__device__ __forceinline__ void group_budget(int n, int* lab, const IdxT* dep, int layer, int b_next, int* first,
+                                             int* cnt, int* wt, int tid, int nt, Active active, Sync sync, Out out) {
+  const int lane = tid & 31, warp = tid >> 5;
+  for (int i = tid; i < n; i += nt) {
+    lab[i] = uf_find(lab, i);  // concurrent finds only ever write roots
+    first[i] = 0x7FFFFFFF;
+  }
+  if (tid < 2) cnt[tid] = 0;
+  sync();
+  // registration order: layer, then index within the layer (n <= 4096 < 2^13)
+  auto key = [&](int i) { return ((int)dep[i] << 13) | i; };
+  for (int i = tid; i < n; i += nt) atomicMin(&first[lab[i]], key(i));
+  sync();
+  auto frontier = [&](int i) { return (int)dep[i] == layer && active(i); };
+  for (int base = 0; base < n; base += nt) {
+    const int i = base + tid;
+    const bool f = i < n && frontier(i);
+    const bool red = f && first[lab[i]] != key(i);
+    const uint32_t mr = __ballot_sync(0xffffffffu, red), mk = __ballot_sync(0xffffffffu, f && !red);
+    if (lane == 0) {
+      if (mr) atomicAdd(&cnt[0], __popc(mr));
+      if (mk) atomicAdd(&cnt[1], __popc(mk));
+    }
+  }
+  sync();
+  const int halved = b_next / 2 > 1 ? b_next / 2 : 1;
+  const long long saved = (long long)cnt[0] * (b_next - halved);
+  const int k = cnt[1];
+  const long long share = k ? saved / k : 0, extra = k ? saved % k : 0;
+  int carry = 0;  // non-redundant frontier states before this chunk
+  for (int base = 0; base < n; base += nt) {
+    const int i = base + tid;
+    const bool f = i < n && frontier(i);
+    const bool red = f && first[lab[i]] != key(i);
+    const uint32_t m = __ballot_sync(0xffffffffu, f && !red);
+    if (lane == 0) wt[warp] = __popc(m);
+    sync();
+    int before = 0, total = 0;
+    for (int w = 0; w < nt / 32; ++w) {
+      before += w < warp ? wt[w] : 0;
+      total += wt[w];
+    }
+    if (i < n) {
+      const int rank = carry + before + __popc(m & ((1u << lane) - 1u));
+      const long long bud = !f ? 0 : (red ? halved : b_next + share + (rank < extra ? 1 : 0));
+      out(i, lab[i], (int)bud);
+    }
+    carry += total;
+    sync();
+  }
+}
+
 }  // namespace gpo

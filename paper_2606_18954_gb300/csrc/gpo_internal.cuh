@@ -84,6 +84,10 @@ struct Sizes {
 struct Params {
   double kappa, w, lambda_eff, eps;
   int ddof, rule;
+  // mode 1: next-layer budgets after layer `layer` instead of advantages (gpo_layer_budget)
+  int mode, layer, b_next;
+  const uint8_t* active;  // [N] frontier states to expand (NULL: all of depth `layer`)
+  int32_t* budget;        // [N] output of mode 1
 };
 
 // ------------------------------------------------------------------ errors
