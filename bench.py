@@ -109,7 +109,8 @@ def algorithmic(b):
         "similarity": (zb + 12 * N, flops),
         "groups": (8 * N + R + 12 * R + 4 * N + 17 * N + 8 * N, 0.0),
         "tokens": (4 * T + 8 * N + 4 * N + 4 * N, 0.0),
-        "fused": (path_bytes, flops),  # the group-resident kernel does the whole path
+        # the group-resident kernel does the whole path, the compensated statistics included
+        "fused": (path_bytes, flops, alu_x),
     }
     return dict(N=N, R=R, G=G, T=T, path_bytes=path_bytes, flops=flops, stages=stages)
 

@@ -334,6 +334,8 @@ gpo_status compute_impl(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs*
   pp.b_next = bud ? bud->b_next : 0;
   pp.active = bud ? bud->active : nullptr;
   pp.budget = bud ? bud->budget : nullptr;
+  pp.stats_in_kernel = 0;
+  pp.pad_ = 0;
   const Ws ws = workspace_views(workspace, L);
   LaunchCtx lc;
   lc.stream = static_cast<cudaStream_t>(stream);
@@ -381,7 +383,11 @@ gpo_status compute_impl(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs*
   if (g1 <= g0) {
     // nothing to compute (a call that only clears the status words)
   } else if (fused) {
-    if (e == cudaSuccess && !bud) e = stage("exact_stats", launch_exact_stats(lc, b, sz, ws));
+    // one group per CTA: the group warps compute the compensated row statistics while the
+    // group streams in (one launch); more groups than CTAs: a launch of their own first
+    // (on the whole GPU), so that the group warps keep pace with the stream
+    pp.stats_in_kernel = !bud && (int64_t)(g1 - g0) <= (int64_t)fused_grid(lc, sz);
+    if (e == cudaSuccess && !bud && !pp.stats_in_kernel) e = stage("exact_stats", launch_exact_stats(lc, b, sz, ws));
     if (e == cudaSuccess) e = stage("fused", launch_fused(lc, map, map32, b, *out, sz, ws, pp));
   } else {
   if (e == cudaSuccess && b.parent) e = stage("tree_prep", launch_tree_prep(lc, b, sz, ws));

@@ -20,10 +20,12 @@
 //                   cos = acc / (|z_i||z_j|) >= kappa goes to an edge list; the
 //                   accumulator is released and the listed pairs are united in a
 //                   shared-memory union-find forest (Alg. S.1)
-//   warps 2..       per-group validation, graph reward and dual-group advantage
-//                   (gpo_group_math.cuh; eta(p(v), v) from the compensated row
-//                   statistics of exact_stats, run just before) and the token scatter
-//                   (Sec. 4.5), overlapping the next group's loads and MMAs
+//   warps 2..       per-group validation; the compensated row statistics of the group
+//                   (eta(p(v), v) needs them) while the producer streams it, when every
+//                   CTA has one group (else exact_stats runs as a launch of its own just
+//                   before, on the whole GPU); graph reward and dual-group advantage
+//                   (gpo_group_math.cuh) and the token scatter (Sec. 4.5), overlapping
+//                   the next group's loads and MMAs
 // Group ranges are assigned round-robin to CTAs.  Every wait is bounded.
 #include "gpo_group_math.cuh"
 
@@ -56,19 +58,23 @@ cudaError_t setup_fused() {
   return e;
 }
 
+int fused_grid(const LaunchCtx& lc, const Sizes& sz) {
+  const int ng = sz.g1 - sz.g0;
+  const int cap = lc.num_sms * (sz.maxn <= fused_small::kMaxN ? fused_small::kMinBlocks : fused_large::kMinBlocks);
+  return ng < cap ? ng : cap;
+}
+
 cudaError_t launch_fused(const LaunchCtx& lc, const CUtensorMap& map, const CUtensorMap& map32, const gpo_batch& b,
                          const gpo_outputs& o, const Sizes& sz, const Ws& ws, const Params& p) {
   const int ng = sz.g1 - sz.g0;
   if (ng <= 0) return cudaSuccess;
-  if (sz.maxn <= fused_small::kMaxN) {
-    const int cap = lc.num_sms * fused_small::kMinBlocks;
-    fused_small::fused_kernel<<<ng < cap ? ng : cap, fused_small::kThreads, fused_small::fused_smem(), lc.stream>>>(
-        map, map32, b, o, sz, ws, p);
-  } else {
-    const int cap = lc.num_sms * fused_large::kMinBlocks;
-    fused_large::fused_kernel<<<ng < cap ? ng : cap, fused_large::kThreads, fused_large::fused_smem(), lc.stream>>>(
-        map, map32, b, o, sz, ws, p);
-  }
+  const int grid = fused_grid(lc, sz);
+  if (sz.maxn <= fused_small::kMaxN)
+    fused_small::fused_kernel<<<grid, fused_small::kThreads, fused_small::fused_smem(), lc.stream>>>(map, map32, b, o,
+                                                                                                   sz, ws, p);
+  else
+    fused_large::fused_kernel<<<grid, fused_large::kThreads, fused_large::fused_smem(), lc.stream>>>(map, map32, b, o,
+                                                                                                   sz, ws, p);
   return cudaGetLastError();
 }
 

@@ -183,6 +183,103 @@ __device__ __forceinline__ float pick(const uint32_t (&r)[32], int j) {
   return v;
 }
 
+// Compensated |z_v|^2 and <z_{p(v)}, z_v> of the group's states [s0, s0 + n) into
+// ws.x_n2 / ws.x_dot (float pairs), and |prompt embedding|^2 into ws.x_root_n2[g]; every
+// group thread calls it (wg = group warp 0.., lane).  Parents from the group layout in
+// shared memory (chain: the previous state unless the state is a rollout's first; tree:
+// gs->par).
+__device__ __forceinline__ void group_row_stats(const gpo_batch& b, const Sizes& sz, const Ws& ws, GroupSmem* gs,
+                                                int g, int s0, int n, bool tree, int wg, int lane, uint32_t* st) {
+  constexpr int kGWarps = kGThreads / 32;
+  const int r = lane >> 2, c = lane & 3;
+  const int nch = sz.d / 8;          // whole 16-byte chunks of a row
+  const int64_t rs = sz.stride / 8;  // row stride in 16-byte chunks
+  const uint4* Z = reinterpret_cast<const uint4*>(b.emb);
+  const uint4* RZ = reinterpret_cast<const uint4*>(b.root_emb);
+  auto finish4 = [&](uint64_t s, uint64_t e) -> float2 {  // the row's 4 lanes, fixed order
+    float2 P = f2_finish(s, e);
+#pragma unroll
+    for (int o = 1; o < 4; o <<= 1) {
+      const float a = __shfl_xor_sync(0xffffffffu, P.x, o), q = __shfl_xor_sync(0xffffffffu, P.y, o);
+      float t, u;
+      two_sum(P.x, a, t, u);
+      P.x = t;
+      P.y = P.y + q + u;
+    }
+    float h, l;
+    two_sum(P.x, P.y, h, l);
+    return make_float2(h, l);
+  };
+  for (int blk = wg; blk * 8 < n; blk += kGWarps) {
+    const int i = blk * 8 + r;  // local row of this lane
+    const bool live = i < n;
+    // parent: >= 0 a local row, -2 the prompt embedding, -1 none (eta 0)
+    int pl = -1;
+    if (live) {
+      pl = tree ? gs->par[i] : (gs->dep[i] > 1 ? i - 1 : -1);
+      if (pl < 0) pl = b.root_emb ? -2 : -1;
+    }
+    const bool from_left = pl >= 0 && pl == i - 1 && r > 0;
+    const uint4* zb = Z + (int64_t)(s0 + (live ? i : 0)) * rs;
+    const uint4* pb = pl >= 0 ? Z + (int64_t)(s0 + pl) * rs : (pl == -2 ? RZ + (int64_t)g * rs : nullptr);
+    uint64_t ns = 0ull, ne = 0ull, ds = 0ull, de = 0ull;
+    constexpr int kU = 4;  // chunks loaded ahead of their arithmetic
+    for (int k0 = 0; k0 < nch; k0 += 4 * kU) {
+      uint4 x[kU], y[kU];
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        const int k = k0 + 4 * u + c;
+        const bool in = k < nch;
+        x[u] = live && in ? zb[k] : make_uint4(0u, 0u, 0u, 0u);
+        y[u] = !from_left && pb && in ? pb[k] : make_uint4(0u, 0u, 0u, 0u);
+      }
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        uint4 t;
+        t.x = __shfl_up_sync(0xffffffffu, x[u].x, 4);
+        t.y = __shfl_up_sync(0xffffffffu, x[u].y, 4);
+        t.z = __shfl_up_sync(0xffffffffu, x[u].z, 4);
+        t.w = __shfl_up_sync(0xffffffffu, x[u].w, 4);
+        if (from_left) y[u] = t;
+        const uint32_t xw[4] = {x[u].x, x[u].y, x[u].z, x[u].w}, yw[4] = {y[u].x, y[u].y, y[u].z, y[u].w};
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+          const uint64_t xx = bf16x2_f32x2(xw[h]), yy = bf16x2_f32x2(yw[h]);
+          f2_acc(ns, ne, f2mul(xx, xx));  // bf16 products are exact in fp32
+          f2_acc(ds, de, f2mul(xx, yy));
+        }
+      }
+    }
+    if (sz.d % 8 != 0 && c == 0 && live) {  // the ragged end of the row, one lane per row
+      const uint16_t* zr = reinterpret_cast<const uint16_t*>(zb);
+      const uint16_t* pr = reinterpret_cast<const uint16_t*>(pb);
+      for (int k = 8 * nch; k < sz.d; ++k) {
+        const uint64_t xx = (uint64_t)((uint32_t)zr[k] << 16);
+        const uint64_t yy = pr ? (uint64_t)((uint32_t)pr[k] << 16) : 0ull;
+        f2_acc(ns, ne, f2mul(xx, xx));  // one fp32 lane (the other stays 0)
+        f2_acc(ds, de, f2mul(xx, yy));
+      }
+    }
+    const float2 n2 = finish4(ns, ne);
+    float2 dot = finish4(ds, de);
+    if (pl == -1) dot = make_float2(0.f, 0.f);
+    if (live && c == 0) {
+      if (!isfinite(n2.x) || !isfinite(dot.x)) report(st, GPO_ERR_NONFINITE, 3, s0 + i);
+      ws.x_n2[s0 + i] = n2;
+      ws.x_dot[s0 + i] = dot;
+    }
+  }
+  if (b.root_emb && wg == kGWarps - 1) {  // |prompt embedding|^2, one warp
+    float2 n2, dot;
+    exact_pair_sums<true>(b.root_emb, (int64_t)g * sz.stride, nullptr, 0, false, sz.d, lane, n2, dot);
+    if (lane == 0) {
+      if (!isfinite(n2.x)) report(st, GPO_ERR_NONFINITE, 3, sz.N + g);
+      ws.x_root_n2[g] = n2;
+    }
+  }
+}
+
+
 // Tree-layout set-up of group g (Sec. 4.2 branching rollouts: parents precede their
 // children, depth-first pre-order): checks, depth, subtree end, own terminal statistics
 // (Sec. 4.3: c_own / t_own of a state = the rewards / the number of the leaves of its
@@ -516,8 +613,18 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
       }
       const bool valid = (gs->flags & 1) == 0;
 
-      // ---- drain the accumulator pass by pass (warps 4..15); warps 2..3 fetch
-      //      the prompt-embedding dots when a root embedding is given
+      // ---- compensated row statistics of the group (eta needs them; the Gram accumulator
+      //      is too coarse): |z_v|^2 and <z_{p(v)}, z_v> as float pairs into ws.x_n2 / x_dot,
+      //      by the group warps while the producer streams the same rows (L2 serves the
+      //      second reader; only when every CTA has one group, so that this work overlaps
+      //      the stream instead of delaying the next group).  A warp takes 8 rows, lane 4 r + c every fourth 16-byte chunk of
+      //      row r starting at chunk c; a parent that is the row before comes from the lane
+      //      4 below, other parents and the prompt embedding are loaded.  bf16 products are
+      //      exact in fp32, every sum is compensated (TwoSum per element, two fp32 lanes per
+      //      instruction), the row's 4 partial pairs are combined in a fixed butterfly.
+      if (valid && p.mode == 0 && p.stats_in_kernel) group_row_stats(b, sz, ws, gs, g, s0, n, tree, wg, lane, st);
+
+      // ---- drain the accumulator pass by pass (warps 4..15)
       bool fail = false;
       if (epi) {
         const Plan& pl = gs->plan;

@@ -86,6 +86,8 @@ struct Params {
   int ddof, rule;
   // mode 1: next-layer budgets after layer `layer` instead of advantages (gpo_layer_budget)
   int mode, layer, b_next;
+  int stats_in_kernel;    // fused path: the group warps compute the compensated row statistics
+  int pad_;
   const uint8_t* active;  // [N] frontier states to expand (NULL: all of depth `layer`)
   int32_t* budget;        // [N] output of mode 1
 };
@@ -554,6 +556,8 @@ cudaError_t launch_tokens(const LaunchCtx& lc, const gpo_batch& b, const gpo_out
 // Records a message on the context (gpo_last_error).
 void note_error(gpo_ctx* ctx, const char* msg);
 
+// CTAs the fused kernel runs with for groups [g0, g1) (one group each when ng <= this).
+int fused_grid(const LaunchCtx& lc, const Sizes& sz);
 cudaError_t launch_fused(const LaunchCtx& lc, const CUtensorMap& map, const CUtensorMap& map32, const gpo_batch& b,
                          const gpo_outputs& o, const Sizes& sz, const Ws& ws, const Params& p);
 cudaError_t setup_fused();
