@@ -8,10 +8,10 @@
 //             and the edge holding the first token of every tile of kLossTile tokens.
 //   loss      token_loss_kernel: persistent CTAs over token tiles; a tile's edges (first
 //             token, weight x advantages; at most one per token) are staged in shared
-//             memory, each thread takes
-//             four 16-byte chunks of tokens (coalesced across the CTA; all four loaded
-//             before the edges are staged), finds the edge of each chunk's first token
-//             by binary search and walks on; per token the ratio, the
+//             memory with a token -> edge map of the tile; each thread takes four 16-byte
+//             chunks of tokens (coalesced across the CTA; all four loaded before the
+//             edges are staged) and reads each token's edge from the map; per token the
+//             ratio, the
 //             clipped surrogate, the k3 KL estimate, the gradient (one 16-byte store per
 //             chunk); sums in fp32 per tile, fp64 across tiles, per-CTA partials combined
 //             by the last CTA in a fixed order (deterministic).
@@ -178,7 +178,8 @@ __device__ __forceinline__ bool surrogate(float r, float rc, float wa, float& f,
 // Shared memory of one CTA: the tile's edges (at most one per token)
 template <bool kSplit, bool kKL>
 struct LossSmem {
-  int start[kLossTile + 1];               // first token of each edge, relative to the tile
+  uint16_t map[kLossTile];                // edge (tile-local) of every token of the tile
+  int16_t start[kLossTile + 2];           // first token of each edge, relative to the tile
   float wa[kLossTile];                    // w A (dual) or w A_cor (split)
   float we[kSplit ? kLossTile : 1];       // split: w lambda m_eff A_eff
   float w[kKL ? kLossTile : 1];           // KL: w
@@ -235,7 +236,7 @@ __global__ void __launch_bounds__(kLossThreads, kKL ? 3 : 4) token_loss_kernel(L
     __syncthreads();  // the previous tile's readers are done
     for (int j = tid; j <= ne; j += kLossThreads) {
       const int64_t st = lp.start[e_lo + j] - t0;
-      sm.start[j] = (int)max(min(st, (int64_t)kLossTile + 1), (int64_t)-1);  // in [-1, kLossTile + 1]
+      sm.start[j] = (int16_t)max(min(st, (int64_t)kLossTile), (int64_t)0);  // clamped to the tile
       if (j < ne) {
         const float w = a.norm_token ? inv_t : lp.w[e_lo + j];
         sm.wa[j] = w * a.adv[e_lo + j];
@@ -244,29 +245,23 @@ __global__ void __launch_bounds__(kLossThreads, kKL ? 3 : 4) token_loss_kernel(L
       }
     }
     __syncthreads();
+    // the token -> edge map of the tile: warp w fills the spans of edges w, w + 8, ...
+    for (int j = warp; j < ne; j += kLossThreads / 32)
+      for (int t = sm.start[j] + lane; t < sm.start[j + 1]; t += 32) sm.map[t] = (uint16_t)j;
+    __syncthreads();
     float pg = 0.f, kl = 0.f, rs = 0.f;
     int nclip = 0;
 #pragma unroll
     for (int k = 0; k < kLossChunks; ++k) {
       const int rel = 4 * (tid + k * kLossThreads);  // first token of this chunk in the tile
       if (rel >= tn) continue;
-      // the edge holding token rel: the last j with start[j] <= rel
-      int lo = 0, hi = ne - 1;
-      while (lo < hi) {
-        const int mid = (lo + hi + 1) >> 1;
-        if (sm.start[mid] <= rel) lo = mid;
-        else hi = mid - 1;
-      }
-      int j = lo;
-      int nxt = sm.start[j + 1];
+      const uint2 m4 = *reinterpret_cast<const uint2*>(sm.map + rel);  // the 4 tokens' edges
+      const int jj[4] = {(int)(m4.x & 0xFFFFu), (int)(m4.x >> 16), (int)(m4.y & 0xFFFFu), (int)(m4.y >> 16)};
       float gr[4];
 #pragma unroll
       for (int c = 0; c < 4; ++c) {
-        if (c > 0 && rel + c >= nxt && j + 1 < ne) {  // the next edge (every edge has a token)
-          ++j;
-          nxt = sm.start[j + 1];
-        }
         const bool in = rel + c < tn;
+        const int j = in ? min(jj[c], ne - 1) : 0;  // tokens past the tile's end read edge 0
         const float r = __expf(x[k][c] - y[k][c]);
         const float rc = fminf(fmaxf(r, a.lo), a.hi);
         float f, df;
