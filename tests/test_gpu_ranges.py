@@ -13,7 +13,8 @@ from paper_2606_18954_gb300 import workloads as W
 
 pytestmark = pytest.mark.gpu
 
-KEYS = ("adv", "adv_cor", "adv_eff", "eff_mask", "class_id", "node_score", "edge_adv")
+KEYS = ("adv", "adv_cor", "adv_eff", "eff_mask", "class_id", "node_score", "edge_adv", "edge_cor", "edge_eff",
+        "edge_eff_mask", "group_eff", "group_eff_graph")
 
 
 @pytest.fixture(scope="module")
@@ -40,9 +41,9 @@ def test_ranges_cover_batch(P, cuts):
     b = _batch("math", 8)
     gp = _gp(P, b)
     db = P.Batch.from_arrays(b, device="cuda")
-    ref = gp(db, components=True, nodes=True)
+    ref = gp(db, components=True, nodes=True, edges=True, efficiency=True)
     gp.check()
-    out = gp.alloc_outputs(db, components=True, nodes=True)
+    out = gp.alloc_outputs(db, components=True, nodes=True, edges=True, efficiency=True)
     for v in out.values():
         v.fill_(-7)  # every element must be overwritten
     ws = gp.workspace(db)

@@ -20,7 +20,8 @@ from paper_2606_18954_gb300 import workloads as W
 pytestmark = pytest.mark.gpu
 
 RTOL, ATOL = 1e-5, 1e-6
-KEYS = ("adv", "adv_cor", "adv_eff", "eff_mask", "class_id", "node_score", "edge_adv")
+KEYS = ("adv", "adv_cor", "adv_eff", "eff_mask", "class_id", "node_score", "edge_adv", "edge_cor", "edge_eff",
+        "edge_eff_mask", "group_eff", "group_eff_graph")  # the order of gpo_outputs
 
 
 @pytest.fixture(scope="module")
@@ -58,9 +59,9 @@ def test_noalloc_matches_compute_twice(P):
         b = W.make_batch(W.CONFIGS[name].scaled(groups))
         gp = P.GraphPO(kappa=b["kappa"], w=b["w"], lambda_eff=b["lambda_eff"])
         db = P.Batch.from_arrays(b, device="cuda")
-        ref = gp(db, components=True, nodes=True)
+        ref = gp(db, components=True, nodes=True, edges=True, efficiency=True)
         gp.check()
-        out = gp.alloc_outputs(db, components=True, nodes=True)
+        out = gp.alloc_outputs(db, components=True, nodes=True, edges=True, efficiency=True)
         for o in out.values():
             o.fill_(7) if o.dtype != torch.float32 else o.fill_(float("nan"))
         assert _noalloc(P, gp, db, out) == 0, gp.last_error()
