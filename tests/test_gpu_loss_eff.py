@@ -285,3 +285,30 @@ def test_loss_errors(gp_mod):
     gp.token_loss(dbad, pbad, logp, old, edge_adv=t(A), out=res)
     torch.cuda.synchronize()
     assert float(res["loss"].cpu()[0]) == 123.0
+    # a plan built for another batch shape: reported, outputs left alone
+    other = P.Batch.from_arrays(batch_of("math", 3), device="cuda")
+    pother = gp.loss_plan(other)
+    gp.check()
+    res = {"loss": torch.full((1,), 123.0, device="cuda")}
+    gp.token_loss(db, pother, logp, old, edge_adv=t(A), out=res)
+    with pytest.raises(P.GraphPOError) as e:
+        gp.check()
+    assert e.value.code == 2
+    assert float(res["loss"].cpu()[0]) == 123.0
+
+
+def test_loss_empty_batch(gp_mod):
+    """Groups without states: no tokens, the loss is 0 and the statistics are 0."""
+    import torch
+    P = gp_mod
+    b = dict(group_rollout_off=np.zeros(3, np.int32), rollout_step_off=np.zeros(1, np.int32),
+             step_len=np.zeros(0, np.int32), rollout_token_off=np.zeros(1, np.int64),
+             emb=np.zeros((0, 16), np.uint16), emb_dtype="bf16", reward=np.zeros(0, np.uint8))
+    gp = P.GraphPO()
+    db = P.Batch.from_arrays(b, device="cuda")
+    plan = gp.loss_plan(db)
+    empty = torch.zeros(0, dtype=torch.float32, device="cuda")
+    res = gp.token_loss(db, plan, empty, empty, edge_adv=empty)
+    gp.check()
+    assert float(res["loss"].cpu()[0]) == 0.0
+    np.testing.assert_array_equal(res["stats"].cpu().numpy(), np.zeros(4))
