@@ -223,9 +223,10 @@ __device__ __forceinline__ void group_row_stats(const gpo_batch& b, const Sizes&
     const uint4* zb = Z + (int64_t)(s0 + (live ? i : 0)) * rs;
     const uint4* pb = pl >= 0 ? Z + (int64_t)(s0 + pl) * rs : (pl == -2 ? RZ + (int64_t)g * rs : nullptr);
     uint64_t ns = 0ull, ne = 0ull, ds = 0ull, de = 0ull;
-    constexpr int kU = 4;  // chunks loaded ahead of their arithmetic
-    for (int k0 = 0; k0 < nch; k0 += 4 * kU) {
-      uint4 x[kU], y[kU];
+    // two stages of kU chunks per lane, software-pipelined: the next stage's loads are in
+    // flight while this one's sums run (no register copies between the stages)
+    constexpr int kU = 2;
+    auto load = [&](int k0, uint4 (&x)[kU], uint4 (&y)[kU]) {
 #pragma unroll
       for (int u = 0; u < kU; ++u) {
         const int k = k0 + 4 * u + c;
@@ -233,6 +234,8 @@ __device__ __forceinline__ void group_row_stats(const gpo_batch& b, const Sizes&
         x[u] = live && in ? zb[k] : make_uint4(0u, 0u, 0u, 0u);
         y[u] = !from_left && pb && in ? pb[k] : make_uint4(0u, 0u, 0u, 0u);
       }
+    };
+    auto accumulate = [&](uint4 (&x)[kU], uint4 (&y)[kU]) {
 #pragma unroll
       for (int u = 0; u < kU; ++u) {
         uint4 t;
@@ -249,6 +252,14 @@ __device__ __forceinline__ void group_row_stats(const gpo_batch& b, const Sizes&
           f2_acc(ds, de, f2mul(xx, yy));
         }
       }
+    };
+    uint4 xa[kU], ya[kU], xb[kU], yb[kU];
+    load(0, xa, ya);
+    for (int k0 = 0; k0 < nch; k0 += 8 * kU) {
+      load(k0 + 4 * kU, xb, yb);  // past the row's end: zeros, which add nothing
+      accumulate(xa, ya);
+      load(k0 + 8 * kU, xa, ya);
+      accumulate(xb, yb);
     }
     if (sz.d % 8 != 0 && c == 0 && live) {  // the ragged end of the row, one lane per row
       const uint16_t* zr = reinterpret_cast<const uint16_t*>(zb);
