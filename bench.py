@@ -265,6 +265,34 @@ def time_token_loss(P, gp, b, db, alg, flush, stream, args):
             "bytes": 12 * T + 16 * N}
 
 
+def time_efficiency(P, gp, db, out, wsp, flush, stream, args):
+    """The path with and without its optional exploration-efficiency outputs (Eq. (eq1),
+    both readings) and per-edge A_cor / A_eff / m_eff, timed like the path."""
+    import torch
+
+    def timed(o):
+        for _ in range(args.warmup):
+            gp.compute_into(db, o, workspace=wsp, stream=stream)
+        ts = []
+        for _ in range(args.steps):
+            flush.zero_()
+            s = torch.cuda.Event(enable_timing=True)
+            e = torch.cuda.Event(enable_timing=True)
+            s.record(stream)
+            gp.compute_into(db, o, workspace=wsp, stream=stream)
+            e.record(stream)
+            e.synchronize()
+            ts.append(s.elapsed_time(e))
+        gp.check(stream)
+        return statistics.mean(ts)
+
+    extra = gp.alloc_outputs(db, edges=True, efficiency=True)
+    with_eff = timed(extra)
+    base = timed(out)
+    return {"ms_with_outputs": with_eff, "ms_without": base, "overhead_ms": with_eff - base,
+            "outputs": "group_eff, group_eff_graph, edge_cor, edge_eff, edge_eff_mask (and adv)"}
+
+
 def time_layer_budget(P, b, flush, stream, args):
     """Per-layer graph construction (gpo_layer_budget: classes of the states sampled so far
     and next-layer budgets, GraphPO Sec. 4.2) after the second-to-last layer of a branching
@@ -446,7 +474,12 @@ def run_ours(args):
         e2e_t = float(t.item())
 
     loss = None if args.no_loss else time_token_loss(P, gp, b, db, alg, flush, stream, args)
-    layer = time_layer_budget(P, b, flush, stream, args) if b.get("parent") is not None else None
+    eff = None if args.no_loss else time_efficiency(P, gp, db, out, wsp, flush, stream, args)
+    layer = None
+    if not args.no_loss:  # per-layer merge on the branching workload (this one if branching)
+        tb = b if b.get("parent") is not None else make_workload("tree", rank)
+        layer = time_layer_budget(P, tb, flush, stream, args)
+        layer["workload"] = WORKLOADS["tree"] if tb is not b else "this workload"
 
     if rank != 0:
         return 0
@@ -498,6 +531,8 @@ def run_ours(args):
                             "traffic": traffic, "traffic_note": tnote, "algorithmic_bytes": lb,
                             "peak_source": f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured" else "fallback"}
         line["token_loss"] = loss
+    if eff is not None:
+        line["efficiency"] = eff
     if layer is not None:
         lb = layer.pop("bytes")
         achieved = lb / (layer["ms"] / 1e3) / 1e9
@@ -518,7 +553,8 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--config", choices=list(WORKLOADS), default="math")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--no-loss", action="store_true", help="skip the policy-loss measurement")
+    ap.add_argument("--no-loss", action="store_true",
+                    help="skip the measurements of the widenings (policy loss, efficiency outputs, per-layer merge)")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)

@@ -199,7 +199,7 @@ class Batch:
     def c_struct(self) -> CBatch:
         import torch
         e = self.emb
-        assert e.dim() == 2 and e.stride(1) == 1, "embeddings must be [N, d] with unit inner stride"
+        assert e.dim() == 2 and (e.numel() == 0 or e.stride(1) == 1), "embeddings must be [N, d] with unit inner stride"
         dt = EMB_BF16 if e.dtype == torch.bfloat16 else EMB_F32
         if e.dtype not in (torch.bfloat16, torch.float32):
             raise TypeError("embeddings must be bfloat16 or float32")
