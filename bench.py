@@ -329,6 +329,34 @@ def time_layer_budget(P, b, flush, stream, args):
             "states_per_s": N / (ms / 1e3), "bytes": nbytes, "b_next": int(b["spec"].schedule[H - 1])}
 
 
+def max_over_ranks(x, device=None):
+    """The largest of the ranks' x (all ranks get it); x itself with one rank."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return x
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(x, device=None):
+    """The sum of the ranks' x (all ranks get it); x itself with one rank."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return x
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+def whole_job_value(tokens_all_ranks, ms_per_step):
+    """Tokens/s of the whole job: every rank labels its own batch of the same shape (weak
+    scaling); the job's tokens are all ranks' and it takes as long as its slowest rank."""
+    return tokens_all_ranks / (ms_per_step / 1e3)
+
+
 def dist_env():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     return ws, int(os.environ.get("RANK", "0")), int(os.environ.get("LOCAL_RANK", "0"))
@@ -441,13 +469,10 @@ def run_ours(args):
     gp.check()
     gp.enable_timing(False)
     total_ms = sum(step_ms)
-    if ws_n > 1:
-        import torch.distributed as dist
-        t = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(total_ms, dev)
     ms = total_ms / args.steps
-    value = ws_n * alg["T"] / (ms / 1e3)
+    tokens_all = sum_over_ranks(alg["T"], dev)  # the ranks' batches differ in their random lengths
+    value = whole_job_value(tokens_all, ms)
 
     # end to end through the public API from pinned host buffers
     hb = P.Batch.from_arrays(b, device="cpu", pin=True)
@@ -467,11 +492,7 @@ def run_ours(args):
         e.synchronize()
         e2e_ms.append(s.elapsed_time(e))
     e2e_t = statistics.mean(e2e_ms)
-    if ws_n > 1:
-        import torch.distributed as dist
-        t = torch.tensor([e2e_t], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_t = float(t.item())
+    e2e_t = max_over_ranks(e2e_t, dev)
 
     loss = None if args.no_loss else time_token_loss(P, gp, b, db, alg, flush, stream, args)
     eff = None if args.no_loss else time_efficiency(P, gp, db, out, wsp, flush, stream, args)
@@ -518,7 +539,7 @@ def run_ours(args):
                           "frac": path_t / (ms / 1e3)},
         "stage_ms": stage_ms,
         "roofline": roof,
-        "e2e": {"value": ws_n * alg["T"] / (e2e_t / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": int(h2d),
+        "e2e": {"value": whole_job_value(tokens_all, e2e_t), "unit": "tokens/s", "h2d_bytes_per_step": int(h2d),
                 "d2h_bytes_per_step": int(4 * alg["T"]), "ms_per_step": e2e_t},
         "clocks": clk.summary(),
         "gpu_launches": nst * args.steps,
