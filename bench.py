@@ -224,9 +224,21 @@ def cpu_baseline(b, budget_s=6.0, max_groups=None):
         if time.perf_counter() - t_start > budget_s and len(times) >= 2:
             break
     t = statistics.median(times)
+    # the same oracle on one core, on the first groups of the sample (a few seconds)
+    one = W.sub_batch(sub, range(min(8, len(sub["group_rollout_off"]) - 1)))
+    t1 = []
+    t_start = time.perf_counter()
+    while True:
+        t0 = time.perf_counter()
+        oracle.run(one, params, threads=1, want={"adv"})
+        t1.append(time.perf_counter() - t0)
+        if time.perf_counter() - t_start > budget_s / 3 and len(t1) >= 2:
+            break
     return {"value": T / t, "unit": "tokens/s", "cores": cores, "kind": "oracle",
             "sample": f"{sample}, {len(times)} timed passes, median",
-            "graphs_per_s": (len(sub["group_rollout_off"]) - 1) / t}
+            "graphs_per_s": (len(sub["group_rollout_off"]) - 1) / t,
+            "single_thread": {"value": batch_tokens(one) / statistics.median(t1), "unit": "tokens/s", "cores": 1,
+                              "sample": f"the first {len(one['group_rollout_off']) - 1} groups, {len(t1)} passes, median"}}
 
 
 def time_token_loss(P, gp, b, db, alg, flush, stream, args):
