@@ -43,6 +43,24 @@ def depths(batch: dict) -> np.ndarray:
     return dep
 
 
+def registered_before(dep, u: int, v: int) -> bool:
+    """State u was registered before state v: an earlier layer, or the same layer and a
+    smaller index."""
+    return dep[u] < dep[v] or (dep[u] == dep[v] and u < v)
+
+
+def halved(b_next: int) -> int:
+    """The budget of a path that reached an existing class: half, at least one."""
+    return max(1, b_next // 2)
+
+
+def spread(saved: int, k: int):
+    """The saved budget over k non-redundant states, in registration order: an even
+    share each and one more for the first saved mod k."""
+    share, extra = divmod(saved, k)
+    return [share + (1 if rank < extra else 0) for rank in range(k)]
+
+
 def layer_budget(batch: dict, layer: int, b_next: int, active=None, params: dict | None = None) -> dict:
     import oracle
     if batch.get("parent") is None:
@@ -54,7 +72,7 @@ def layer_budget(batch: dict, layer: int, b_next: int, active=None, params: dict
     N = len(dep)
     act = np.ones(N, dtype=bool) if active is None else np.asarray(active).astype(bool)
     frontier = (dep == layer) & act
-    halved = max(1, b_next // 2)
+    half = halved(b_next)
     budget = np.zeros(N, dtype=np.int64)
     redundant = np.zeros(N, dtype=bool)
     gs = batch["group_state_off"]
@@ -65,17 +83,16 @@ def layer_budget(batch: dict, layer: int, b_next: int, active=None, params: dict
             if not frontier[v]:
                 continue
             for u in range(s0, s1):  # an earlier-registered member of v's class?
-                if u != v and label[u] == label[v] and (dep[u] < dep[v] or (dep[u] == dep[v] and u < v)):
+                if u != v and label[u] == label[v] and registered_before(dep, u, v):
                     redundant[v] = True
                     break
             if redundant[v]:
-                budget[v] = halved
-                saved += b_next - halved
+                budget[v] = half
+                saved += b_next - half
             else:
                 budget[v] = b_next
                 keep.append(v)
         if keep:
-            share, extra = divmod(saved, len(keep))
-            for rank, v in enumerate(keep):
-                budget[v] += share + (1 if rank < extra else 0)
+            for v, more in zip(keep, spread(saved, len(keep))):
+                budget[v] += more
     return dict(class_id=label, budget=budget, redundant=redundant, frontier=frontier)

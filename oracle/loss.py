@@ -94,6 +94,12 @@ def surrogate(ratio: np.ndarray, A: np.ndarray, clip_low: float, clip_high: floa
     return value, np.where(takes_unclipped, ratio * A, 0.0), ~takes_unclipped
 
 
+def kl_k3(x: np.ndarray):
+    """The k3 estimate e^x - x - 1 (x = log pi_ref - log pi_theta) and its derivative with
+    respect to log pi_theta, 1 - e^x."""
+    return np.expm1(x) - x, -np.expm1(x)
+
+
 def token_loss(batch: dict, logp, old_logp, ref_logp=None, edge_adv=None, edge_cor=None, edge_eff=None,
                edge_mask=None, clip_low: float = 0.2, clip_high: float = 0.2, beta: float = 0.0,
                lambda_eff: float = 1.0, form: str = "dual", norm: str = "edge") -> dict:
@@ -116,9 +122,7 @@ def token_loss(batch: dict, logp, old_logp, ref_logp=None, edge_adv=None, edge_c
     else:
         raise ValueError(form)
     if beta != 0.0:
-        x = np.asarray(ref_logp, dtype=np.float64) - logp
-        kl = np.expm1(x) - x  # k3 = exp(x) - x - 1
-        dkl = -np.expm1(x)    # d k3 / d logp = 1 - exp(x)
+        kl, dkl = kl_k3(np.asarray(ref_logp, dtype=np.float64) - logp)
     else:
         kl = dkl = np.zeros_like(logp)
     j_pg = float(np.sum(w * f))
