@@ -272,9 +272,21 @@ def time_token_loss(P, gp, b, db, alg, flush, stream, args):
         times.append(s.elapsed_time(e))
     gp.check(stream)
     ms = statistics.mean(times)
-    return {"ms": ms, "tokens_per_s": T / (ms / 1e3), "form": "dual", "norm": "edge", "beta_kl": 0.0,
-            "loss": float(out["loss"].cpu()[0]), "launches_per_step": 1,
-            "bytes": 12 * T + 16 * N}
+    res = {"ms": ms, "tokens_per_s": T / (ms / 1e3), "form": "dual", "norm": "edge", "beta_kl": 0.0,
+           "loss": float(out["loss"].cpu()[0]), "launches_per_step": 1,
+           "bytes": 12 * T + 16 * N}
+    if not args.no_cpu_baseline:  # the loss oracle (numpy fp64) on the same batch and inputs
+        import numpy as np
+        from oracle import loss as OL
+        A = np.random.default_rng(0).normal(0.0, 1.0, N)  # timing only: any per-edge advantages
+        ts = []
+        for _ in range(3):
+            t0 = time.perf_counter()
+            OL.token_loss(b, lp["logp"], lp["old_logp"], edge_adv=A)
+            ts.append(time.perf_counter() - t0)
+        res["cpu_baseline"] = {"value": T / statistics.median(ts), "unit": "tokens/s", "cores": 1, "kind": "oracle",
+                               "sample": "the whole batch, 3 passes, median (numpy, one thread)"}
+    return res
 
 
 def time_efficiency(P, gp, db, out, wsp, flush, stream, args):
@@ -337,8 +349,18 @@ def time_layer_budget(P, b, flush, stream, args):
     esz = 2 if t["emb_dtype"] == "bf16" else 4
     nbytes = N * t["emb"].shape[1] * esz + 4 * N + 4 * N + 4 * N + N
     ms = statistics.mean(times)
-    return {"ms": ms, "layer": H - 1, "states": N, "frontier": int((W.tree_depths(t) == H - 1).sum()), "active": int(t["active"].sum()),
-            "states_per_s": N / (ms / 1e3), "bytes": nbytes, "b_next": int(b["spec"].schedule[H - 1])}
+    res = {"ms": ms, "layer": H - 1, "states": N, "frontier": int((W.tree_depths(t) == H - 1).sum()),
+           "active": int(t["active"].sum()), "states_per_s": N / (ms / 1e3), "bytes": nbytes,
+           "b_next": int(b["spec"].schedule[H - 1])}
+    if not args.no_cpu_baseline:  # the budget oracle on the first groups (a bounded sample)
+        from oracle import budget as OB
+        sub = W.truncate_tree(W.sub_batch(b, range(min(8, len(b["group_rollout_off"]) - 1))), H - 1)
+        t0 = time.perf_counter()
+        OB.layer_budget(sub, H - 1, int(b["spec"].schedule[H - 1]), sub["active"], dict(kappa=b["kappa"]))
+        dt = time.perf_counter() - t0
+        res["cpu_baseline"] = {"value": len(sub["step_len"]) / dt, "unit": "states/s", "cores": 1, "kind": "oracle",
+                               "sample": f"the first {len(sub['group_state_off']) - 1} groups, one pass"}
+    return res
 
 
 def max_over_ranks(x, device=None):
