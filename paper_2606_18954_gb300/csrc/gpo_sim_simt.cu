@@ -42,10 +42,76 @@ __device__ __forceinline__ float ld_elem(const void* base, int64_t i) {
   return reinterpret_cast<const float*>(base)[i];
 }
 
+constexpr int kSmall = 64;   // rows and columns of a small item
+constexpr int kKs = 32;      // k-chunk of a small item (kKs x kSmall floats fit in As and in Bs)
+static_assert(kKs * kSmall <= kKc * (kTileM + 4) && kKs * kSmall <= kKc * (kTileN + 4), "small-item staging");
+
+// A small item: the same products, pair test and unions as the general path below, with
+// every thread on a 4 x 4 micro-tile of the 64 x 64 block (all 256 threads busy) and
+// k-chunks of kKs elements (fewer barriers and load round trips per item).  As / Bs are
+// the general path's staging arrays, viewed as [kKs][kSmall].
+template <bool kBf16>
+__device__ __forceinline__ void small_item(const gpo_batch& b, const Sizes& sz, const Item& item, int nrows, int send,
+                                           float* As, float* Bs, const int* rm_roll, const int* rm_depth,
+                                           const int* rm_end, const float* rm_rn, const int* cm_roll,
+                                           const int* cm_depth, const float* cm_rn, int* lp, bool tree, float kappa,
+                                           int rule) {
+  const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;  // columns 4 tx.., rows 4 ty..
+  float acc[4][4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+  for (int k0 = 0; k0 < sz.d; k0 += kKs) {
+    __syncthreads();
+    for (int e = threadIdx.x; e < kKs * nrows; e += kThreads) {
+      const int r = e / kKs, k = e % kKs;
+      const int row = item.row0 + r;
+      As[k * kSmall + r] = (row < send && k0 + k < sz.d) ? ld_elem<kBf16>(b.emb, (int64_t)row * sz.stride + k0 + k) : 0.f;
+    }
+    for (int e = threadIdx.x; e < kKs * item.ncols; e += kThreads) {
+      const int c = e / kKs, k = e % kKs;
+      Bs[k * kSmall + c] = k0 + k < sz.d ? ld_elem<kBf16>(b.emb, (int64_t)(item.col0 + c) * sz.stride + k0 + k) : 0.f;
+    }
+    __syncthreads();
+    if (ty * 4 < nrows && tx * 4 < item.ncols) {
+      const int kn = min(kKs, sz.d - k0);
+      for (int k = 0; k < kn; ++k) {
+        const float4 a = *reinterpret_cast<const float4*>(As + k * kSmall + ty * 4);
+        const float4 bv = *reinterpret_cast<const float4*>(Bs + k * kSmall + tx * 4);
+        const float av[4] = {a.x, a.y, a.z, a.w}, bw[4] = {bv.x, bv.y, bv.z, bv.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+          for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(av[i], bw[j], acc[i][j]);
+      }
+    }
+  }
+  __syncthreads();
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int r = ty * 4 + i;
+    if (r >= nrows || rm_roll[r] < 0) continue;
+    const int row = item.row0 + r;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int c = tx * 4 + j;
+      const int col = item.col0 + c;
+      // comparable: not the row's own rollout (tree layout: outside the row's subtree)
+      if (c >= item.ncols || col <= row || (tree ? col < rm_end[r] : cm_roll[c] == rm_roll[r])) continue;
+      if (rule == GPO_MERGE_SAME_DEPTH && cm_depth[c] != rm_depth[r]) continue;
+      if (acc[i][j] * rm_rn[r] * cm_rn[c] >= kappa) {
+        const int sc = (col < item.row0 + kTileM) ? col - item.row0 : kTileM + (col - item.col0);
+        sunion(lp, r, sc);
+      }
+    }
+  }
+}
+
 template <bool kBf16>
 __global__ void __launch_bounds__(kThreads) sim_simt_kernel(gpo_batch b, Sizes sz, Ws ws, float kappa, int rule) {
-  __shared__ float As[kKc][kTileM + 4];
-  __shared__ float Bs[kKc][kTileN + 4];
+  __shared__ __align__(16) float As[kKc][kTileM + 4];
+  __shared__ __align__(16) float Bs[kKc][kTileN + 4];
   __shared__ int lp[kSlots];
   __shared__ int cm_roll[kTileN], cm_depth[kTileN];
   __shared__ float cm_rn[kTileN];
@@ -86,6 +152,13 @@ __global__ void __launch_bounds__(kThreads) sim_simt_kernel(gpo_batch b, Sizes s
     }
     if (threadIdx.x == 0) edge_n = 0;
 
+    const int nrows = min(kTileM, send - item.row0);
+    if (nrows <= kSmall && item.ncols <= kSmall) {
+      // a small item (groups of at most 64 states): every thread one 4 x 4 micro-tile of the
+      // 64 x 64 block, k-chunks of kKs staged at once
+      small_item<kBf16>(b, sz, item, nrows, send, &As[0][0], &Bs[0][0], rm_roll, rm_depth, rm_end, rm_rn, cm_roll,
+                        cm_depth, cm_rn, lp, tree, kappa, rule);
+    } else {
     float acc[8][16];
 #pragma unroll
     for (int i = 0; i < 8; ++i)
@@ -93,7 +166,6 @@ __global__ void __launch_bounds__(kThreads) sim_simt_kernel(gpo_batch b, Sizes s
       for (int j = 0; j < 16; ++j) acc[i][j] = 0.f;
     // only the tile's valid rows and columns are staged and multiplied (a thread's rows
     // and columns past them accumulate stale values that the epilogue never reads)
-    const int nrows = min(kTileM, send - item.row0);
     const bool busy = ty * 8 < nrows && tx * 16 < item.ncols;
 
     for (int k0 = 0; k0 < sz.d; k0 += kKc) {
@@ -143,6 +215,7 @@ __global__ void __launch_bounds__(kThreads) sim_simt_kernel(gpo_batch b, Sizes s
           sunion(lp, r, sc);
         }
       }
+    }
     }
     __syncthreads();
     int2* out = ws.edges + (size_t)it * kEdgeCap;
