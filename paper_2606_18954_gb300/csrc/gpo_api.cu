@@ -386,8 +386,16 @@ gpo_status compute_impl(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs*
     // one group per CTA: the group warps compute the compensated row statistics while the
     // group streams in (one launch); more groups than CTAs: a launch of their own first
     // (on the whole GPU), so that the group warps keep pace with the stream
-    pp.stats_in_kernel = !bud && (int64_t)(g1 - g0) <= (int64_t)fused_grid(lc, sz);
-    if (e == cudaSuccess && !bud && !pp.stats_in_kernel) e = stage("exact_stats", launch_exact_stats(lc, b, sz, ws));
+    // the group warps compute the compensated statistics of each CTA's first group while
+    // it streams in; the groups after those (more groups than CTAs) get theirs from a
+    // launch of its own first, on the whole GPU
+    pp.stats_in_kernel = !bud;
+    const int grid = fused_grid(lc, sz);
+    if (e == cudaSuccess && !bud && (int64_t)(g1 - g0) > (int64_t)grid) {
+      Sizes rest = sz;
+      rest.g0 = sz.g0 + grid;
+      e = stage("exact_stats", launch_exact_stats(lc, b, rest, ws));
+    }
     if (e == cudaSuccess) e = stage("fused", launch_fused(lc, map, map32, b, *out, sz, ws, pp));
   } else {
   if (e == cudaSuccess && b.parent) e = stage("tree_prep", launch_tree_prep(lc, b, sz, ws));

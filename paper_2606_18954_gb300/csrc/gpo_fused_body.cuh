@@ -627,13 +627,14 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
       // ---- compensated row statistics of the group (eta needs them; the Gram accumulator
       //      is too coarse): |z_v|^2 and <z_{p(v)}, z_v> as float pairs into ws.x_n2 / x_dot,
       //      by the group warps while the producer streams the same rows (L2 serves the
-      //      second reader; only when every CTA has one group, so that this work overlaps
-      //      the stream instead of delaying the next group).  A warp takes 8 rows, lane 4 r + c every fourth 16-byte chunk of
+      //      second reader; only for each CTA's first group, whose stream has nothing to
+      //      overlap before it, so that the work does not delay the CTA's next groups).  A warp takes 8 rows, lane 4 r + c every fourth 16-byte chunk of
       //      row r starting at chunk c; a parent that is the row before comes from the lane
       //      4 below, other parents and the prompt embedding are loaded.  bf16 products are
       //      exact in fp32, every sum is compensated (TwoSum per element, two fp32 lanes per
       //      instruction), the row's 4 partial pairs are combined in a fixed butterfly.
-      if (valid && p.mode == 0 && p.stats_in_kernel) group_row_stats(b, sz, ws, gs, g, s0, n, tree, wg, lane, st);
+      if (valid && p.mode == 0 && p.stats_in_kernel && g < sz.g0 + (int)gridDim.x)
+        group_row_stats(b, sz, ws, gs, g, s0, n, tree, wg, lane, st);
 
       // ---- drain the accumulator pass by pass (warps 4..15)
       bool fail = false;

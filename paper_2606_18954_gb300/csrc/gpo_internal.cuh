@@ -87,6 +87,7 @@ struct Params {
   // mode 1: next-layer budgets after layer `layer` instead of advantages (gpo_layer_budget)
   int mode, layer, b_next;
   int stats_in_kernel;    // fused path: the group warps compute the compensated row statistics
+                          // of each CTA's first group (the other groups' come from exact_stats)
   int pad_;
   const uint8_t* active;  // [N] frontier states to expand (NULL: all of depth `layer`)
   int32_t* budget;        // [N] output of mode 1
