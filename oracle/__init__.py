@@ -6,8 +6,10 @@ use this package.  The product path (`paper_2606_18954_gb300`) never imports it.
 """
 from __future__ import annotations
 
+import contextlib
 import ctypes
 import os
+import shutil
 import subprocess
 import threading
 
@@ -89,6 +91,39 @@ def _load():
             lib.oracle_validate.restype = ctypes.c_int
             _lib = lib
     return _lib
+
+
+@contextlib.contextmanager
+def library(path: str):
+    """Runs the oracle from another build of its C source (for the tests' mutation
+    checks, which compile deliberately broken copies) inside the block."""
+    global _lib
+    _load()
+    with _lock:
+        saved = _lib
+        lib = ctypes.CDLL(path)
+        lib.oracle_run.argtypes = saved.oracle_run.argtypes
+        lib.oracle_run.restype = ctypes.c_int
+        lib.oracle_validate.argtypes = saved.oracle_validate.argtypes
+        lib.oracle_validate.restype = ctypes.c_int
+        _lib = lib
+    try:
+        yield
+    finally:
+        with _lock:
+            _lib = saved
+
+
+def compile_variant(source: str, out_dir: str) -> str:
+    """Compiles C source text of the oracle (the header beside it) like build() does."""
+    src = os.path.join(out_dir, "oracle.c")
+    with open(src, "w") as f:
+        f.write(source)
+    shutil.copy(os.path.join(_HERE, "oracle.h"), os.path.join(out_dir, "oracle.h"))
+    so = os.path.join(out_dir, "liboracle_variant.so")
+    subprocess.check_call(["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-pthread", "-ffp-contract=off", src, "-o", so,
+                           "-lm"])
+    return so
 
 
 def default_params(batch: dict, **kw) -> dict:

@@ -94,6 +94,21 @@ def test_tree_root_embedding_variant(oracle_mod):
     np.testing.assert_allclose(out["a_cor"][[0, 5]], [-v, v], rtol=1e-12)
 
 
+def test_tree_eta_is_clamped_at_zero(oracle_mod):
+    """eta = max(0, sim) (Sec. 4.3): with E's embedding anti-parallel to its parent B
+    (cosine -1) eta(B, E) is 0, not -1, so r(E) = S(E) - S(B) = 1 - 2/3 = 1/3 (the
+    unclamped value would double it); no other link changes (E is orthogonal to the
+    others and anti-parallel to D, which stays unmerged)."""
+    fx = golden("tree_micro.json")
+    b = _fixture_batch(fx)
+    b["emb"] = b["emb"].copy()
+    b["emb"][6] = -b["emb"][5]
+    out = oracle_mod.run(b, fx["params"])
+    assert out["eta"][6] == 0.0
+    assert out["step_reward"][6] == pytest.approx(1.0 / 3.0, abs=1e-15)
+    np.testing.assert_array_equal(out["class_id"], [0, 1, 2, 1, 4, 2, 6])
+
+
 # ------------------------------------------------------------------ chain layout as a tree
 
 
