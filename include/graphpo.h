@@ -166,8 +166,11 @@ typedef struct gpo_ctx gpo_ctx;
  * sm_103, GPO_ERR_CUDA if the runtime fails. */
 gpo_status gpo_create(gpo_ctx** ctx, const gpo_params* params);
 
-/* Bytes of device workspace gpo_compute needs for batches of this shape
- * (reads only the host-side sizes of `batch`). */
+/* Bytes of device workspace gpo_compute needs for batches of this shape.
+ * Reads only the host-side sizes of `batch` and the nullness and alignment of
+ * its pointers (no device access), and returns the status gpo_compute would
+ * give for those checks.  `ctx` may be NULL (no device or context needed);
+ * with a context, the reason for a failure is left in gpo_last_error. */
 gpo_status gpo_workspace_size(const gpo_ctx* ctx, const gpo_batch* batch, size_t* bytes);
 
 /* Enqueues the whole path on `stream` (a cudaStream_t; NULL = legacy default

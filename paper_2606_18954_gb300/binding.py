@@ -151,6 +151,30 @@ def load(build_if_missing: bool = False):
         return L
 
 
+def workspace_size(batch, ctx=None) -> int:
+    """Device workspace bytes of gpo_compute for this batch (a `Batch`, or a `CBatch`).
+    Reads only the batch's host-side sizes, pointer nullness and alignment: no device
+    is needed without a context."""
+    L = load()
+    cb = batch if isinstance(batch, CBatch) else batch.c_struct()
+    n = ctypes.c_size_t()
+    code = L.gpo_workspace_size(ctx, ctypes.byref(cb), ctypes.byref(n))
+    if code != GPO_OK:
+        raise GraphPOError(code, L.gpo_last_error(ctx).decode() if ctx else "gpo_workspace_size")
+    return n.value
+
+
+def loss_plan_size(batch) -> int:
+    """Device bytes of the token-loss plan for this batch (no device needed)."""
+    L = load()
+    cb = batch if isinstance(batch, CBatch) else batch.c_struct()
+    n = ctypes.c_size_t()
+    code = L.gpo_loss_plan_size(ctypes.byref(cb), ctypes.byref(n))
+    if code != GPO_OK:
+        raise GraphPOError(code, "gpo_loss_plan_size")
+    return n.value
+
+
 def _ptr(t) -> Optional[int]:
     return None if t is None else t.data_ptr()
 
@@ -293,12 +317,7 @@ class GraphPO:
         return self._lib.gpo_last_error(self._h).decode()
 
     def workspace_size(self, batch: Batch) -> int:
-        n = ctypes.c_size_t()
-        cb = batch.c_struct()
-        code = self._lib.gpo_workspace_size(self._h, ctypes.byref(cb), ctypes.byref(n))
-        if code != GPO_OK:
-            raise GraphPOError(code, self.last_error())
-        return n.value
+        return workspace_size(batch, self._h)
 
     def workspace(self, batch: Batch):
         import torch
@@ -397,12 +416,9 @@ class GraphPO:
         if stream is None:
             stream = torch.cuda.current_stream(batch.step_len.device)
         cb = batch.c_struct()
-        n = ctypes.c_size_t()
-        code = self._lib.gpo_loss_plan_size(ctypes.byref(cb), ctypes.byref(n))
-        if code != GPO_OK:
-            raise GraphPOError(code, "gpo_loss_plan_size")
-        if plan is None or plan.numel() < n.value:
-            plan = torch.empty(max(n.value, 256), dtype=torch.uint8, device=batch.step_len.device)
+        need = loss_plan_size(cb)
+        if plan is None or plan.numel() < need:
+            plan = torch.empty(max(need, 256), dtype=torch.uint8, device=batch.step_len.device)
         code = self._lib.gpo_loss_plan(self._h, ctypes.byref(cb), plan.data_ptr(), plan.numel(),
                                        ctypes.c_void_p(stream.cuda_stream))
         if code != GPO_OK:

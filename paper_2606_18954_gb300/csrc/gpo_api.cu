@@ -181,7 +181,7 @@ gpo_status check_batch(gpo_ctx* c, const gpo_batch* b) {
   if (b->num_rollouts > 0 && !b->reward) return set_msg(c, "reward NULL"), GPO_ERR_INVALID_ARG;
   if ((b->emb && !aligned(b->emb, 16)) || (b->root_emb && !aligned(b->root_emb, 16)))
     return set_msg(c, "embeddings must be 16-byte aligned"), GPO_ERR_UNSUPPORTED;
-  if ((int64_t)b->num_states * b->emb_row_stride >= (int64_t)1 << 40)
+  if (b->emb_row_stride >= (int64_t)1 << 40 || (int64_t)b->num_states * b->emb_row_stride >= (int64_t)1 << 40)
     return set_msg(c, "embedding matrix too large"), GPO_ERR_UNSUPPORTED;
   return GPO_OK;
 }
@@ -271,7 +271,7 @@ void gpo_destroy(gpo_ctx* ctx) {
 }
 
 gpo_status gpo_workspace_size(const gpo_ctx* ctx, const gpo_batch* batch, size_t* bytes) {
-  if (!ctx || !bytes) return GPO_ERR_INVALID_ARG;
+  if (!bytes) return GPO_ERR_INVALID_ARG;
   gpo_status s = check_batch(const_cast<gpo_ctx*>(ctx), batch);
   if (s != GPO_OK) return s;
   Layout L;
@@ -342,6 +342,12 @@ gpo_status compute_impl(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs*
   lc.num_sms = ctx->num_sms;
 
   const bool use_tc = b.emb_dtype == GPO_EMB_BF16 && !(p.flags & GPO_FLAG_SIMT_SIMILARITY) && sz.N > 0;
+  const bool fused = use_tc && !(p.flags & GPO_FLAG_TILED) && sz.G > 0 && sz.maxn <= kFusedMaxStates;
+  const bool whole = g0 == 0 && g1 == sz.G;
+  if (!whole && !fused && g1 > g0) {
+    return set_msg(ctx, "a group range needs the group-resident path (bf16, at most %d states per group, no flags)",
+                   kFusedMaxStates), GPO_ERR_UNSUPPORTED;
+  }
   // embedding tensor maps: boxes of 64 elements x 128 rows and x 32 rows, 128B swizzle
   CUtensorMap map, map32;
   memset(&map, 0, sizeof map);
@@ -374,12 +380,6 @@ gpo_status compute_impl(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs*
   cudaError_t e = cudaSuccess;
   if (ctx->timing) e = cudaEventRecord(ctx->ev[0], lc.stream);
   if (e == cudaSuccess && clear) e = cudaMemsetAsync(ws.status, 0, sizeof(uint32_t) * kStatusWords, lc.stream);
-  const bool fused = use_tc && !(p.flags & GPO_FLAG_TILED) && sz.G > 0 && sz.maxn <= kFusedMaxStates;
-  const bool whole = g0 == 0 && g1 == sz.G;
-  if (!whole && !fused && g1 > g0) {
-    return set_msg(ctx, "a group range needs the group-resident path (bf16, at most %d states per group, no flags)",
-                   kFusedMaxStates), GPO_ERR_UNSUPPORTED;
-  }
   if (g1 <= g0) {
     // nothing to compute (a call that only clears the status words)
   } else if (fused) {
