@@ -99,7 +99,8 @@ def loss_tolerances(b, lp, A1, A2, mask, lam, beta, norm, clip=(0.2, 0.2)):
     return f.sum(), g
 
 
-def run_loss(P, b, lp, form, norm, beta, lam, A=None, cor=None, eff=None, mask=None, db=None, plan=None, gp=None):
+def run_loss(P, b, lp, form, norm, beta, lam, A=None, cor=None, eff=None, mask=None, db=None, plan=None, gp=None,
+             clip_low=0.2, clip_high=0.2):
     import torch
     gp = gp or P.GraphPO()
     db = db or P.Batch.from_arrays(b, device="cuda")
@@ -108,7 +109,7 @@ def run_loss(P, b, lp, form, norm, beta, lam, A=None, cor=None, eff=None, mask=N
     t = lambda x, dt=torch.float32: None if x is None else torch.as_tensor(np.asarray(x), dtype=dt, device=dev)
     out = gp.token_loss(db, plan, t(lp["logp"]), t(lp["old_logp"]), t(lp["ref_logp"]) if beta > 0 else None,
                         edge_adv=t(A), edge_cor=t(cor), edge_eff=t(eff), edge_eff_mask=t(mask, torch.uint8),
-                        beta_kl=beta, lambda_eff=lam, form=form, norm=norm)
+                        beta_kl=beta, lambda_eff=lam, form=form, norm=norm, clip_low=clip_low, clip_high=clip_high)
     gp.check()
     torch.cuda.synchronize()
     return {k: v.cpu().numpy() for k, v in out.items()}
@@ -171,6 +172,26 @@ def test_loss_parity(gp_mod, bname, form, norm, beta):
     A1, A2 = (A, None) if form == "dual" else (cor, eff)
     scale, gscale = loss_tolerances(b, lp, A1, A2, mask, lam, beta, norm)
     check_loss(gpu, ref, scale, gscale, f"{bname}/{form}/{norm}/{beta}")
+
+
+@pytest.mark.parametrize("form", ["dual", "split"])
+def test_loss_decoupled_clip(gp_mod, form):
+    """DAPO's decoupled bounds (clip range [0.8, 1.28]); the log-probabilities keep their
+    ratios 1e-4 away from both bounds, so both sides clip the same tokens."""
+    b = batch_of("agentic", 4)
+    T = int(b["rollout_token_off"][-1])
+    lp = W.make_logprobs(T, W.config_seed("agentic") + W.LOGP_SEED_OFFSET + 7, clip_low=0.2, clip_high=0.28,
+                         spread=0.25)
+    _, A, cor, eff, mask = loss_inputs(b, 81)
+    ref = OL.token_loss(b, lp["logp"], lp["old_logp"], lp["ref_logp"], edge_adv=A, edge_cor=cor, edge_eff=eff,
+                        edge_mask=mask, beta=0.05, lambda_eff=0.7, form=form, clip_low=0.2, clip_high=0.28)
+    r = np.exp(lp["logp"].astype(np.float64) - lp["old_logp"])
+    assert ((r > 1.2) & (r < 1.28)).any()  # tokens that only the upper bound's change leaves unclipped
+    gpu = run_loss(gp_mod, b, lp, form, "edge", 0.05, 0.7, A=A, cor=cor, eff=eff, mask=mask, clip_low=0.2,
+                   clip_high=0.28)
+    A1, A2 = (A, None) if form == "dual" else (cor, eff)
+    scale, gscale = loss_tolerances(b, lp, A1, A2, mask, 0.7, 0.05, "edge", clip=(0.2, 0.28))
+    check_loss(gpu, ref, scale, gscale, f"decoupled/{form}")
 
 
 @pytest.mark.parametrize("layout", ["chain", "tree"])

@@ -54,6 +54,57 @@ MUTANTS = {
     "tree reachability counts every step": (
         "if (c_own[i] > 0.0) good_tree += len;",
         "if (c_own[i] >= 0.0) good_tree += len;"),
+    "same-depth rule ignored": (
+        "if (p->merge_rule == 1 && G.depth[i] != G.depth[j]) continue;",
+        "if (0) continue;"),
+    "prompt embedding ignored": (
+        "if (u > 0 || G.has_root_emb) sim = cosine(&G, d, u, i);",
+        "if (u > 0) sim = cosine(&G, d, u, i);"),
+    "root statistics not gathered": (
+        "      c_own[G.parent[i]] += c_own[i];\n      t_own[G.parent[i]] += t_own[i];",
+        "      if (G.parent[i] > 0) c_own[G.parent[i]] += c_own[i];\n"
+        "      if (G.parent[i] > 0) t_own[G.parent[i]] += t_own[i];"),
+    "terminal counts not propagated": (
+        "t_own[G.parent[i]] += t_own[i];",
+        "t_own[G.parent[i]] += 1.0;"),
+    "every terminal correct": (
+        "c_own[i] += (double)b->reward[G.rollout[i]];",
+        "c_own[i] += 1.0;"),
+    "pooling counts the state among the others": (
+        "if (q == i) continue;",
+        "if (0) continue;"),
+    "correctness group of one member's children": (
+        "for (int m = G.mem_off[L]; m < G.mem_off[L + 1]; ++m) {\n      const int q = G.mem_list[m];\n"
+        "      for (int c = G.child_off[q]",
+        "for (int m = G.mem_off[L]; m < G.mem_off[L] + 1; ++m) {\n      const int q = G.mem_list[m];\n"
+        "      for (int c = G.child_off[q]"),
+    "population std": (
+        "return sqrt(s / (n - ddof));",
+        "return sqrt(s / n);"),
+    "class score summed, not averaged": (
+        "sbar /= Q;",
+        "sbar /= 1;"),
+    "route contributions overwritten": (
+        "e_eff[x] += A;",
+        "e_eff[x] = A;"),
+    "lambda ignored on tokens": (
+        "      const double dual = a_cor[i] + p->lambda_eff * e_eff[i];\n      for (int k = 0;",
+        "      const double dual = a_cor[i] + e_eff[i];\n      for (int k = 0;"),
+    "lambda ignored on edges": (
+        "    const double dual = a_cor[i] + p->lambda_eff * e_eff[i];\n    if (o->class_id)",
+        "    const double dual = a_cor[i] + e_eff[i];\n    if (o->class_id)"),
+    "graph reachability seeded by every terminal": (
+        "if (G.terminal[i] && b->reward[G.rollout[i]] && !reach[G.label[i]]) {",
+        "if (G.terminal[i] && !reach[G.label[i]]) {"),
+    "cosine without the norms": (
+        "return dot / (G->nrm[i] * G->nrm[j]);",
+        "return dot;"),
+    "leaves matched to rollouts in reverse": (
+        "G.rollout[i] = G.terminal[i] ? r0 + k++ : -1;",
+        "G.rollout[i] = G.terminal[i] ? r1 - 1 - k++ : -1;"),
+    "mask only on the member's own edge": (
+        "        emask[x] = 1;",
+        "        emask[v] = 1;"),
 }
 
 
@@ -62,6 +113,9 @@ def _pins(oracle_mod):
         lambda: CP.test_micro_worked_example(oracle_mod),
         lambda: CP.test_threshold_is_inclusive(oracle_mod),
         lambda: CP.test_classes_are_library_connected_components(oracle_mod, "tiny", 8, 0),
+        lambda: CP.test_classes_are_library_connected_components(oracle_mod, "tiny", 8, 1),
+        lambda: CP.test_micro_root_embedding_variant(oracle_mod),
+        lambda: TP.test_tree_root_embedding_variant(oracle_mod),
         lambda: CP.test_group_invariants(oracle_mod, "tiny", 8),
         lambda: CP.test_routes_by_path_enumeration(oracle_mod),
         lambda: CP.test_two_edge_group_closed_form(oracle_mod),

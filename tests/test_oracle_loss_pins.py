@@ -44,6 +44,16 @@ def test_loss_worked_example_dual():
     np.testing.assert_allclose(out["grad"], t["grad"], rtol=1e-14, atol=1e-16)
 
 
+def test_loss_worked_example_decoupled_clip():
+    fx, b, logp, old = _micro()
+    c = fx["dual_decoupled_clip"]
+    out = OL.token_loss(b, logp, old, edge_adv=fx["dual"]["edge_adv"], clip_low=c["clip_low"],
+                        clip_high=c["clip_high"])
+    assert out["loss"] == pytest.approx(c["loss"], abs=1e-15)
+    np.testing.assert_allclose(out["grad"], c["grad"], rtol=1e-14, atol=1e-16)
+    assert out["clipped"] == c["clipped"]
+
+
 def test_loss_worked_example_kl():
     fx, b, logp, old = _micro()
     k = fx["dual_kl"]

@@ -61,6 +61,22 @@ def _surrogate_clip_grad(ratio, A, lo, hi):
     return np.minimum(u, c), np.where(take, c, 0.0), ~take  # derivative of clip(r) A
 
 
+def _surrogate_bounds_swapped(ratio, A, lo, hi):
+    u, c = ratio * A, np.clip(ratio, 1 - hi, 1 + lo) * A
+    take = u <= c
+    return np.minimum(u, c), np.where(take, ratio * A, 0.0), ~take
+
+
+def _weights_token_norm_per_edge(batch, norm="edge"):
+    edge, elen = OL.edge_of_token(batch)
+    if norm == "token":
+        return 1.0 / (len(np.unique(edge)) * elen)  # "token" taken as a mean over edges
+    grp = OL.group_of_state(batch)
+    G = len(batch["group_rollout_off"]) - 1
+    n_edges = np.bincount(grp, minlength=G).astype(np.float64)
+    return 1.0 / (float(np.count_nonzero(n_edges)) * n_edges[grp[edge]] * elen)
+
+
 def _kl_wrong_sign(x):
     return np.expm1(x) + x, -np.expm1(x)
 
@@ -75,6 +91,8 @@ LOSS_MUTANTS = {
     "max instead of min": ("surrogate", _surrogate_max),
     "gradient through clipped branch": ("surrogate", _surrogate_grad_always),
     "derivative of the clipped term": ("surrogate", _surrogate_clip_grad),
+    "clip bounds swapped": ("surrogate", _surrogate_bounds_swapped),
+    "token normalisation as an edge mean": ("token_weights", _weights_token_norm_per_edge),
     "k3 sign": ("kl_k3", _kl_wrong_sign),
     "k3 derivative sign": ("kl_k3", _kl_wrong_derivative),
 }
@@ -83,6 +101,7 @@ LOSS_MUTANTS = {
 def _loss_pins(oracle_mod):
     return [
         LP.test_loss_worked_example_dual,
+        LP.test_loss_worked_example_decoupled_clip,
         LP.test_loss_worked_example_kl,
         LP.test_loss_worked_example_split,
         lambda: LP.test_loss_at_ratio_one(oracle_mod, "chain"),
