@@ -383,12 +383,10 @@ gpo_status compute_impl(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs*
   if (g1 <= g0) {
     // nothing to compute (a call that only clears the status words)
   } else if (fused) {
-    // one group per CTA: the group warps compute the compensated row statistics while the
-    // group streams in (one launch); more groups than CTAs: a launch of their own first
-    // (on the whole GPU), so that the group warps keep pace with the stream
-    // the group warps compute the compensated statistics of each CTA's first group while
-    // it streams in; the groups after those (more groups than CTAs) get theirs from a
-    // launch of its own first, on the whole GPU
+    // one group per CTA at a time: the group warps compute the compensated statistics of
+    // each CTA's first group while it streams in; the groups after those (more groups than
+    // CTAs) get theirs from a launch of its own first, on the whole GPU, so that the group
+    // warps keep pace with the stream
     pp.stats_in_kernel = !bud;
     const int grid = fused_grid(lc, sz);
     if (e == cudaSuccess && !bud && (int64_t)(g1 - g0) > (int64_t)grid) {
@@ -398,18 +396,18 @@ gpo_status compute_impl(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs*
     }
     if (e == cudaSuccess) e = stage("fused", launch_fused(lc, map, map32, b, *out, sz, ws, pp));
   } else {
-  if (e == cudaSuccess && b.parent) e = stage("tree_prep", launch_tree_prep(lc, b, sz, ws));
-  if (e == cudaSuccess) e = stage("prep", launch_prep(lc, b, sz, ws));
-  if (e == cudaSuccess && sz.N > 0) {
-    // eta takes compensated norms and parent dots (exact_stats); the fp32 norms of the
-    // threshold test come from the Gram tiles (tcgen05) or from row_stats (CUDA cores)
-    if (!bud) e = stage("exact_stats", launch_exact_stats(lc, b, sz, ws));
-    if (e == cudaSuccess && !use_tc) e = stage("row_stats", launch_row_stats(lc, b, sz, ws));
-    if (e == cudaSuccess)
-      e = stage("similarity", use_tc ? launch_sim_tc(lc, map, b, sz, ws, pp) : launch_sim_simt(lc, b, sz, ws, pp));
-    if (e == cudaSuccess) e = stage("groups", launch_groups(lc, b, *out, sz, ws, pp));
-    if (e == cudaSuccess && !bud) e = stage("tokens", launch_tokens(lc, b, *out, sz, ws));
-  }
+    if (e == cudaSuccess && b.parent) e = stage("tree_prep", launch_tree_prep(lc, b, sz, ws));
+    if (e == cudaSuccess) e = stage("prep", launch_prep(lc, b, sz, ws));
+    if (e == cudaSuccess && sz.N > 0) {
+      // eta takes compensated norms and parent dots (exact_stats); the fp32 norms of the
+      // threshold test come from the Gram tiles (tcgen05) or from row_stats (CUDA cores)
+      if (!bud) e = stage("exact_stats", launch_exact_stats(lc, b, sz, ws));
+      if (e == cudaSuccess && !use_tc) e = stage("row_stats", launch_row_stats(lc, b, sz, ws));
+      if (e == cudaSuccess)
+        e = stage("similarity", use_tc ? launch_sim_tc(lc, map, b, sz, ws, pp) : launch_sim_simt(lc, b, sz, ws, pp));
+      if (e == cudaSuccess) e = stage("groups", launch_groups(lc, b, *out, sz, ws, pp));
+      if (e == cudaSuccess && !bud) e = stage("tokens", launch_tokens(lc, b, *out, sz, ws));
+    }
   }
   ctx->nstages = ns;
   ctx->last_status = ws.status;
