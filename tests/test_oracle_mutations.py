@@ -138,6 +138,10 @@ BUDGET_MUTANTS = {
     "no halving": ("halved", lambda b: b),
     "registration by index only": ("registered_before", lambda dep, u, v: u < v),
     "registration by layer only": ("registered_before", lambda dep, u, v: dep[u] < dep[v]),
+    "registration in reverse index order": ("registered_before",
+                                            lambda dep, u, v: dep[u] < dep[v] or (dep[u] == dep[v] and u > v)),
+    "registration with later layers first": ("registered_before",
+                                             lambda dep, u, v: dep[u] > dep[v] or (dep[u] == dep[v] and u < v)),
     "remainder to the last states": ("spread", lambda saved, k: [saved // k + (1 if r >= k - saved % k else 0)
                                                                 for r in range(k)]),
     "savings not spent": ("spread", lambda saved, k: [0] * k),
@@ -157,6 +161,16 @@ def test_budget_pins_catch_mutant(oracle_mod, monkeypatch, name):
     attr, fn = BUDGET_MUTANTS[name]
     monkeypatch.setattr(OB, attr, fn)
     assert _fails(_budget_pins(oracle_mod)), f"no pin catches the mutant: {name}"
+
+
+def test_budget_pins_catch_inactive_states_on_the_frontier(oracle_mod, monkeypatch):
+    orig = OB.layer_budget
+
+    def mutant(batch, layer, b_next, active=None, params=None):
+        return orig(batch, layer, b_next, None, params)  # every state of the layer expanded
+
+    monkeypatch.setattr(OB, "layer_budget", mutant)
+    assert _fails(_budget_pins(oracle_mod))
 
 
 def test_unmutated_budget_oracle_passes(oracle_mod):
