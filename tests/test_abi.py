@@ -92,3 +92,46 @@ def test_product_never_imports_the_oracle():
             if f.endswith((".py", ".cu", ".cuh", ".h")):
                 txt = open(os.path.join(dirpath, f)).read()
                 assert "import oracle" not in txt and "liboracle" not in txt and "oracle.c" not in txt, f
+
+
+C_CLIENT = r"""
+#include <stdio.h>
+#include <string.h>
+#include "graphpo.h"
+
+int main(void) {
+  /* a plain C99 client: the header needs no CUDA or C++ types; host-only calls work
+     without a device */
+  gpo_batch b;
+  size_t bytes = 0;
+  int32_t go[1] = {0}, so[1] = {0};
+  int64_t to[1] = {0};
+  memset(&b, 0, sizeof b);  /* an empty batch: no groups, rollouts, states or tokens */
+  b.d = 8;
+  b.emb_row_stride = 8;
+  b.group_rollout_off = go;  /* the offset arrays (G + 1, R + 1 entries) are required */
+  b.rollout_step_off = so;
+  b.rollout_token_off = to;
+  if (gpo_workspace_size(NULL, &b, &bytes) != GPO_OK || bytes == 0) return 1;
+  b.num_groups = -1;
+  if (gpo_workspace_size(NULL, &b, &bytes) != GPO_ERR_INVALID_ARG) return 2;
+  if (strncmp(gpo_version(), "graphpo-gb300", 13) != 0) return 3;
+  printf("%s|%s|%zu\n", gpo_version(), gpo_status_string(GPO_ERR_SHAPE), bytes);
+  return 0;
+}
+"""
+
+
+def test_header_is_plain_c_and_links(lib, tmp_path):
+    """include/graphpo.h compiles as C99 with warnings as errors, and a C program links
+    against the library and calls its host-only entry points."""
+    src = tmp_path / "client.c"
+    src.write_text(C_CLIENT)
+    exe = tmp_path / "client"
+    so = lib._name
+    subprocess.check_call(["gcc", "-std=c99", "-Wall", "-Wextra", "-Werror", "-pedantic", "-I",
+                           os.path.join(ROOT, "include"), str(src), "-o", str(exe), so,
+                           "-Wl,-rpath," + os.path.dirname(so)])
+    out = subprocess.run([str(exe)], capture_output=True, text=True)
+    assert out.returncode == 0, out
+    assert out.stdout.startswith("graphpo-gb300") and "inconsistent offsets" in out.stdout
