@@ -11,6 +11,16 @@ the device with CUDA events on the launching stream.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--config math]
 
+The same line carries `per_config`: the path timed the same way on each of the
+other workload shapes (tiny, agentic search, wide groups, full batch, and the
+branching-rollout tree layout), each with its own stage times, clocks and roofline.
+
+Roofline: the bound of a kernel is the slower of its algorithmic bytes at the
+measured HBM copy peak and its algorithmic FLOPs (the cosine GEMM's comparable upper
+triangle) at the measured bf16 tensor peak.  The fp32 work of the compensated eta
+statistics is an implementation device, not the method's work: it is reported apart
+(`alu_note`), never as the bound.
+
 Multi-GPU (torchrun, one rank per GPU): every rank runs its own batch of the same
 shape (weak scaling, no collective on the data path); value = tokens of all ranks
 divided by the slowest rank's time.  `--impl reference` times the CPU oracle.
@@ -432,48 +442,53 @@ def run_reference(args):
     return 0
 
 
-def run_ours(args):
-    import numpy as np
-    import torch
-    import paper_2606_18954_gb300 as P
-    from paper_2606_18954_gb300 import workloads as W
-
-    ws_n, rank, local = dist_env()
-    if ws_n > 1:
-        import torch.distributed as dist
-        torch.cuda.set_device(local)
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+def kernel_roofline(name, stage_ms, alg, hbm, tc, workload):
+    """Roofline of one kernel: its algorithmic bytes and FLOPs per launch (the method's
+    work, as `algorithmic` counts it) over its average launch time; the bound is the
+    slower of bytes at the HBM copy peak and FLOPs at the bf16 tensor peak (burst: each
+    kernel runs alone, well under a millisecond)."""
+    sb, sf = alg["stages"][name][:2]
+    t = stage_ms[name] / 1e3
+    if sf / (tc * 1e12) > sb / (hbm * 1e9):
+        roof = {"bound": "tensor", "achieved": sf / t / 1e12, "peak": tc, "unit": "TFLOP/s",
+                "algorithmic": sf, "peak_kind": "bf16 dense, burst"}
     else:
-        torch.cuda.set_device(0)
-    dev = torch.device("cuda", torch.cuda.current_device())
-    P.build()
-    b = make_workload(args.config, rank)
+        roof = {"bound": "hbm", "achieved": sb / t / 1e9, "peak": hbm, "unit": "GB/s", "algorithmic": sb,
+                "peak_kind": "HBM copy"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    traffic, tnote = traffic_for(STAGE_SOURCE.get(name, ""), workload)
+    roof.update(kernel=name, ms_per_launch=stage_ms[name], traffic=traffic, traffic_note=tnote)
+    return roof
+
+
+def alu_note(name, stage_ms, alg):
+    """The compensated statistics' fp32 operations of a kernel against the fp32 issue peak
+    (an implementation device for the accuracy of eta, not part of the roofline)."""
+    st = alg["stages"][name]
+    if len(st) < 3 or not st[2]:
+        return None
+    peak = alu_peak_tops()
+    achieved = st[2] / (stage_ms[name] / 1e3) / 1e12
+    return {"kernel": name, "fp32_ops": st[2], "achieved": achieved, "peak": peak, "unit": "Top/s",
+            "frac": achieved / peak, "peak_note": "152 SMs x 128 fp32 lanes x the max SM clock"}
+
+
+def time_path(P, b, dev, stream, flush, args, barrier, bus):
+    """The whole path on one batch: W warm-up steps, then K steps each timed on the device
+    (CUDA events on the launching stream, L2 flushed before each), with the clocks sampled
+    meanwhile; then K more steps with the library's per-kernel events."""
+    import torch
     alg = algorithmic(b)
     db = P.Batch.from_arrays(b, device=dev)
     gp = P.GraphPO(kappa=b["kappa"], w=b["w"], lambda_eff=b["lambda_eff"])
     out = gp.alloc_outputs(db)
     wsp = gp.workspace(db)
-    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
-    stream = torch.cuda.current_stream(dev)
-
     for _ in range(args.warmup):
-        gp.compute_into(db, out, workspace=wsp)
-    gp.check()
+        gp.compute_into(db, out, workspace=wsp, stream=stream)
+    gp.check(stream)
     torch.cuda.synchronize()
-
-    def barrier():
-        if ws_n > 1:
-            import torch.distributed as dist
-            dist.barrier()
-
-    bus = None
-    try:
-        bus = torch.cuda.get_device_properties(dev).pci_bus_id
-    except Exception:
-        pass
-    # timed steps: device time of each step between events on the launching stream
-    # (the library's per-stage events are off here: they add a few microseconds per step)
-    step_ms, stage_acc, nst = [], {}, 0
+    # timed steps (the library's per-stage events are off here: they add a few microseconds)
+    step_ms = []
     barrier()
     torch.cuda.synchronize()
     with ClockSampler(bus) as clk:
@@ -488,9 +503,9 @@ def run_ours(args):
             step_ms.append(s.elapsed_time(e))
         torch.cuda.synchronize()
         barrier()
-    gp.check()
-    # per-kernel durations for the roofline: the same K steps again, with the library's
-    # CUDA events around each kernel on the launching stream
+    gp.check(stream)
+    # per-kernel durations: the same K steps again with CUDA events around each kernel
+    stage_acc, nst = {}, 0
     gp.enable_timing(True)
     for _ in range(args.steps):
         flush.zero_()
@@ -500,11 +515,72 @@ def run_ours(args):
         for k, v in st.items():
             stage_acc[k] = stage_acc.get(k, 0.0) + v
     torch.cuda.synchronize()
-    gp.check()
+    gp.check(stream)
     gp.enable_timing(False)
-    total_ms = sum(step_ms)
-    total_ms = max_over_ranks(total_ms, dev)
-    ms = total_ms / args.steps
+    return dict(alg=alg, db=db, gp=gp, out=out, wsp=wsp, step_ms=step_ms, clocks=clk.summary(),
+                stage_ms={k: v / args.steps for k, v in stage_acc.items()}, launches_per_step=nst)
+
+
+def config_summary(name, b, r, ms, tokens_all, n_ranks, peaks):
+    """Throughput, stage times, clocks and rooflines of one shape."""
+    hbm, tc = peaks[0], peaks[1]
+    alg, stage_ms = r["alg"], r["stage_ms"]
+    dom = max(stage_ms, key=stage_ms.get)
+    path_t = max(alg["path_bytes"] / (hbm * 1e9), alg["flops"] / (tc * 1e12))
+    res = {"workload": WORKLOADS[name], "ms_per_step": ms, "value": whole_job_value(tokens_all, ms),
+           "unit": "tokens/s", "graphs_per_s": n_ranks * alg["G"] / (ms / 1e3),
+           "groups": alg["G"], "rollouts": alg["R"], "states": alg["N"], "tokens": alg["T"],
+           "d": int(b["emb"].shape[1]), "emb_dtype": b["emb_dtype"],
+           "layout": "tree" if b.get("parent") is not None else "chain", "seed": _seed(name),
+           "path_roofline": {"bytes": alg["path_bytes"], "flops": alg["flops"], "roofline_us": path_t * 1e6,
+                             "bound": "tensor" if alg["flops"] / (tc * 1e12) > alg["path_bytes"] / (hbm * 1e9)
+                             else "hbm", "frac": path_t / (ms / 1e3)},
+           "stage_ms": stage_ms, "roofline": kernel_roofline(dom, stage_ms, alg, hbm, tc, name),
+           "clocks": r["clocks"], "gpu_launches": r["launches_per_step"] * len(r["step_ms"])}
+    note = alu_note(dom, stage_ms, alg)
+    if note is not None:
+        res["alu_note"] = note
+    return res
+
+
+def _seed(name):
+    from paper_2606_18954_gb300 import workloads as W
+    return W.config_seed(name)
+
+
+def run_ours(args):
+    import torch
+    import paper_2606_18954_gb300 as P
+
+    ws_n, rank, local = dist_env()
+    if ws_n > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    dev = torch.device("cuda", torch.cuda.current_device())
+    P.build()
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    peaks = load_peaks()
+    hbm, tc, tc_sus, peak_src = peaks
+
+    def barrier():
+        if ws_n > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    bus = None
+    try:
+        bus = torch.cuda.get_device_properties(dev).pci_bus_id
+    except Exception:
+        pass
+
+    b = make_workload(args.config, rank)
+    r = time_path(P, b, dev, stream, flush, args, barrier, bus)
+    alg, db, gp, out, wsp = r["alg"], r["db"], r["gp"], r["out"], r["wsp"]
+    ms = max_over_ranks(sum(r["step_ms"]), dev) / args.steps
     tokens_all = sum_over_ranks(alg["T"], dev)  # the ranks' batches differ in their random lengths
     value = whole_job_value(tokens_all, ms)
 
@@ -525,8 +601,8 @@ def run_ours(args):
         e.record(stream)
         e.synchronize()
         e2e_ms.append(s.elapsed_time(e))
-    e2e_t = statistics.mean(e2e_ms)
-    e2e_t = max_over_ranks(e2e_t, dev)
+    e2e_t = max_over_ranks(statistics.mean(e2e_ms), dev)
+    del hb, host_out
 
     loss = None if args.no_loss else time_token_loss(P, gp, b, db, alg, flush, stream, args)
     eff = None if args.no_loss else time_efficiency(P, gp, db, out, wsp, flush, stream, args)
@@ -536,48 +612,48 @@ def run_ours(args):
         layer = time_layer_budget(P, tb, flush, stream, args)
         layer["workload"] = WORKLOADS["tree"] if tb is not b else "this workload"
 
+    head = config_summary(args.config, b, r, ms, tokens_all, ws_n, peaks)
+    del r, db, gp, out, wsp
+
+    # the other shapes, timed the same way (same K and W), one after another
+    per_config = {}
+    others = [c for c in (WORKLOADS if args.per_config == "all" else
+                          ([] if args.per_config == "none" else args.per_config.split(",")))
+              if c != args.config]
+    for name in others:
+        bo = make_workload(name, rank)
+        ro = time_path(P, bo, dev, stream, flush, args, barrier, bus)
+        mo = max_over_ranks(sum(ro["step_ms"]), dev) / args.steps
+        to = sum_over_ranks(ro["alg"]["T"], dev)
+        per_config[name] = config_summary(name, bo, ro, mo, to, ws_n, peaks)
+        del ro, bo
+        torch.cuda.empty_cache()
+
     if rank != 0:
         return 0
-    hbm, tc, tc_sus, peak_src = load_peaks()
-    stage_ms = {k: v / args.steps for k, v in stage_acc.items()}
-    dom = max(stage_ms, key=stage_ms.get)
-    sb, sf, sa = (tuple(alg["stages"][dom]) + (0.0,))[:3]
-    t_dom = stage_ms[dom] / 1e3
-    alu = alu_peak_tops()
-    if sa and sa / (alu * 1e12) > max(sb / (hbm * 1e9), sf / (tc * 1e12)):
-        roof = {"bound": "alu", "achieved": sa / t_dom / 1e12, "peak": alu, "unit": "Top/s",
-                "peak_note": "fp32 lanes x SMs x max SM clock (152 x 128 x 2070 MHz); the kernel's HBM fraction "
-                             f"is {sb / t_dom / 1e9 / hbm:.3f} of measured"}
-    elif sf and sf / (tc * 1e12) > sb / (hbm * 1e9):
-        roof = {"bound": "tensor", "achieved": sf / t_dom / 1e12, "peak": tc, "unit": "TFLOP/s"}
-    else:
-        roof = {"bound": "hbm", "achieved": sb / t_dom / 1e9, "peak": hbm, "unit": "GB/s"}
-    roof["frac"] = roof["achieved"] / roof["peak"]
-    traffic, tnote = traffic_for(STAGE_SOURCE.get(dom, ""), args.config)
-    roof.update(traffic=traffic, kernel=dom, traffic_note=tnote,
-                peak_source=("derived from the measured max SM clock" if roof["bound"] == "alu" else
-                             f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured" else "fallback"))
-    path_t = max(alg["path_bytes"] / (hbm * 1e9), alg["flops"] / (tc * 1e12))
+    roof = dict(head["roofline"])
+    roof["peak_source"] = f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured" else "fallback"
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": ws_n, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": WORKLOADS[args.config], "groups": alg["G"], "rollouts": alg["R"],
-                   "states": alg["N"], "tokens": alg["T"], "d": int(b["emb"].shape[1]),
-                   "emb_dtype": b["emb_dtype"], "layout": "tree" if b.get("parent") is not None else "chain",
+                   "states": alg["N"], "tokens": alg["T"], "d": head["d"],
+                   "emb_dtype": b["emb_dtype"], "layout": head["layout"],
                    "merge_rule": "noncausal", "kappa": b["kappa"], "w": b["w"],
                    "lambda_eff": b["lambda_eff"], "l2": "flushed by a 256 MiB write before every timed step",
-                   "seed": W.config_seed(args.config)},
-        "graphs_per_s": ws_n * alg["G"] / (ms / 1e3),
-        "path_roofline": {"bytes": alg["path_bytes"], "flops": alg["flops"], "roofline_us": path_t * 1e6,
-                          "frac": path_t / (ms / 1e3)},
-        "stage_ms": stage_ms,
+                   "seed": _seed(args.config)},
+        "graphs_per_s": head["graphs_per_s"],
+        "path_roofline": head["path_roofline"],
+        "stage_ms": head["stage_ms"],
         "roofline": roof,
         "e2e": {"value": whole_job_value(tokens_all, e2e_t), "unit": "tokens/s", "h2d_bytes_per_step": int(h2d),
                 "d2h_bytes_per_step": int(4 * alg["T"]), "ms_per_step": e2e_t},
-        "clocks": clk.summary(),
-        "gpu_launches": nst * args.steps,
+        "clocks": head["clocks"],
+        "gpu_launches": head["gpu_launches"],
     }
+    if "alu_note" in head:
+        line["alu_note"] = head["alu_note"]
     if loss is not None:
         lb = loss.pop("bytes")
         achieved = lb / (loss["ms"] / 1e3) / 1e9
@@ -594,6 +670,8 @@ def run_ours(args):
         layer["roofline"] = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
                              "algorithmic_bytes": lb, "launches": "fused kernel alone (no row statistics)"}
         line["layer_budget"] = layer
+    if per_config:
+        line["per_config"] = per_config
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(b, max_groups={"wide": 2, "full": 64}.get(args.config))
     print(json.dumps(line), flush=True)
@@ -608,6 +686,8 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--config", choices=list(WORKLOADS), default="math")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--per-config", default="all",
+                    help="other shapes timed into per_config: 'all', 'none' or a comma-separated list")
     ap.add_argument("--no-loss", action="store_true",
                     help="skip the measurements of the widenings (policy loss, efficiency outputs, per-layer merge)")
     args = ap.parse_args()

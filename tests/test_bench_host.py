@@ -73,5 +73,32 @@ def test_traffic_lookup_follows_the_kernel_source():
     assert bench.traffic_for("gpo_fused.cu", "no such workload")[0] is None
 
 
+def test_kernel_roofline_takes_the_slower_of_bytes_and_flops():
+    """The bound of a kernel is max(bytes / HBM peak, FLOPs / tensor peak) of its
+    algorithmic work; the fp32 work of the compensated statistics never decides it and
+    is reported apart."""
+    b = W.make_batch(W.CONFIGS["math"].scaled(groups=3))
+    a = bench.algorithmic(b)
+    hbm, tc = 6686.8, 1877.4
+    ms = {"fused": 0.05, "exact_stats": 0.01, "similarity": 0.02}
+    r = bench.kernel_roofline("fused", ms, a, hbm, tc, "math")
+    assert r["bound"] == "hbm" and r["unit"] == "GB/s"
+    assert r["achieved"] == pytest.approx(a["path_bytes"] / 0.05e-3 / 1e9)
+    assert r["frac"] == pytest.approx(r["achieved"] / hbm)
+    assert r["algorithmic"] == a["path_bytes"]
+    # a contraction-heavy kernel: wide groups make the cosine GEMM the bound
+    a2 = dict(a)
+    a2["stages"] = dict(a["stages"], similarity=(1e6, 1e12))
+    r2 = bench.kernel_roofline("similarity", ms, a2, hbm, tc, "wide")
+    assert r2["bound"] == "tensor" and r2["achieved"] == pytest.approx(1e12 / 0.02e-3 / 1e12)
+    # the statistics kernel has no FLOPs of the method: HBM-bound, its fp32 work in the note
+    r3 = bench.kernel_roofline("exact_stats", ms, a, hbm, tc, "math")
+    assert r3["bound"] == "hbm"
+    note = bench.alu_note("exact_stats", ms, a)
+    assert note["fp32_ops"] == a["stages"]["exact_stats"][2]
+    assert note["frac"] == pytest.approx(note["achieved"] / bench.alu_peak_tops())
+    assert bench.alu_note("similarity", ms, a) is None
+
+
 def test_whole_job_value():
     assert bench.whole_job_value(4_000_000, 2.0) == pytest.approx(2e9)
