@@ -225,13 +225,18 @@ gpo_status gpo_stage_times(gpo_ctx* ctx, float* ms, const char** names, int capa
  * pool, a plug-in whose host forbids allocation calls, a loop that cannot take
  * cudaMalloc's implicit synchronisation.  Same inputs and outputs as
  * gpo_compute, but the workspace is one array of GPO_NOALLOC_SCRATCH_BYTES
- * compiled into the library (held by every GPU that loads it until exit); it
- * calls no cudaMalloc/cudaFree.  Batches whose gpo_workspace_size exceeds that
- * size are rejected with GPO_ERR_WORKSPACE before anything is enqueued.  The
- * first call on a device looks up the array's address; make it before any
- * stream capture.  All calls on a device share the array: calls that overlap on
- * the GPU race and must be ordered by the caller.  Errors and gpo_sync_status
- * behave as for gpo_compute. */
+ * compiled into the library; it calls no cudaMalloc/cudaFree.  The array
+ * belongs to a CUDA context, not to a device: it is reserved in the current
+ * context when this library's device code is first loaded there (at the latest
+ * by the first gpo_compute_noalloc call in that context) and stays there until
+ * the context is destroyed; every context has its own.  The first call in a
+ * context looks up the array's address in that context (it is cached per
+ * context, so other contexts and a new primary context after a device reset
+ * get their own); make that first call before any stream capture.  Batches
+ * whose gpo_workspace_size exceeds GPO_NOALLOC_SCRATCH_BYTES are rejected with
+ * GPO_ERR_WORKSPACE before anything is enqueued.  All calls in one context
+ * share the array: calls that overlap on the GPU race and must be ordered by
+ * the caller.  Errors and gpo_sync_status behave as for gpo_compute. */
 #define GPO_NOALLOC_SCRATCH_BYTES ((size_t)32 << 20)
 gpo_status gpo_compute_noalloc(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* out, void* stream);
 
