@@ -327,6 +327,11 @@ gpo_status compute_impl(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs*
   pp.w = p.w;
   pp.lambda_eff = p.lambda_eff;
   pp.eps = p.std_eps;
+  pp.kappa_f = (float)pp.kappa;
+  pp.w_hi = (float)pp.w;
+  pp.w_lo = (float)(pp.w - (double)pp.w_hi);
+  pp.lambda_f = (float)pp.lambda_eff;
+  pp.eps_f = (float)pp.eps;
   pp.ddof = p.std_ddof;
   pp.rule = p.merge_rule;
   pp.mode = bud ? 1 : 0;
@@ -606,6 +611,7 @@ gpo_status gpo_token_loss(gpo_ctx* ctx, const gpo_batch* batch, void* plan, cons
   a.hi = (float)(1.0 + p.clip_high);
   a.beta = (float)p.beta_kl;
   a.lambda = (float)p.lambda_eff;
+  a.inv_t = T > 0 ? (float)(1.0 / (double)T) : 0.f;
   a.norm_token = p.norm == GPO_LOSS_NORM_TOKEN;
   a.split = split;
   a.kl = kl;

@@ -405,7 +405,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
   uint32_t* st = ws.status;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int KT = (sz.d + kTileK - 1) / kTileK;
-  const float kappa = (float)p.kappa;
+  const float kappa = p.kappa_f;
 
   const bool tree = b.parent != nullptr;
   if (blockIdx.x == 0 && threadIdx.x == 0) {

@@ -206,8 +206,8 @@ template <int kPer, bool kZeroed, class IdxT, class Sync, class Eta, class Out>
 __device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const IdxT* roll, const IdxT* dep,
                                                  const int* rstart, const uint8_t* rew, const GroupScratch& sc,
                                                  const Params& p, int tid, int nt, Sync sync, Eta eta, Out out) {
-  const float w = (float)p.w, eps = (float)p.eps;
-  const float wl = (float)(p.w - (double)w);  // w = w + wl to ~2^-48
+  const float w = p.w_hi, eps = p.eps_f;
+  const float wl = p.w_lo;  // w = w + wl to ~2^-48
   // ---- phase A: class sums C_Q (rewards), |Q|, sum l, sum l^2
   if (!kZeroed) {
     for (int i = tid; i < n; i += nt) {
@@ -367,7 +367,7 @@ __device__ __forceinline__ void group_advantages(int n, int nr, int* lab, const 
     }
   }
   sync();
-  const float lam = (float)p.lambda_eff;
+  const float lam = p.lambda_f;
 #pragma unroll
   for (int k = 0; k < kPer; ++k) {
     const int i = tid + k * nt;
@@ -467,8 +467,8 @@ __device__ __forceinline__ void group_advantages_tree(int n, int nleaf, int* lab
                                                       const IdxT* end, const IdxT* cown, const IdxT* town,
                                                       const TreeScratch& sc, const Params& p, int tid, int nt,
                                                       Sync sync, Eta eta, Out out) {
-  const float w = (float)p.w, eps = (float)p.eps;
-  const float wl = (float)(p.w - (double)w);
+  const float w = p.w_hi, eps = p.eps_f;
+  const float wl = p.w_lo;
   for (int i = tid; i < sc.nzero; i += nt) sc.ccnt[i] = 0;
   sync();
   // ---- phase A: class sums
@@ -598,7 +598,7 @@ __device__ __forceinline__ void group_advantages_tree(int n, int nleaf, int* lab
     }
   }
   sync();
-  const float lam = (float)p.lambda_eff;
+  const float lam = p.lambda_f;
 #pragma unroll
   for (int k = 0; k < kPer; ++k) {
     const int i = tid + k * nt;

@@ -83,6 +83,8 @@ struct Sizes {
 
 struct Params {
   double kappa, w, lambda_eff, eps;
+  // the same in fp32, rounded once on the host: w = w_hi + w_lo to ~2^-48
+  float kappa_f, w_hi, w_lo, lambda_f, eps_f;
   int ddof, rule;
   // mode 1: next-layer budgets after layer `layer` instead of advantages (gpo_layer_budget)
   int mode, layer, b_next;
@@ -596,6 +598,7 @@ struct LossArgs {
   float* grad;
   double* stats;
   float lo, hi, beta, lambda;
+  float inv_t;           // (float)(1 / T) rounded once on the host (0 for T = 0)
   int norm_token;        // 1: weights 1/T
   int split, kl;
   int N;

@@ -183,7 +183,8 @@ struct LossSmem {
   float wa[kLossTile];                    // w A (dual) or w A_cor (split)
   float we[kSplit ? kLossTile : 1];       // split: w lambda m_eff A_eff
   float w[kKL ? kLossTile : 1];           // KL: w
-  double red[kLossThreads / 32][4];
+  float2 red[kLossThreads / 32][3];
+  long long redn[kLossThreads / 32];
   int last;
 };
 
@@ -197,8 +198,11 @@ __global__ void __launch_bounds__(kLossThreads, kKL ? 3 : 4) token_loss_kernel(L
     return;
   }
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const float inv_t = a.T > 0 ? (float)(1.0 / (double)a.T) : 0.f;
-  double acc[4] = {0.0, 0.0, 0.0, 0.0};  // policy term, KL term, clipped tokens, sum of r
+  const float inv_t = a.inv_t;
+  // across tiles: float pairs for the policy term, the KL term and the sum of r (every
+  // addition's rounding error kept in the low word), an integer count of clipped tokens
+  float2 acc[3] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+  long long nclip_all = 0;
   const int64_t ntiles = a.N > 0 ? lp.ntiles : 0;  // (a valid plan has no tokens without edges)
   for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
     const int64_t t0 = tile * kLossTile;
@@ -294,73 +298,98 @@ __global__ void __launch_bounds__(kLossThreads, kKL ? 3 : 4) token_loss_kernel(L
           for (int c = 0; rel + c < tn; ++c) a.grad[q + c] = gr[c];
       }
     }
-    acc[0] += (double)pg;
-    acc[1] += (double)kl;
-    acc[2] += (double)nclip;
-    acc[3] += (double)rs;
+    ff_acc(acc[0].x, acc[0].y, pg);
+    ff_acc(acc[1].x, acc[1].y, kl);
+    ff_acc(acc[2].x, acc[2].y, rs);
+    nclip_all += nclip;
   }
-  // CTA sums in a fixed tree, then the last CTA adds the partials in a fixed order
+  // CTA sums in a fixed tree of pair additions, then the last CTA adds the partials in a
+  // fixed order; the slots of lp.partial hold float pairs (and the clip count as an integer)
+  float2* part = reinterpret_cast<float2*>(lp.partial);
+  long long* part_n = reinterpret_cast<long long*>(lp.partial);
+  auto warp_tree = [&](float2 (&v)[3], long long& n) {
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
+    for (int o = 16; o > 0; o >>= 1) {
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) acc[i] += __shfl_xor_sync(0xffffffffu, acc[i], o);
-    if (lane == 0) sm.red[warp][i] = acc[i];
+      for (int i = 0; i < 3; ++i) {
+        const float2 u = make_float2(__shfl_xor_sync(0xffffffffu, v[i].x, o), __shfl_xor_sync(0xffffffffu, v[i].y, o));
+        v[i] = ff_add(v[i], u);
+      }
+      n += __shfl_xor_sync(0xffffffffu, n, o);
+    }
+  };
+  warp_tree(acc, nclip_all);
+  if (lane == 0) {
+#pragma unroll
+    for (int i = 0; i < 3; ++i) sm.red[warp][i] = acc[i];
+    sm.redn[warp] = nclip_all;
   }
   __syncthreads();
   if (tid == 0) {
+    float2 t[3] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+    long long n = 0;
+    for (int k = 0; k < kLossThreads / 32; ++k) {
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      double t = 0.0;
-      for (int k = 0; k < kLossThreads / 32; ++k) t += sm.red[k][i];
-      lp.partial[4 * blockIdx.x + i] = t;
+      for (int i = 0; i < 3; ++i) t[i] = ff_add(t[i], sm.red[k][i]);
+      n += sm.redn[k];
     }
+#pragma unroll
+    for (int i = 0; i < 3; ++i) part[4 * blockIdx.x + i] = t[i];
+    part_n[4 * blockIdx.x + 3] = n;
     __threadfence();
     sm.last = atomicAdd(&lp.status[kLossWordTicket], 1u) == gridDim.x - 1;
   }
   __syncthreads();
   if (!sm.last) return;
   // the last CTA: every thread loads the partials of CTAs tid, tid + 256, ... (all loads in
-  // flight together), then the same fixed tree as above
+  // flight together), then the same fixed trees as above
   __threadfence();
   constexpr int kMaxPer = kLossMaxBlocks / kLossThreads;
-  double pt[kMaxPer][4];
+  float2 pt[kMaxPer][3];
+  long long pn[kMaxPer];
 #pragma unroll
   for (int m = 0; m < kMaxPer; ++m) {
     const int blk = tid + m * kLossThreads;
+    const bool have = blk < (int)gridDim.x;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) pt[m][i] = blk < (int)gridDim.x ? __ldcg(&lp.partial[4 * blk + i]) : 0.0;
+    for (int i = 0; i < 3; ++i) pt[m][i] = have ? __ldcg(&part[4 * blk + i]) : make_float2(0.f, 0.f);
+    pn[m] = have ? __ldcg(&part_n[4 * blk + 3]) : 0ll;
   }
-  double t[4];
+  float2 t[3] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+  long long n = 0;
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    t[i] = 0.0;
+  for (int m = 0; m < kMaxPer; ++m) {
 #pragma unroll
-    for (int m = 0; m < kMaxPer; ++m) t[i] += pt[m][i];
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) t[i] += __shfl_xor_sync(0xffffffffu, t[i], o);
+    for (int i = 0; i < 3; ++i) t[i] = ff_add(t[i], pt[m][i]);
+    n += pn[m];
   }
+  warp_tree(t, n);
   __syncthreads();  // every thread has read sm.red above
-  if (lane == 0)
+  if (lane == 0) {
 #pragma unroll
-    for (int i = 0; i < 4; ++i) sm.red[warp][i] = t[i];
+    for (int i = 0; i < 3; ++i) sm.red[warp][i] = t[i];
+    sm.redn[warp] = n;
+  }
   __syncthreads();
   if (tid == 0) {
+    float2 u[3] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+    long long nn = 0;
+    for (int k = 0; k < kLossThreads / 32; ++k) {
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      t[i] = 0.0;
-      for (int k = 0; k < kLossThreads / 32; ++k) t[i] += sm.red[k][i];
+      for (int i = 0; i < 3; ++i) u[i] = ff_add(u[i], sm.red[k][i]);
+      nn += sm.redn[k];
     }
-    {
-      const double kl_term = kKL ? t[1] : 0.0;
-      *a.loss = (float)(-(t[0] - (double)a.beta * kl_term));
-      if (a.stats) {
-        a.stats[0] = t[0];
-        a.stats[1] = kl_term;
-        a.stats[2] = t[2];
-        a.stats[3] = a.T > 0 ? t[3] / (double)a.T : 0.0;
-      }
-      lp.status[kLossWordTicket] = 0u;  // ready for the next call on this plan
+    const double pg = (double)u[0].x + (double)u[0].y;
+    const double kl_term = kKL ? (double)u[1].x + (double)u[1].y : 0.0;
+    const double rsum = (double)u[2].x + (double)u[2].y;
+    *a.loss = (float)(-(pg - (double)a.beta * kl_term));
+    if (a.stats) {
+      a.stats[0] = pg;
+      a.stats[1] = kl_term;
+      a.stats[2] = (double)nn;
+      a.stats[3] = a.T > 0 ? rsum / (double)a.T : 0.0;
     }
+    lp.status[kLossWordTicket] = 0u;  // ready for the next call on this plan
   }
 }
 
