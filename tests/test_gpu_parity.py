@@ -321,40 +321,23 @@ def test_error_workspace_too_small(gp_mod):
 # --------------------------------------------------------------------- full-size configs
 
 
-def _sampled_groups(G, rng, k=5):
-    pick = {0, G - 1}
-    pick.update(rng.choice(G, size=min(k, G), replace=False).tolist())
-    return sorted(pick)
-
-
-@pytest.mark.parametrize("name", ["math", "agentic", "full"])
+@pytest.mark.parametrize("name", ["math", "agentic", "full", "wide"])
 def test_full_size_whole_batch(gp_mod, name):
     """Whole config on the GPU in the benchmark's launch configuration, every output of
-    every group against the oracle (16 host threads)."""
+    every group against the oracle (16 host threads; the wide groups' dense fp64
+    similarities take the oracle about 3 s per group and thread)."""
     b = batch_of(name)
     params = oracle_params(b)
     compare(run_gpu(gp_mod, b, params), oracle_run(b, params, threads=16), f"{name} whole batch")
 
 
-@pytest.mark.parametrize("name", ["wide"])
-def test_full_size_sampled(gp_mod, name):
-    """Whole config on the GPU in the benchmark's launch configuration; sampled groups
-    are recomputed by the oracle one by one (groups are independent; the dense fp64
-    similarity of all 64 groups would take the oracle minutes)."""
+@pytest.mark.parametrize("name", ["wide", "full"])
+def test_full_size_properties(gp_mod, name):
+    """Properties that hold at any size, on the whole config in the benchmark's launch
+    configuration."""
     b = batch_of(name)
     params = oracle_params(b)
     gpu = run_gpu(gp_mod, b, params, components=False)
-    G = len(b["group_rollout_off"]) - 1
-    rng = np.random.default_rng(1234)
-    groups = _sampled_groups(G, rng, k=2 if name == "wide" else 6)
-    sub = W.sub_batch(b, groups)
-    ref = oracle_run(sub, params)
-    st = sub["source_states"]
-    tok = W.token_index(b, sub)
-    np.testing.assert_array_equal(gpu["class_id"][st], st[ref["class_id"]], err_msg=f"{name} class_id")
-    assert_close(gpu["node_score"][st], ref["node_score"], f"{name} node_score")
-    assert_close(gpu["edge_adv"][st], ref["edge_adv"], f"{name} edge_adv")
-    assert_close(gpu["adv"][tok], ref["adv"], f"{name} adv")
     # properties that hold everywhere: every token of an edge carries the edge's value
     np.testing.assert_array_equal(gpu["adv"], np.repeat(gpu["edge_adv"], b["step_len"]))
     assert np.all(np.isfinite(gpu["adv"]))
