@@ -222,7 +222,12 @@ __device__ __forceinline__ void group_row_stats(const gpo_batch& b, const Sizes&
     const bool from_left = pl >= 0 && pl == i - 1 && r > 0;
     const uint4* zb = Z + (int64_t)(s0 + (live ? i : 0)) * rs;
     const uint4* pb = pl >= 0 ? Z + (int64_t)(s0 + pl) * rs : (pl == -2 ? RZ + (int64_t)g * rs : nullptr);
-    uint64_t ns = 0ull, ne = 0ull, ds = 0ull, de = 0ull;
+    // error-free sums of the exact bf16 products (BiasedSum: a plain fp32 bound of each
+    // segment's |products|, then Fast2Sum against a power-of-two bias, four operations per
+    // product); a segment is one stage of kU chunks per lane
+    BiasedSum sn, sd;
+    bs_init(sn);
+    bs_init(sd);
     // two stages of kU chunks per lane, software-pipelined: the next stage's loads are in
     // flight while this one's sums run (no register copies between the stages)
     constexpr int kU = 2;
@@ -236,6 +241,7 @@ __device__ __forceinline__ void group_row_stats(const gpo_batch& b, const Sizes&
       }
     };
     auto accumulate = [&](uint4 (&x)[kU], uint4 (&y)[kU]) {
+      uint64_t xx[4 * kU], yy[4 * kU];
 #pragma unroll
       for (int u = 0; u < kU; ++u) {
         uint4 t;
@@ -247,10 +253,23 @@ __device__ __forceinline__ void group_row_stats(const gpo_batch& b, const Sizes&
         const uint32_t xw[4] = {x[u].x, x[u].y, x[u].z, x[u].w}, yw[4] = {y[u].x, y[u].y, y[u].z, y[u].w};
 #pragma unroll
         for (int h = 0; h < 4; ++h) {
-          const uint64_t xx = bf16x2_f32x2(xw[h]), yy = bf16x2_f32x2(yw[h]);
-          f2_acc(ns, ne, f2mul(xx, xx));  // bf16 products are exact in fp32
-          f2_acc(ds, de, f2mul(xx, yy));
+          xx[4 * u + h] = bf16x2_f32x2(xw[h]);
+          yy[4 * u + h] = bf16x2_f32x2(yw[h]);
         }
+      }
+      uint64_t px = 0ull, py = 0ull;  // the segment's sums of squares (bounds only)
+#pragma unroll
+      for (int i = 0; i < 4 * kU; ++i) {
+        px = f2fma(xx[i], xx[i], px);
+        py = f2fma(yy[i], yy[i], py);
+      }
+      const float qx = f2_lanes_sum(px), qy = f2_lanes_sum(py);
+      bs_reserve(sn, qx);
+      bs_reserve(sd, 0.5f * (qx + qy));  // |x y| <= (x^2 + y^2) / 2
+#pragma unroll
+      for (int i = 0; i < 4 * kU; ++i) {
+        bs_add(sn, xx[i], xx[i]);  // bf16 products are exact in fp32
+        bs_add(sd, xx[i], yy[i]);
       }
     };
     uint4 xa[kU], ya[kU], xb[kU], yb[kU];
@@ -264,13 +283,24 @@ __device__ __forceinline__ void group_row_stats(const gpo_batch& b, const Sizes&
     if (sz.d % 8 != 0 && c == 0 && live) {  // the ragged end of the row, one lane per row
       const uint16_t* zr = reinterpret_cast<const uint16_t*>(zb);
       const uint16_t* pr = reinterpret_cast<const uint16_t*>(pb);
+      float qx = 0.f, qy = 0.f;
       for (int k = 8 * nch; k < sz.d; ++k) {
-        const uint64_t xx = (uint64_t)((uint32_t)zr[k] << 16);
-        const uint64_t yy = pr ? (uint64_t)((uint32_t)pr[k] << 16) : 0ull;
-        f2_acc(ns, ne, f2mul(xx, xx));  // one fp32 lane (the other stays 0)
-        f2_acc(ds, de, f2mul(xx, yy));
+        const float x = __uint_as_float((uint32_t)zr[k] << 16), y = pr ? __uint_as_float((uint32_t)pr[k] << 16) : 0.f;
+        qx = fmaf(x, x, qx);
+        qy = fmaf(y, y, qy);
+      }
+      bs_reserve(sn, qx);
+      bs_reserve(sd, 0.5f * (qx + qy));
+      for (int k = 8 * nch; k < sz.d; ++k) {
+        const uint64_t xx = pack_f2((uint32_t)zr[k] << 16, 0u);  // one fp32 lane (the other stays 0)
+        const uint64_t yy = pack_f2(pr ? (uint32_t)pr[k] << 16 : 0u, 0u);
+        bs_add(sn, xx, xx);
+        bs_add(sd, xx, yy);
       }
     }
+    uint64_t ns, ne, ds, de;
+    bs_finish(sn, ns, ne);
+    bs_finish(sd, ds, de);
     const float2 n2 = finish4(ns, ne);
     float2 dot = finish4(ds, de);
     if (pl == -1) dot = make_float2(0.f, 0.f);

@@ -409,9 +409,17 @@ __device__ __forceinline__ uint64_t f2mul(uint64_t a, uint64_t b) {
   return d;
 }
 // The two bf16 of a 32-bit word as fp32 lanes (low half first).
-__device__ __forceinline__ uint64_t bf16x2_f32x2(uint32_t w) {
-  return ((uint64_t)(w & 0xFFFF0000u) << 32) | (uint64_t)(w << 16);
+// Packing and unpacking go through mov.b64 {lo, hi}, a register pair, rather than 64-bit
+// shifts and ors.
+__device__ __forceinline__ uint64_t pack_f2(uint32_t lo, uint32_t hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "r"(lo), "r"(hi));
+  return r;
 }
+__device__ __forceinline__ void unpack_f2(uint64_t a, uint32_t& lo, uint32_t& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=r"(lo), "=r"(hi) : "l"(a));
+}
+__device__ __forceinline__ uint64_t bf16x2_f32x2(uint32_t w) { return pack_f2(w << 16, w & 0xFFFF0000u); }
 // Compensated accumulation (TwoSum per lane) of x into (s, e).
 __device__ __forceinline__ void f2_acc(uint64_t& s, uint64_t& e, uint64_t x) {
   const uint64_t t = f2add(s, x);
@@ -428,6 +436,80 @@ __device__ __forceinline__ float2 f2_finish(uint64_t s, uint64_t e) {
   float hh, ll;
   two_sum(h, t + e0 + e1, hh, ll);
   return make_float2(hh, ll);
+}
+
+// ------------------------------------------------------------------ biased error-free sums
+// Sums of exact products (bf16 x bf16 is exact in fp32) with four fp32 operations per
+// product instead of TwoSum's seven, at the same accuracy.  The running sum carries a bias
+// sigma, a power of two >= 2 B where B bounds the sum of |products| added so far: then the
+// running sum s stays in [sigma/2, 3 sigma/2], every product p has |p| <= sigma/2 <= |s|,
+// so t = fl(s + p) is Dekker's Fast2Sum case (Dekker 1971; Muller et al., Handbook of
+// Floating-Point Arithmetic, Sec. 4.3): s - t and p + (s - t) are exact, and
+//   t = fma(x, y, s),  z = s - t,  err = fma(x, y, z) = p - (t - s)
+// gives the rounding error of every addition exactly (collected, rounded, in e).  s - sigma
+// is exact (Sterbenz), so the sum is (s - sigma) + e.  B comes from a plain fp32 pass over
+// the next segment of the operands (sum of x^2, and (x^2 + y^2) / 2 >= |x y| for a dot),
+// with a relative margin that covers that pass's rounding; when 2 B would pass sigma, the
+// current epoch is closed into a float pair by TwoSum and a new one starts with
+// sigma = 2^ceil(log2 4 B).  Two fp32 lanes per instruction, as in f2_acc.
+
+__device__ __forceinline__ uint64_t f2fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2splat(float x) { return pack_f2(__float_as_uint(x), __float_as_uint(x)); }
+// The sum of a pair's two fp32 lanes (rounded once).
+__device__ __forceinline__ float f2_lanes_sum(uint64_t a) {
+  uint32_t lo, hi;
+  unpack_f2(a, lo, hi);
+  return __uint_as_float(lo) + __uint_as_float(hi);
+}
+// Smallest power of two >= x, for finite x >= 0 (0 for 0; +inf beyond the fp32 range).
+__device__ __forceinline__ float pow2_ceil(float x) {
+  return __uint_as_float((__float_as_uint(x) + 0x007FFFFFu) & 0xFF800000u);
+}
+
+struct BiasedSum {
+  uint64_t s, e;  // biased running sums and their rounding errors (two lanes)
+  uint64_t h, l;  // float pairs (two lanes) of the epochs closed so far
+  float sigma;    // bias of the current epoch (both lanes)
+  float bound;    // bound of the sum of |products| added so far (plus the reserved segment)
+};
+
+__device__ __forceinline__ void bs_init(BiasedSum& a) {
+  a.s = a.e = a.h = a.l = 0ull;
+  a.sigma = 0.f;
+  a.bound = 0.f;
+}
+// Closes the current epoch: (s - sigma) + e joins the pair (h, l).
+__device__ __forceinline__ void bs_close(BiasedSum& a) {
+  f2_acc(a.h, a.l, f2sub(a.s, f2splat(a.sigma)));  // s - sigma is exact in each lane
+  a.l = f2add(a.l, a.e);
+}
+// Reserves room for a segment whose sum of |products| is at most `add` (a plain fp32
+// estimate; the relative margin 2^-12 covers its rounding and that of the bound itself).
+__device__ __forceinline__ void bs_reserve(BiasedSum& a, float add) {
+  a.bound = fmaf(add, 1.000244140625f, a.bound);
+  if (2.f * a.bound > a.sigma) {
+    bs_close(a);
+    a.sigma = pow2_ceil(4.f * a.bound);
+    a.s = f2splat(a.sigma);
+    a.e = 0ull;
+  }
+}
+// Adds the exact products x y (two lanes).
+__device__ __forceinline__ void bs_add(BiasedSum& a, uint64_t x, uint64_t y) {
+  const uint64_t t = f2fma(x, y, a.s);
+  const uint64_t z = f2sub(a.s, t);
+  a.e = f2add(a.e, f2fma(x, y, z));
+  a.s = t;
+}
+// The two lanes' pairs of the finished sum, to be combined by f2_finish.
+__device__ __forceinline__ void bs_finish(BiasedSum& a, uint64_t& s, uint64_t& e) {
+  bs_close(a);
+  s = a.h;
+  e = a.l;
 }
 
 // One warp: |z|^2 of the row at element offset zrow of `base` and, if has_p, its dot with
