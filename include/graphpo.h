@@ -113,6 +113,14 @@ typedef struct {
  * group-resident kernel (bf16 embeddings, max_states_per_group <= 384);
  * for comparisons and tests. */
 #define GPO_FLAG_TILED 2
+/* For tests of the failure path only: in every CTA of the tensor-core kernels the MMA warp's
+ * first wait runs out (it waits about a millisecond on an mbarrier that nothing arrives on),
+ * as a stalled copy or MMA would make it; the kernel then reports GPO_ERR_TIMEOUT and winds
+ * down as it does after any timed-out wait (copies in flight land, issued MMAs complete,
+ * TMEM is released).  gpo_sync_status returns GPO_ERR_TIMEOUT; outputs are undefined; the
+ * CUDA context stays usable.  Paths without tensor-core kernels (fp32 embeddings,
+ * GPO_FLAG_SIMT_SIMILARITY) ignore the flag. */
+#define GPO_FLAG_DEBUG_TIMEOUT 4
 
 typedef struct {
   int32_t num_groups;     /* G >= 0 */

@@ -23,6 +23,7 @@ STATUS_NAMES = {0: "ok", 1: "invalid argument", 2: "shape", 3: "bad reward", 4: 
 MERGE_RULES = {"noncausal": 0, "same_depth": 1}
 FLAG_SIMT_SIMILARITY = 1
 FLAG_TILED = 2
+FLAG_DEBUG_TIMEOUT = 4  # tests of the failure path: the tensor-core kernels' first wait runs out
 EMB_BF16, EMB_F32 = 0, 1
 
 

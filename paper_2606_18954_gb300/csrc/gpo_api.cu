@@ -145,7 +145,7 @@ Ws workspace_views(void* base, const Layout& L) {
 gpo_status check_params(const gpo_params& p) {
   if (!std::isfinite(p.kappa) || !(p.kappa > 0.0) || !(p.w >= 0.0 && p.w <= 1.0) || !(p.lambda_eff >= 0.0) ||
       !std::isfinite(p.lambda_eff) || !(p.std_eps >= 0.0) || !std::isfinite(p.std_eps) || p.std_ddof < 0 ||
-      p.std_ddof > 1 || p.merge_rule < 0 || p.merge_rule > 1 || (p.flags & ~(GPO_FLAG_SIMT_SIMILARITY | GPO_FLAG_TILED)))
+      p.std_ddof > 1 || p.merge_rule < 0 || p.merge_rule > 1 || (p.flags & ~(GPO_FLAG_SIMT_SIMILARITY | GPO_FLAG_TILED | GPO_FLAG_DEBUG_TIMEOUT)))
     return GPO_ERR_INVALID_ARG;
   return GPO_OK;
 }
@@ -340,7 +340,7 @@ gpo_status compute_impl(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs*
   pp.active = bud ? bud->active : nullptr;
   pp.budget = bud ? bud->budget : nullptr;
   pp.stats_in_kernel = 0;
-  pp.pad_ = 0;
+  pp.debug_timeout = (p.flags & GPO_FLAG_DEBUG_TIMEOUT) != 0;
   const Ws ws = workspace_views(workspace, L);
   LaunchCtx lc;
   lc.stream = static_cast<cudaStream_t>(stream);

@@ -539,6 +539,12 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
     uint32_t seq = 0;  // slices consumed (the producer's sequence)
     int u = 0;         // accumulator uses (passes) so far
     bool ok = true;
+    // GPO_FLAG_DEBUG_TIMEOUT: the first wait runs out (nothing arrives on `drain` before the
+    // commit below), and the CTA winds down as after any timeout
+    if (p.debug_timeout) {
+      mbar_wait(&ctl->drain, 0, st, 27, kDebugTimeoutNs);  // returns false: reports GPO_ERR_TIMEOUT
+      ok = false;
+    }
     for (int g = sz.g0 + (int)blockIdx.x; g < sz.g1 && ok; g += gridDim.x) {
       int r0, nr, s0, n;
       if (!group_active(b, sz, g, r0, nr, s0, n)) continue;

@@ -90,7 +90,7 @@ struct Params {
   int mode, layer, b_next;
   int stats_in_kernel;    // fused path: the group warps compute the compensated row statistics
                           // of each CTA's first group (the other groups' come from exact_stats)
-  int pad_;
+  int debug_timeout;      // GPO_FLAG_DEBUG_TIMEOUT: the MMA warp's first wait runs out
   const uint8_t* active;  // [N] frontier states to expand (NULL: all of depth `layer`)
   int32_t* budget;        // [N] output of mode 1
 };
@@ -171,6 +171,11 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32
     }
   }
 }
+
+// GPO_FLAG_DEBUG_TIMEOUT: a wait that runs out on purpose, on an mbarrier that has no arrival
+// before the caller's own later commit (about a millisecond, then GPO_ERR_TIMEOUT as any
+// timed-out wait reports it).
+constexpr uint64_t kDebugTimeoutNs = 1000000ull;
 
 // ------------------------------------------------------------------ flags between CTAs
 

@@ -108,7 +108,7 @@ __device__ __forceinline__ void lunion(int* p, int a, int b) {
 
 __global__ void __launch_bounds__(kThreads, 1)
     sim_tc_kernel(const __grid_constant__ CUtensorMap zmap, const int32_t* __restrict__ rollout_step_off, Sizes sz,
-                  Ws ws, float kappa, int rule) {
+                  Ws ws, float kappa, int rule, int debug_timeout) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   // control block first, then the tiles on a 1024-byte boundary (128B swizzle); both are
   // smem_raw plus an offset, so the compiler keeps the shared address space
@@ -194,6 +194,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t phase = 0;
     int m = 0;
     bool ok = true;
+    // GPO_FLAG_DEBUG_TIMEOUT: the first wait runs out (nothing arrives on `drain` before the
+    // commit below), and the CTA winds down as after any timeout
+    if (debug_timeout) {
+      mbar_wait(&ctl->drain, 0, st, 17, kDebugTimeoutNs);  // returns false: reports GPO_ERR_TIMEOUT
+      ok = false;
+    }
     for (int it = blockIdx.x; it < nitems && ok; it += gridDim.x, ++m) {
       const Item item = ws.items[it];
       const bool diag = item.col0 == item.row0;
@@ -446,7 +452,7 @@ cudaError_t launch_sim_tc(const LaunchCtx& lc, const CUtensorMap& map, const gpo
   int grid = ws.max_items < lc.num_sms ? ws.max_items : lc.num_sms;
   if (grid < 1) return cudaSuccess;
   sim_tc_kernel<<<grid, kThreads, sim_tc_smem_bytes(), lc.stream>>>(map, b.rollout_step_off, sz, ws, (float)p.kappa,
-                                                                      p.rule);
+                                                                      p.rule, p.debug_timeout);
   return cudaGetLastError();
 }
 
