@@ -134,3 +134,17 @@ def test_compute_host_matches_oracle(P, chunk_bytes):
     want = o["adv"].astype(np.float32)
     got = out.numpy()
     assert np.all(np.abs(got - want) <= 1e-5 * np.abs(want) + 1e-6)
+
+
+def test_compute_host_tree_layout_pipelined(P):
+    """compute_host over chunks of a tree-layout batch (token spans per group) against the
+    device-resident call."""
+    import torch
+    b = W.make_tree_batch(W.TREE_CONFIGS["tree"].scaled(groups=8))
+    gp = _gp(P, b)
+    hb = P.Batch.from_arrays(b, device="cpu", pin=True)
+    out = gp.compute_host(hb, chunk_bytes=1 << 19)  # 3.4 MB of embeddings: six chunks
+    again = gp.compute_host(hb, chunk_bytes=1 << 19)  # staging buffers reused
+    ref = gp(P.Batch.from_arrays(b, device="cuda"))
+    gp.check()
+    assert torch.equal(out, ref["adv"].cpu()) and torch.equal(again, out)
