@@ -404,12 +404,13 @@ gpo_status compute_impl(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs*
     if (e == cudaSuccess && b.parent) e = stage("tree_prep", launch_tree_prep(lc, b, sz, ws));
     if (e == cudaSuccess) e = stage("prep", launch_prep(lc, b, sz, ws));
     if (e == cudaSuccess && sz.N > 0) {
-      // eta takes compensated norms and parent dots (exact_stats); the fp32 norms of the
-      // threshold test come from the Gram tiles (tcgen05) or from row_stats (CUDA cores)
-      if (!bud) e = stage("exact_stats", launch_exact_stats(lc, b, sz, ws));
+      // the fp32 norms of the threshold test come from the Gram tiles (tcgen05) or from
+      // row_stats (CUDA cores); eta takes compensated norms and parent dots (exact_stats),
+      // after the similarity stage so that the fp32 norms give the sums' biases
       if (e == cudaSuccess && !use_tc) e = stage("row_stats", launch_row_stats(lc, b, sz, ws));
       if (e == cudaSuccess)
         e = stage("similarity", use_tc ? launch_sim_tc(lc, map, b, sz, ws, pp) : launch_sim_simt(lc, b, sz, ws, pp));
+      if (e == cudaSuccess && !bud) e = stage("exact_stats", launch_exact_stats(lc, b, sz, ws, true));
       if (e == cudaSuccess) e = stage("groups", launch_groups(lc, b, *out, sz, ws, pp));
       if (e == cudaSuccess && !bud) e = stage("tokens", launch_tokens(lc, b, *out, sz, ws));
     }

@@ -503,6 +503,13 @@ __device__ __forceinline__ void bs_reserve(BiasedSum& a, float add) {
     a.e = 0ull;
   }
 }
+// One Fast2Sum step of a biased running sum s (error collected in e): the exact products
+// x y (two lanes), |x y| <= |s| with s - t exact (the caller's bias guarantees both).
+__device__ __forceinline__ void biased_add(uint64_t& s, uint64_t& e, uint64_t x, uint64_t y) {
+  const uint64_t t = f2fma(x, y, s);
+  e = f2add(e, f2fma(x, y, f2sub(s, t)));
+  s = t;
+}
 // Adds the exact products x y (two lanes).
 __device__ __forceinline__ void bs_add(BiasedSum& a, uint64_t x, uint64_t y) {
   const uint64_t t = f2fma(x, y, a.s);
@@ -630,7 +637,9 @@ struct LaunchCtx {
 };
 
 cudaError_t launch_prep(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws);
-cudaError_t launch_exact_stats(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws);
+// with_norms: ws.nrm2 holds every row's fp32 squared norm (the similarity stage ran first)
+cudaError_t launch_exact_stats(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws,
+                               bool with_norms = false);
 cudaError_t launch_tree_prep(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws);
 cudaError_t setup_tree_prep();
 cudaError_t launch_row_stats(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws);

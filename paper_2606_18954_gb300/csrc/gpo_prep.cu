@@ -532,8 +532,18 @@ __global__ void __launch_bounds__(256) exact_stats_kernel(gpo_batch b, Sizes sz,
 // 4 r + j summing quarter j of row base + r in 16-byte chunks, four chunks in flight.  In the
 // chain layout the parent of a row is the row before, whose chunk the lane 4 below already
 // holds (a shuffle); the first row's parent chunk, a tree parent or a prompt embedding is
-// loaded.  Compensated sums per lane, two fp32 lanes per instruction (f2_acc), then a fixed
-// butterfly over the 4 quarters: the accuracy of exact_stats_kernel with every row read once.
+// loaded.  Compensated sums per lane, two fp32 lanes per instruction, then a fixed butterfly
+// over the 4 quarters: the accuracy of exact_stats_kernel with every row read once.
+//   kNorms = false: TwoSum per product (f2_acc).
+//   kNorms = true (after the similarity stage, which leaves fp32 squared norms in ws.nrm2,
+//   accurate to far better than 1 %): biased error-free sums with one bias per row and sum,
+//   sigma = 2^ceil(log2 (4.04 |z_v|^2)) for |z_v|^2 and 2^ceil(log2 (2.02 (|z_v|^2 + |z_p|^2)))
+//   for <z_p, z_v> (|x y| <= (x^2 + y^2) / 2), so that each running sum stays in
+//   [sigma/2, 3 sigma/2] and every product is Fast2Sum's case (see BiasedSum): four fp32
+//   operations per product, two independent chains per sum, no bound pass.  A lane whose sum
+//   ends outside the range (a norm that was not what the similarity stage reported) sends its
+//   row through the TwoSum path instead.
+template <bool kNorms>
 __global__ void __launch_bounds__(256) exact_stats_lane_kernel(gpo_batch b, Sizes sz, Ws ws) {
   const int lane = threadIdx.x & 31, r = lane >> 2, j = lane & 3;
   const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -556,8 +566,7 @@ __global__ void __launch_bounds__(256) exact_stats_lane_kernel(gpo_batch b, Size
     v0 = max(0, min(v0, sz.N));
     v1 = max(v0, min(v1, sz.N));
   }
-  auto finish4 = [&](uint64_t s, uint64_t e) -> float2 {  // the 4 quarters' pairs, fixed order
-    float2 P = f2_finish(s, e);
+  auto quad = [&](float2 P) -> float2 {  // the 4 quarters' pairs, fixed order
 #pragma unroll
     for (int o = 1; o < 4; o <<= 1) {
       const float a = __shfl_xor_sync(0xffffffffu, P.x, o), c = __shfl_xor_sync(0xffffffffu, P.y, o);
@@ -569,6 +578,24 @@ __global__ void __launch_bounds__(256) exact_stats_lane_kernel(gpo_batch b, Size
     float h, l;
     two_sum(P.x, P.y, h, l);
     return make_float2(h, l);
+  };
+  auto finish4 = [&](uint64_t s, uint64_t e) -> float2 { return quad(f2_finish(s, e)); };
+  // TwoSum sums of this lane's quarter of row zb and its parent pb (chunks loaded here)
+  auto twosum_quarter = [&](const uint4* zb, const uint4* pb, bool on, float2& n2, float2& dot) {
+    uint64_t ns = 0ull, ne = 0ull, ds = 0ull, de = 0ull;
+    for (int c = 0; on && c < nq; ++c) {
+      const int k = j * nq + c;
+      const uint4 x = zb[k], y = pb ? pb[k] : make_uint4(0u, 0u, 0u, 0u);
+      const uint32_t xw[4] = {x.x, x.y, x.z, x.w}, yw[4] = {y.x, y.y, y.z, y.w};
+#pragma unroll
+      for (int h = 0; h < 4; ++h) {
+        const uint64_t xx = bf16x2_f32x2(xw[h]), yy = bf16x2_f32x2(yw[h]);
+        f2_acc(ns, ne, f2mul(xx, xx));
+        f2_acc(ds, de, f2mul(xx, yy));
+      }
+    }
+    n2 = finish4(ns, ne);
+    dot = finish4(ds, de);
   };
   for (int64_t base = v0 + warp * 8; base < v1; base += nwarps * 8) {
     const int64_t v = base + r;
@@ -612,35 +639,107 @@ __global__ void __launch_bounds__(256) exact_stats_lane_kernel(gpo_batch b, Size
     const bool from_left = p >= 0 && p == v - 1 && r > 0;
     const uint4* pb = p >= 0 ? Z + (int64_t)p * rs : (p <= -2 ? RZ + (int64_t)(-2 - p) * rs : nullptr);
     const uint4* zb = Z + (live ? v : base) * rs;
-    uint64_t ns = 0ull, ne = 0ull, ds = 0ull, de = 0ull;
-    constexpr int kU = 4;  // chunks loaded ahead of their arithmetic (memory-level parallelism)
-    for (int c0 = 0; c0 < nq; c0 += kU) {
-      uint4 x[kU], y[kU];
+    float2 n2, dot;
+    if (!kNorms) {
+      uint64_t ns = 0ull, ne = 0ull, ds = 0ull, de = 0ull;
+      constexpr int kU = 4;  // chunks loaded ahead of their arithmetic (memory-level parallelism)
+      for (int c0 = 0; c0 < nq; c0 += kU) {
+        uint4 x[kU], y[kU];
 #pragma unroll
-      for (int u = 0; u < kU; ++u) {
-        const int k = j * nq + c0 + u;
-        x[u] = live && c0 + u < nq ? zb[k] : make_uint4(0u, 0u, 0u, 0u);
-        y[u] = (!from_left && pb && c0 + u < nq) ? pb[k] : make_uint4(0u, 0u, 0u, 0u);
+        for (int u = 0; u < kU; ++u) {
+          const int k = j * nq + c0 + u;
+          x[u] = live && c0 + u < nq ? zb[k] : make_uint4(0u, 0u, 0u, 0u);
+          y[u] = (!from_left && pb && c0 + u < nq) ? pb[k] : make_uint4(0u, 0u, 0u, 0u);
+        }
+#pragma unroll
+        for (int u = 0; u < kU; ++u) {
+          uint4 t;
+          t.x = __shfl_up_sync(0xffffffffu, x[u].x, 4);
+          t.y = __shfl_up_sync(0xffffffffu, x[u].y, 4);
+          t.z = __shfl_up_sync(0xffffffffu, x[u].z, 4);
+          t.w = __shfl_up_sync(0xffffffffu, x[u].w, 4);
+          if (from_left) y[u] = t;
+          const uint32_t xw[4] = {x[u].x, x[u].y, x[u].z, x[u].w}, yw[4] = {y[u].x, y[u].y, y[u].z, y[u].w};
+#pragma unroll
+          for (int h = 0; h < 4; ++h) {
+            const uint64_t xx = bf16x2_f32x2(xw[h]), yy = bf16x2_f32x2(yw[h]);
+            f2_acc(ns, ne, f2mul(xx, xx));  // bf16 products are exact in fp32
+            f2_acc(ds, de, f2mul(xx, yy));
+          }
+        }
       }
+      n2 = finish4(ns, ne);
+      dot = finish4(ds, de);
+    } else {
+      // the biases: fp32 squared norms of the row and its parent (ws.nrm2; the prompt
+      // embedding's from root_norms_kernel, which ran first)
+      float nv = 0.f, np = 0.f;
+      if (live) {
+        nv = ws.nrm2[v];
+        if (p >= 0) np = ws.nrm2[p];
+        else if (p <= -2) np = ws.x_root_n2[-2 - p].x;
+      }
+      const float sgn = pow2_ceil(4.04f * nv), sgd = pow2_ceil(2.02f * (nv + np));
+      const uint64_t sn0 = f2splat(sgn), sd0 = f2splat(sgd);
+      uint64_t a0 = sn0, a1 = sn0, b0 = sd0, b1 = sd0, ea0 = 0ull, ea1 = 0ull, eb0 = 0ull, eb1 = 0ull;
+      constexpr int kU = 4;
+      for (int c0 = 0; c0 < nq; c0 += kU) {
+        uint4 x[kU], y[kU];
 #pragma unroll
-      for (int u = 0; u < kU; ++u) {
-        uint4 t;
-        t.x = __shfl_up_sync(0xffffffffu, x[u].x, 4);
-        t.y = __shfl_up_sync(0xffffffffu, x[u].y, 4);
-        t.z = __shfl_up_sync(0xffffffffu, x[u].z, 4);
-        t.w = __shfl_up_sync(0xffffffffu, x[u].w, 4);
-        if (from_left) y[u] = t;
-        const uint32_t xw[4] = {x[u].x, x[u].y, x[u].z, x[u].w}, yw[4] = {y[u].x, y[u].y, y[u].z, y[u].w};
+        for (int u = 0; u < kU; ++u) {
+          const int k = j * nq + c0 + u;
+          x[u] = live && c0 + u < nq ? zb[k] : make_uint4(0u, 0u, 0u, 0u);
+          y[u] = (!from_left && pb && c0 + u < nq) ? pb[k] : make_uint4(0u, 0u, 0u, 0u);
+        }
 #pragma unroll
-        for (int h = 0; h < 4; ++h) {
-          const uint64_t xx = bf16x2_f32x2(xw[h]), yy = bf16x2_f32x2(yw[h]);
-          f2_acc(ns, ne, f2mul(xx, xx));  // bf16 products are exact in fp32
-          f2_acc(ds, de, f2mul(xx, yy));
+        for (int u = 0; u < kU; ++u) {
+          uint4 t;
+          t.x = __shfl_up_sync(0xffffffffu, x[u].x, 4);
+          t.y = __shfl_up_sync(0xffffffffu, x[u].y, 4);
+          t.z = __shfl_up_sync(0xffffffffu, x[u].z, 4);
+          t.w = __shfl_up_sync(0xffffffffu, x[u].w, 4);
+          if (from_left) y[u] = t;
+          const uint32_t xw[4] = {x[u].x, x[u].y, x[u].z, x[u].w}, yw[4] = {y[u].x, y[u].y, y[u].z, y[u].w};
+#pragma unroll
+          for (int h = 0; h < 4; h += 2) {
+            const uint64_t x0 = bf16x2_f32x2(xw[h]), y0 = bf16x2_f32x2(yw[h]);
+            const uint64_t x1 = bf16x2_f32x2(xw[h + 1]), y1 = bf16x2_f32x2(yw[h + 1]);
+            biased_add(a0, ea0, x0, x0);
+            biased_add(b0, eb0, x0, y0);
+            biased_add(a1, ea1, x1, x1);
+            biased_add(b1, eb1, x1, y1);
+          }
+        }
+      }
+      // every running sum still in [sigma/2, 3 sigma/2]: then each step was error-free
+      auto in_range = [](uint64_t s, float sg) {
+        uint32_t lo, hi;
+        unpack_f2(s, lo, hi);
+        return fabsf(__uint_as_float(lo) - sg) <= 0.5f * sg && fabsf(__uint_as_float(hi) - sg) <= 0.5f * sg;
+      };
+      int okv = !live || (in_range(a0, sgn) && in_range(a1, sgn) && in_range(b0, sgd) && in_range(b1, sgd));
+      // the row's 4 lanes agree (lanes 4 r .. 4 r + 3); every lane takes part in both shuffles
+      okv &= __shfl_xor_sync(0xffffffffu, okv, 1);
+      okv &= __shfl_xor_sync(0xffffffffu, okv, 2);
+      const bool ok = okv != 0;
+      // (s - sigma) is exact in each lane; the lane's pair: both chains' parts and errors
+      auto lane_pair = [](uint64_t s0, uint64_t e0, uint64_t s1, uint64_t e1, float sg) {
+        uint64_t h = 0ull, l = 0ull;
+        f2_acc(h, l, f2sub(s0, f2splat(sg)));
+        f2_acc(h, l, f2sub(s1, f2splat(sg)));
+        return f2_finish(h, f2add(l, f2add(e0, e1)));
+      };
+      n2 = quad(lane_pair(a0, ea0, a1, ea1, sgn));
+      dot = quad(lane_pair(b0, eb0, b1, eb1, sgd));
+      if (__any_sync(0xffffffffu, !ok)) {  // rare: the rows out of range, by TwoSum
+        float2 n2b, dotb;
+        twosum_quarter(zb, pb ? pb : nullptr, live && !ok, n2b, dotb);
+        if (!ok) {
+          n2 = n2b;
+          dot = dotb;
         }
       }
     }
-    const float2 n2 = finish4(ns, ne);
-    float2 dot = finish4(ds, de);
     if (p == -1) dot = make_float2(0.f, 0.f);
     if (live && j == 0) {
       if (!isfinite(n2.x) || !isfinite(dot.x)) report(ws.status, GPO_ERR_NONFINITE, 3, (int)v);
@@ -665,7 +764,8 @@ __global__ void __launch_bounds__(256) root_norms_kernel(gpo_batch b, Sizes sz, 
   }
 }
 
-cudaError_t launch_exact_stats(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws) {
+cudaError_t launch_exact_stats(const LaunchCtx& lc, const gpo_batch& b, const Sizes& sz, const Ws& ws,
+                               bool with_norms) {
   const int64_t jobs = (int64_t)sz.N + (b.root_emb ? sz.G : 0);  // at most (range calls take fewer)
   if (jobs == 0) return cudaSuccess;
   const bool aligned16 = (reinterpret_cast<uintptr_t>(b.emb) & 15u) == 0 && sz.stride % 8 == 0 && sz.d % 8 == 0 &&
@@ -674,12 +774,15 @@ cudaError_t launch_exact_stats(const LaunchCtx& lc, const gpo_batch& b, const Si
     int64_t blocks = ((int64_t)sz.N + 63) / 64;  // a warp per 8 rows
     const int64_t bcap = (int64_t)lc.num_sms * 32;
     blocks = blocks < 1 ? 1 : (blocks > bcap ? bcap : blocks);
-    exact_stats_lane_kernel<<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
-    if (b.root_emb && sz.g1 > sz.g0) {
+    if (b.root_emb && sz.g1 > sz.g0) {  // first: the norms-based path reads them
       int64_t rblocks = ((int64_t)(sz.g1 - sz.g0) + 7) / 8;
       if (rblocks > (int64_t)lc.num_sms * 8) rblocks = (int64_t)lc.num_sms * 8;
       root_norms_kernel<<<(int)rblocks, 256, 0, lc.stream>>>(b, sz, ws);
     }
+    if (with_norms)
+      exact_stats_lane_kernel<true><<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
+    else
+      exact_stats_lane_kernel<false><<<(int)blocks, 256, 0, lc.stream>>>(b, sz, ws);
     return cudaGetLastError();
   }
   int64_t blocks = (jobs + 7) / 8;  // a warp per row
