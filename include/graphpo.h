@@ -206,6 +206,37 @@ gpo_status gpo_compute_groups(gpo_ctx* ctx, const gpo_batch* batch, const gpo_ou
                               int64_t num_groups, int clear_status, void* workspace, size_t workspace_bytes,
                               void* stream);
 
+/* End-to-end variant for a batch held in HOST memory (the paper has no counterpart: it
+ * lets a caller whose rollouts and embeddings arrive in host memory overlap their upload
+ * with the work, and take the per-token advantages back into host memory).
+ *   host      the batch, every array in host memory: pinned (page-locked) memory for the
+ *             copies to be asynchronous and overlap; pageable memory works but each copy
+ *             then completes before the call goes on.  The host arrays must stay valid
+ *             and unchanged until `stream` reaches the end of this call's work.
+ *   dev       the same batch's device staging buffers: identical sizes, layout and row
+ *             stride, every array pointer a device buffer of the same size as its host
+ *             array, owned by the caller; the library copies the host arrays into them.
+ *   out       device outputs as for gpo_compute (adv required; optional outputs are
+ *             written on the device, not copied back).
+ *   host_adv  host array of total_tokens floats that receives out->adv.
+ *   chunk_bytes  about how many bytes of embeddings one pipeline stage uploads
+ *             (0: the larger of 8 MiB and a tenth of the embeddings; a value above the
+ *             embeddings' size: one stage).
+ * Enqueues, in order of `stream`: the small arrays' uploads, then the groups in chunks of
+ * about equal state counts -- chunk k's embeddings are uploaded while earlier chunks run,
+ * and each chunk's advantages are copied to host_adv once they are ready -- on helper
+ * streams of the context that rejoin `stream` at the end (so work enqueued later on
+ * `stream`, such as gpo_sync_status, follows all of it).  The chunks are the calls of
+ * gpo_compute_groups and need the group-resident path (bf16 embeddings,
+ * max_states_per_group <= 384, no flags) and host offsets that partition the batch;
+ * otherwise: one upload, gpo_compute and one download, all on `stream`.  The first
+ * pipelined call on a context creates its helper streams and events (released by
+ * gpo_destroy).  Checks and errors as for gpo_compute, plus GPO_ERR_INVALID_ARG when the
+ * two batches differ in size or layout or a host array is NULL. */
+gpo_status gpo_compute_host(gpo_ctx* ctx, const gpo_batch* host, const gpo_batch* dev, const gpo_outputs* out,
+                            float* host_adv, int64_t chunk_bytes, void* workspace, size_t workspace_bytes,
+                            void* stream);
+
 /* Waits for `stream` and returns the first error the kernels of the last
  * gpo_compute (or of the gpo_compute_groups calls since the last clearing one)
  * on this context reported (GPO_OK if none). */

@@ -82,7 +82,8 @@ LOSS_NSTATS = 4
 
 EXPORTS = ["gpo_create", "gpo_workspace_size", "gpo_compute", "gpo_sync_status", "gpo_status_string",
            "gpo_last_error", "gpo_version", "gpo_destroy", "gpo_enable_timing", "gpo_stage_times", "gpo_compute_noalloc",
-           "gpo_compute_groups", "gpo_loss_plan_size", "gpo_loss_plan", "gpo_token_loss", "gpo_layer_budget"]
+           "gpo_compute_groups", "gpo_compute_host", "gpo_loss_plan_size", "gpo_loss_plan", "gpo_token_loss",
+           "gpo_layer_budget"]
 
 FUSED_MAX_STATES = 384  # largest group the group-resident path (and gpo_compute_groups) serves
 
@@ -117,6 +118,10 @@ def load(build_if_missing: bool = False):
                                          ctypes.c_int64, ctypes.c_int64, ctypes.c_int, ctypes.c_void_p,
                                          ctypes.c_size_t, ctypes.c_void_p]
         L.gpo_compute_groups.restype = ctypes.c_int
+        L.gpo_compute_host.argtypes = [ctypes.c_void_p, ctypes.POINTER(CBatch), ctypes.POINTER(CBatch),
+                                       ctypes.POINTER(COutputs), ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p,
+                                       ctypes.c_size_t, ctypes.c_void_p]
+        L.gpo_compute_host.restype = ctypes.c_int
         L.gpo_sync_status.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
         L.gpo_sync_status.restype = ctypes.c_int
         L.gpo_status_string.argtypes = [ctypes.c_int]
@@ -482,20 +487,14 @@ class GraphPO:
         if code != GPO_OK:
             raise GraphPOError(code, self.last_error())
 
-    def compute_host(self, host_batch: Batch, out=None, stream=None, chunk_bytes=32 << 20) -> "torch.Tensor":
-        """End-to-end call on HOST tensors (pinned for asynchronous copies): copies the
-        inputs into device staging buffers (kept between calls of the same shape),
-        runs the path and copies the per-token advantages back into `out` (a pinned
-        float32 tensor of total_tokens elements, allocated if None).  Waits for the
-        result and raises on a device-side error.
-
-        When the group-resident path serves the batch and its embeddings span at least
-        four chunks, the work is pipelined over chunks of groups (about `chunk_bytes` of
-        embeddings each; below four chunks the fixed cost of a pipeline stage outweighs
-        the overlap): chunk k's
-        embeddings are copied in on one stream while earlier chunks run (each on one
-        of a few compute streams, so that their kernels share the GPU) and the
-        advantages of finished chunks are copied back on a third stream."""
+    def compute_host(self, host_batch: Batch, out=None, stream=None, chunk_bytes=0) -> "torch.Tensor":
+        """End-to-end call on HOST tensors (pinned for asynchronous copies) through
+        gpo_compute_host: the library uploads the batch into device staging buffers (kept
+        here between calls of the same shape), runs the path over chunks of groups with the
+        uploads of later chunks overlapping the work on earlier ones, and copies the
+        per-token advantages back into `out` (a pinned float32 tensor of total_tokens
+        elements, allocated if None).  chunk_bytes: embedding bytes per pipeline stage (0:
+        the library's default).  Waits for the result and raises on a device-side error."""
         import torch
         dev = torch.device("cuda", torch.cuda.current_device())
         main = torch.cuda.current_stream(dev) if stream is None else stream
@@ -504,79 +503,20 @@ class GraphPO:
         host = [getattr(host_batch, n) for n in names]
         key = (dev, tuple(None if t is None else (tuple(t.shape), t.dtype) for t in host))
         if getattr(self, "_stage_key", None) != key:
-            staged = [None if t is None else torch.empty(t.shape, dtype=t.dtype, device=dev) for t in host]
-            self._staged = staged
+            self._staged = [None if t is None else torch.empty(t.shape, dtype=t.dtype, device=dev) for t in host]
             self._stage_key = key
             self._stage_out = None
         if out is None:
             out = torch.empty(host_batch.total_tokens, dtype=torch.float32, pin_memory=True)
-        emb_h = host_batch.emb
-        G = host_batch.num_groups
-        nchunk = min(G, max(1, emb_h.numel() * emb_h.element_size() // max(1, chunk_bytes)))
-        piped = (nchunk >= 4 and emb_h.dtype == torch.bfloat16 and self.params.flags == 0 and
-                 host_batch.max_states_per_group <= FUSED_MAX_STATES and emb_h.is_pinned())
-        with torch.cuda.stream(main):
-            for i, (h, d) in enumerate(zip(host, self._staged)):
-                if h is not None and (not piped or names[i] != "emb"):
-                    d.copy_(h, non_blocking=True)
-            db = Batch(*self._staged[:6], host_batch.total_tokens, host_batch.max_states_per_group,
-                       *self._staged[6:])
-            if self._stage_out is None:
-                self._stage_out = self.alloc_outputs(db)
-            res = self._stage_out["adv"]
-            if not piped:
-                self.compute_into(db, self._stage_out, stream=main)
-                out.copy_(res, non_blocking=True)
-                self.check(main)
-                return out
-            ws = self.workspace(db)
-            # chunks of groups with about equal numbers of states
-            if host_batch.is_tree:
-                s_of_g = host_batch.group_state_off.tolist()
-                t_of_g = host_batch.group_token_off.tolist()
-            else:
-                so = host_batch.rollout_step_off
-                go = host_batch.group_rollout_off
-                to = host_batch.rollout_token_off
-                s_of_g = so[go.long()].tolist()
-                t_of_g = to[go.long()].tolist()
-            N = s_of_g[-1]
-            bounds, g = [0], 0
-            for k in range(1, nchunk):
-                target = N * k // nchunk
-                while g < G and s_of_g[g] < target:
-                    g += 1
-                if g > bounds[-1] and g < G:
-                    bounds.append(g)
-            bounds.append(G)
-            if getattr(self, "_pipe_streams", None) is None or self._pipe_streams[0].device != dev:
-                self._pipe_streams = [torch.cuda.Stream(dev) for _ in range(4)]  # in, out, 2 compute
-            s_in, s_out, comp = self._pipe_streams[0], self._pipe_streams[1], self._pipe_streams[2:]
-            cb, co = db.c_struct(), _c_outputs(self._stage_out)
-            self._groups_raw(cb, co, 0, 0, True, ws, main)  # clears the status words
-            ready = torch.cuda.Event()
-            ready.record(main)
-            s_in.wait_event(ready)
-            s_out.wait_event(ready)
-            for cs in comp:
-                cs.wait_event(ready)
-            emb_d = self._staged[4]
-            for k in range(len(bounds) - 1):
-                ga, gb = bounds[k], bounds[k + 1]
-                sa, sb = s_of_g[ga], s_of_g[gb]
-                with torch.cuda.stream(s_in):
-                    emb_d[sa:sb].copy_(emb_h[sa:sb], non_blocking=True)
-                    e_in = torch.cuda.Event()
-                    e_in.record(s_in)
-                cs = comp[k % len(comp)]
-                cs.wait_event(e_in)
-                self._groups_raw(cb, co, ga, gb - ga, False, ws, cs)
-                e_c = torch.cuda.Event()
-                e_c.record(cs)
-                s_out.wait_event(e_c)
-                ta, tb = t_of_g[ga], t_of_g[gb]
-                with torch.cuda.stream(s_out):
-                    out[ta:tb].copy_(res[ta:tb], non_blocking=True)
-            main.wait_stream(s_out)
+        db = Batch(*self._staged[:6], host_batch.total_tokens, host_batch.max_states_per_group, *self._staged[6:])
+        if self._stage_out is None:
+            self._stage_out = self.alloc_outputs(db)
+        ws = self.workspace(db)
+        hb, cb, co = host_batch.c_struct(), db.c_struct(), _c_outputs(self._stage_out)
+        code = self._lib.gpo_compute_host(self._h, ctypes.byref(hb), ctypes.byref(cb), ctypes.byref(co),
+                                          out.data_ptr() if out.numel() else None, int(chunk_bytes), ws.data_ptr(),
+                                          ws.numel(), ctypes.c_void_p(main.cuda_stream))
+        if code != GPO_OK:
+            raise GraphPOError(code, self.last_error())
         self.check(main)
         return out

@@ -9,6 +9,11 @@
 #include <cstring>
 #include <mutex>
 
+#include <algorithm>
+#include <vector>
+
+#include <nvtx3/nvToolsExt.h>
+
 #include "gpo_internal.cuh"
 
 struct gpo_ctx {
@@ -22,6 +27,12 @@ struct gpo_ctx {
   int nstages;                 // stages recorded by the last gpo_compute
   cudaEvent_t ev[gpo::kMaxStages + 1];
   const char* stage_name[gpo::kMaxStages];
+  // gpo_compute_host: helper streams and events (created by its first pipelined call) and
+  // the per-group state and token offsets of the last host batch
+  bool pipe_ready;
+  cudaStream_t pipe_in, pipe_out, pipe_comp[gpo::kPipeComputeStreams];
+  cudaEvent_t pipe_ev[2 * gpo::kPipeMaxChunks + 2];
+  std::vector<int64_t> pipe_s, pipe_t;
 };
 
 namespace gpo {
@@ -243,6 +254,7 @@ gpo_status gpo_create(gpo_ctx** out, const gpo_params* params) {
   }
   c->num_sms = prop.multiProcessorCount;
   c->timing = false;
+  c->pipe_ready = false;
   c->nstages = 0;
   for (int i = 0; i <= kMaxStages; ++i) {
     if (cudaEventCreate(&c->ev[i]) != cudaSuccess) {
@@ -264,6 +276,12 @@ gpo_status gpo_create(gpo_ctx** out, const gpo_params* params) {
 
 void gpo_destroy(gpo_ctx* ctx) {
   if (!ctx) return;
+  if (ctx->pipe_ready) {
+    cudaStreamDestroy(ctx->pipe_in);
+    cudaStreamDestroy(ctx->pipe_out);
+    for (cudaStream_t cs : ctx->pipe_comp) cudaStreamDestroy(cs);
+    for (cudaEvent_t ev : ctx->pipe_ev) cudaEventDestroy(ev);
+  }
   if (ctx->host_status) cudaFreeHost(ctx->host_status);
   for (int i = 0; i <= kMaxStages; ++i)
     if (ctx->ev[i]) cudaEventDestroy(ctx->ev[i]);
@@ -375,7 +393,12 @@ gpo_status compute_impl(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs*
   }
 
   int ns = 0;
-  auto stage = [&](const char* name, cudaError_t e) {
+  // one kernel launch of the path: an NVTX range around its enqueue (host-side trace) and,
+  // with timing on, a CUDA event after it
+  auto stage = [&](const char* name, auto launch) {
+    nvtxRangePushA(name);
+    cudaError_t e = launch();
+    nvtxRangePop();
     if (ctx->timing && e == cudaSuccess && ns < kMaxStages) {
       ctx->stage_name[ns] = name;
       e = cudaEventRecord(ctx->ev[++ns], lc.stream);
@@ -397,22 +420,24 @@ gpo_status compute_impl(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs*
     if (e == cudaSuccess && !bud && (int64_t)(g1 - g0) > (int64_t)grid) {
       Sizes rest = sz;
       rest.g0 = sz.g0 + grid;
-      e = stage("exact_stats", launch_exact_stats(lc, b, rest, ws));
+      e = stage("exact_stats", [&] { return launch_exact_stats(lc, b, rest, ws); });
     }
-    if (e == cudaSuccess) e = stage("fused", launch_fused(lc, map, map32, b, *out, sz, ws, pp));
+    if (e == cudaSuccess) e = stage("fused", [&] { return launch_fused(lc, map, map32, b, *out, sz, ws, pp); });
   } else {
-    if (e == cudaSuccess && b.parent) e = stage("tree_prep", launch_tree_prep(lc, b, sz, ws));
-    if (e == cudaSuccess) e = stage("prep", launch_prep(lc, b, sz, ws));
+    if (e == cudaSuccess && b.parent) e = stage("tree_prep", [&] { return launch_tree_prep(lc, b, sz, ws); });
+    if (e == cudaSuccess) e = stage("prep", [&] { return launch_prep(lc, b, sz, ws); });
     if (e == cudaSuccess && sz.N > 0) {
       // the fp32 norms of the threshold test come from the Gram tiles (tcgen05) or from
       // row_stats (CUDA cores); eta takes compensated norms and parent dots (exact_stats),
       // after the similarity stage so that the fp32 norms give the sums' biases
-      if (e == cudaSuccess && !use_tc) e = stage("row_stats", launch_row_stats(lc, b, sz, ws));
+      if (e == cudaSuccess && !use_tc) e = stage("row_stats", [&] { return launch_row_stats(lc, b, sz, ws); });
       if (e == cudaSuccess)
-        e = stage("similarity", use_tc ? launch_sim_tc(lc, map, b, sz, ws, pp) : launch_sim_simt(lc, b, sz, ws, pp));
-      if (e == cudaSuccess && !bud) e = stage("exact_stats", launch_exact_stats(lc, b, sz, ws, true));
-      if (e == cudaSuccess) e = stage("groups", launch_groups(lc, b, *out, sz, ws, pp));
-      if (e == cudaSuccess && !bud) e = stage("tokens", launch_tokens(lc, b, *out, sz, ws));
+        e = stage("similarity", [&] {
+          return use_tc ? launch_sim_tc(lc, map, b, sz, ws, pp) : launch_sim_simt(lc, b, sz, ws, pp);
+        });
+      if (e == cudaSuccess && !bud) e = stage("exact_stats", [&] { return launch_exact_stats(lc, b, sz, ws, true); });
+      if (e == cudaSuccess) e = stage("groups", [&] { return launch_groups(lc, b, *out, sz, ws, pp); });
+      if (e == cudaSuccess && !bud) e = stage("tokens", [&] { return launch_tokens(lc, b, *out, sz, ws); });
     }
   }
   ctx->nstages = ns;
@@ -456,6 +481,151 @@ gpo_status gpo_compute_groups(gpo_ctx* ctx, const gpo_batch* batch, const gpo_ou
                    (long long)(first_group + num_groups), (long long)batch->num_groups), GPO_ERR_INVALID_ARG;
   return compute_impl(ctx, batch, out, workspace, workspace_bytes, first_group, first_group + num_groups,
                       clear_status != 0, stream);
+}
+
+gpo_status gpo_compute_host(gpo_ctx* ctx, const gpo_batch* host, const gpo_batch* dev, const gpo_outputs* out,
+                            float* host_adv, int64_t chunk_bytes, void* workspace, size_t workspace_bytes,
+                            void* stream) {
+  if (!ctx || !host || !dev) return GPO_ERR_INVALID_ARG;
+  ctx->msg[0] = 0;
+  gpo_status s = check_batch(ctx, dev);
+  if (s == GPO_OK) s = check_outputs(ctx, dev, out);
+  if (s != GPO_OK) return s;
+  const gpo_batch& h = *host;
+  const gpo_batch& d = *dev;
+  const bool tree = d.parent != nullptr;
+  if (h.num_groups != d.num_groups || h.num_rollouts != d.num_rollouts || h.num_states != d.num_states ||
+      h.d != d.d || h.emb_dtype != d.emb_dtype || h.emb_row_stride != d.emb_row_stride ||
+      h.total_tokens != d.total_tokens || (h.parent != nullptr) != tree || (h.root_emb != nullptr) != (d.root_emb != nullptr))
+    return set_msg(ctx, "host and device batches differ in size or layout"), GPO_ERR_INVALID_ARG;
+  const int64_t G = d.num_groups, R = d.num_rollouts, N = d.num_states, T = d.total_tokens;
+  if (!h.group_rollout_off || (N > 0 && (!h.step_len || !h.emb)) || (R > 0 && !h.reward) ||
+      (tree ? (!h.group_state_off || !h.group_token_off) : (!h.rollout_step_off || !h.rollout_token_off)) ||
+      (T > 0 && !host_adv))
+    return set_msg(ctx, "a host array is NULL"), GPO_ERR_INVALID_ARG;
+  if (chunk_bytes < 0) return set_msg(ctx, "chunk_bytes < 0"), GPO_ERR_INVALID_ARG;
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const size_t esz = d.emb_dtype == GPO_EMB_BF16 ? 2 : 4;
+  const size_t row = (size_t)d.emb_row_stride * esz;
+  cudaError_t e = cudaSuccess;
+  auto up = [&](const void* dst, const void* src, size_t bytes, cudaStream_t s) {
+    if (e == cudaSuccess && bytes > 0) e = cudaMemcpyAsync(const_cast<void*>(dst), src, bytes, cudaMemcpyHostToDevice, s);
+  };
+  // the small arrays first, on the caller's stream
+  up(d.group_rollout_off, h.group_rollout_off, 4 * (G + 1), st);
+  if (tree) {
+    up(d.parent, h.parent, 4 * N, st);
+    up(d.group_state_off, h.group_state_off, 4 * (G + 1), st);
+    up(d.group_token_off, h.group_token_off, 8 * (G + 1), st);
+  }
+  if (d.rollout_step_off && h.rollout_step_off) up(d.rollout_step_off, h.rollout_step_off, 4 * (R + 1), st);
+  if (d.rollout_token_off && h.rollout_token_off) up(d.rollout_token_off, h.rollout_token_off, 8 * (R + 1), st);
+  up(d.step_len, h.step_len, 4 * N, st);
+  up(d.reward, h.reward, R, st);
+  if (d.root_emb) up(d.root_emb, h.root_emb, row * G, st);
+  if (e != cudaSuccess) return set_msg(ctx, "upload failed: %s", cudaGetErrorString(e)), GPO_ERR_CUDA;
+
+  // chunks of groups with about equal numbers of states, from the host offsets (checked here;
+  // offsets that do not partition the batch leave it to one launch, whose kernels report them)
+  const int64_t emb_bytes = N * (int64_t)row;
+  // default: stages of at least 8 MiB, at most ten of them
+  if (chunk_bytes == 0) chunk_bytes = std::max<int64_t>(kPipeMinChunkBytes, emb_bytes / 10);
+  int64_t nchunk = emb_bytes / chunk_bytes;
+  nchunk = std::min<int64_t>(std::min<int64_t>(nchunk, G), kPipeMaxChunks);
+  bool piped = nchunk >= 2 && d.emb_dtype == GPO_EMB_BF16 && ctx->params.flags == 0 &&
+               d.max_states_per_group <= kFusedMaxStates;
+  if (piped) {
+    ctx->pipe_s.resize(G + 1);
+    ctx->pipe_t.resize(G + 1);
+    for (int64_t g = 0; g <= G && piped; ++g) {
+      int64_t sv, tv;
+      if (tree) {
+        sv = h.group_state_off[g];
+        tv = h.group_token_off[g];
+      } else {
+        const int32_t r = h.group_rollout_off[g];
+        piped = r >= 0 && r <= R;
+        sv = piped ? h.rollout_step_off[r] : 0;
+        tv = piped ? h.rollout_token_off[r] : 0;
+      }
+      piped = piped && sv >= 0 && sv <= N && tv >= 0 && tv <= T &&
+              (g == 0 ? sv == 0 && tv == 0 : sv >= ctx->pipe_s[g - 1] && tv >= ctx->pipe_t[g - 1]) &&
+              (g < G || (sv == N && tv == T));
+      ctx->pipe_s[g] = sv;
+      ctx->pipe_t[g] = tv;
+    }
+  }
+  if (piped && !ctx->pipe_ready) {
+    bool ok = cudaStreamCreateWithFlags(&ctx->pipe_in, cudaStreamNonBlocking) == cudaSuccess &&
+              cudaStreamCreateWithFlags(&ctx->pipe_out, cudaStreamNonBlocking) == cudaSuccess;
+    for (cudaStream_t& cs : ctx->pipe_comp) ok = ok && cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking) == cudaSuccess;
+    for (cudaEvent_t& ev : ctx->pipe_ev) ok = ok && cudaEventCreateWithFlags(&ev, cudaEventDisableTiming) == cudaSuccess;
+    if (!ok) {
+      cudaGetLastError();
+      return set_msg(ctx, "could not create the pipeline's streams and events"), GPO_ERR_CUDA;
+    }
+    ctx->pipe_ready = true;
+  }
+  if (!piped) {  // one upload, the whole path, one download
+    up(d.emb, h.emb, (size_t)emb_bytes, st);
+    if (e != cudaSuccess) return set_msg(ctx, "upload failed: %s", cudaGetErrorString(e)), GPO_ERR_CUDA;
+    s = compute_impl(ctx, dev, out, workspace, workspace_bytes, 0, G, true, stream);
+    if (s != GPO_OK) return s;
+    if (T > 0 && (e = cudaMemcpyAsync(host_adv, out->adv, 4 * T, cudaMemcpyDeviceToHost, st)) != cudaSuccess)
+      return set_msg(ctx, "download failed: %s", cudaGetErrorString(e)), GPO_ERR_CUDA;
+    return GPO_OK;
+  }
+  nvtxRangePushA("gpo_compute_host pipeline");
+  const bool timing = ctx->timing;  // per-stage events would interleave across the streams
+  ctx->timing = false;
+  s = compute_impl(ctx, dev, out, workspace, workspace_bytes, 0, 0, true, stream);  // clears the status words
+  cudaEvent_t* ev = ctx->pipe_ev;
+  const cudaEvent_t ready = ev[2 * kPipeMaxChunks], done = ev[2 * kPipeMaxChunks + 1];
+  if (s == GPO_OK) {
+    e = cudaEventRecord(ready, st);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(ctx->pipe_in, ready, 0);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(ctx->pipe_out, ready, 0);
+    for (cudaStream_t cs : ctx->pipe_comp)
+      if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, ready, 0);
+    // chunk k: its embeddings in on pipe_in, its groups on a compute stream
+    int64_t bounds[kPipeMaxChunks + 1];
+    int64_t nb = 0, ga = 0;
+    bounds[0] = 0;
+    for (int64_t k = 0; k < nchunk && e == cudaSuccess && s == GPO_OK; ++k) {
+      int64_t gb = ga;
+      const int64_t target = k + 1 == nchunk ? N : N * (k + 1) / nchunk;
+      while (gb < G && (ctx->pipe_s[gb] < target || gb == ga)) ++gb;
+      if (k + 1 == nchunk) gb = G;
+      if (gb <= ga) continue;
+      const int64_t sa = ctx->pipe_s[ga], sb = ctx->pipe_s[gb];
+      up(static_cast<const char*>(d.emb) + sa * row, static_cast<const char*>(h.emb) + sa * row, (size_t)(sb - sa) * row,
+         ctx->pipe_in);
+      if (e == cudaSuccess) e = cudaEventRecord(ev[2 * nb], ctx->pipe_in);
+      const cudaStream_t cs = ctx->pipe_comp[nb % kPipeComputeStreams];
+      if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, ev[2 * nb], 0);
+      if (e == cudaSuccess) s = compute_impl(ctx, dev, out, workspace, workspace_bytes, ga, gb, false, cs);
+      if (e == cudaSuccess && s == GPO_OK) e = cudaEventRecord(ev[2 * nb + 1], cs);
+      bounds[++nb] = gb;
+      ga = gb;
+    }
+    // the chunks' tokens out on pipe_out, each as soon as its groups are done: downloads
+    // share the host link with the later chunks' uploads, which moves more bytes per second
+    // than uploads first and downloads after
+    for (int64_t k = 0; k < nb && e == cudaSuccess && s == GPO_OK; ++k) {
+      const int64_t ta = ctx->pipe_t[bounds[k]], tb = ctx->pipe_t[bounds[k + 1]];
+      e = cudaStreamWaitEvent(ctx->pipe_out, ev[2 * k + 1], 0);
+      if (e == cudaSuccess && tb > ta)
+        e = cudaMemcpyAsync(host_adv + ta, out->adv + ta, 4 * (tb - ta), cudaMemcpyDeviceToHost, ctx->pipe_out);
+    }
+    // the caller's stream continues after the last download (which follows every chunk)
+    if (e == cudaSuccess) e = cudaEventRecord(done, ctx->pipe_out);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(st, done, 0);
+  }
+  ctx->timing = timing;
+  nvtxRangePop();
+  if (s != GPO_OK) return s;
+  if (e != cudaSuccess) return set_msg(ctx, "pipeline enqueue failed: %s", cudaGetErrorString(e)), GPO_ERR_CUDA;
+  return GPO_OK;
 }
 
 }  // extern "C"

@@ -20,6 +20,9 @@ constexpr int kEdgeCap = 384;        // spanning-forest edges one item can emit 
 constexpr int kStatusWords = 16;
 constexpr int kMaxStages = 8;        // timed stages of one gpo_compute
 constexpr int kFusedMaxStates = 384; // largest group of the fused group-resident kernel
+constexpr int kPipeMaxChunks = 64;   // gpo_compute_host: pipeline stages at most
+constexpr int kPipeComputeStreams = 3;
+constexpr int64_t kPipeMinChunkBytes = (int64_t)8 << 20;
 
 // status words (uint32) at the head of the workspace
 enum : int {

@@ -148,3 +148,52 @@ def test_compute_host_tree_layout_pipelined(P):
     ref = gp(P.Batch.from_arrays(b, device="cuda"))
     gp.check()
     assert torch.equal(out, ref["adv"].cpu()) and torch.equal(again, out)
+
+
+@pytest.mark.gpu
+def test_compute_host_argument_checks(P):
+    """gpo_compute_host refuses host and device batches of different sizes, and a NULL host array."""
+    import ctypes
+    import torch
+    b = W.make_batch(W.CONFIGS["math"].scaled(2))
+    gp = P.GraphPO(kappa=b["kappa"], w=b["w"], lambda_eff=b["lambda_eff"])
+    hb = P.Batch.from_arrays(b, device="cpu", pin=True)
+    db = P.Batch.from_arrays(b, device="cuda")
+    out = gp.alloc_outputs(db)
+    ws = gp.workspace(db)
+    host_adv = torch.empty(hb.total_tokens, dtype=torch.float32, pin_memory=True)
+    L = P.binding.load()
+    co = P.binding._c_outputs(out)
+    stream = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+
+    def call(h, d, adv_ptr):
+        return L.gpo_compute_host(gp._h, ctypes.byref(h), ctypes.byref(d), ctypes.byref(co), adv_ptr, 0,
+                                  ws.data_ptr(), ws.numel(), stream)
+
+    h, d = hb.c_struct(), db.c_struct()
+    h.total_tokens += 1
+    assert call(h, d, host_adv.data_ptr()) == 1
+    h = hb.c_struct()
+    h.emb_row_stride += 8
+    assert call(h, d, host_adv.data_ptr()) == 1
+    assert call(hb.c_struct(), d, None) == 1  # no host output
+    h = hb.c_struct()
+    h.step_len = None
+    assert call(h, d, host_adv.data_ptr()) == 1
+    # a correct call on the same context afterwards
+    assert call(hb.c_struct(), d, host_adv.data_ptr()) == 0
+    gp.check()
+    ref = gp(db)["adv"].cpu()
+    torch.cuda.synchronize()
+    assert torch.equal(host_adv, ref)
+
+
+@pytest.mark.gpu
+def test_compute_host_pageable_memory(P):
+    """Host arrays in pageable memory (no pinning): same advantages, one upload at a time."""
+    b = W.make_batch(W.CONFIGS["math"].scaled(4))
+    gp = P.GraphPO(kappa=b["kappa"], w=b["w"], lambda_eff=b["lambda_eff"])
+    hb = P.Batch.from_arrays(b, device="cpu", pin=False)
+    out = gp.compute_host(hb, chunk_bytes=1 << 20)
+    ref = gp(P.Batch.from_arrays(b, device="cuda"))["adv"].cpu()
+    assert (out == ref).all()
