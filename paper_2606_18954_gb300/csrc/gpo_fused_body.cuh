@@ -17,6 +17,7 @@ constexpr int kWarpEdges = 256;                 // linked pairs listed per epilo
 constexpr int kEdgeList = kWarpEdges * (kEpiThreads / 32);
 constexpr int kBarGroup = 1;                    // named barrier of the group warps
 constexpr int kBarEpi = 2;                      // named barrier of the drain warps
+constexpr int kBarSetup = 3;                    // named barrier of warps 2 and 3 (early set-up)
 static_assert(kThreads % 128 == 0 && kThreads >= 256 && kGThreads >= kMaxN, "fused kernel shape");
 
 struct Seg {
@@ -132,6 +133,7 @@ struct __align__(16) GroupSmem {
   unsigned long long esum[3];  // exploration efficiency: token sums
   int flags;             // bit 0: group invalid
   int overflow;          // some warp found more pairs than its part of elist holds
+  int stats_next;        // next block of 8 rows for the row statistics (claimed by warps)
   Plan plan;
   uint32_t elist[kEdgeList];  // linked pairs of the group, kWarpEdges per epilogue warp: i | j << 16
   alignas(16) unsigned char X[group_scratch_sep_bytes(kMaxN)];  // group-math sums (separate layout)
@@ -157,6 +159,7 @@ static_assert(kTilesOff + 1023 + kRingBytes <= 232448, "fused kernel exceeds 227
 
 __device__ __forceinline__ void bar_group() { asm volatile("bar.sync %0, %1;" ::"n"(kBarGroup), "n"(kGThreads) : "memory"); }
 __device__ __forceinline__ void bar_epi() { asm volatile("bar.sync %0, %1;" ::"n"(kBarEpi), "n"(kEpiThreads) : "memory"); }
+__device__ __forceinline__ void bar_setup() { asm volatile("bar.sync %0, %1;" ::"n"(kBarSetup), "n"(64) : "memory"); }
 
 // Bits a..31 of a word (all for a <= 0, none for a >= 32).
 __device__ __forceinline__ uint32_t bits_from(int a) { return a <= 0 ? 0xFFFFFFFFu : (a >= 32 ? 0u : 0xFFFFFFFFu << a); }
@@ -184,13 +187,15 @@ __device__ __forceinline__ float pick(const uint32_t (&r)[32], int j) {
 }
 
 // Compensated |z_v|^2 and <z_{p(v)}, z_v> of the group's states [s0, s0 + n) into
-// ws.x_n2 / ws.x_dot (float pairs), and |prompt embedding|^2 into ws.x_root_n2[g]; every
-// group thread calls it (wg = group warp 0.., lane).  Parents from the group layout in
-// shared memory (chain: the previous state unless the state is a rollout's first; tree:
-// gs->par).
+// ws.x_n2 / ws.x_dot (float pairs).  The calling warps claim blocks of 8 rows from
+// gs->stats_next until none is left, so that warps that join late or run slower take
+// fewer.  Parents: with `early` (chain layout, before the group's set-up) the previous
+// state for every state but the group's first (the set-up fixes the rollouts' first
+// states afterwards: their parent is the prompt root); otherwise from the group layout
+// in shared memory (chain: the previous state unless the state is a rollout's first; tree:
+// gs->par; the prompt embedding for a root child when there is one).
 __device__ __forceinline__ void group_row_stats(const gpo_batch& b, const Sizes& sz, const Ws& ws, GroupSmem* gs,
-                                                int g, int s0, int n, bool tree, int wg, int lane, uint32_t* st) {
-  constexpr int kGWarps = kGThreads / 32;
+                                                int g, int s0, int n, bool tree, bool early, int lane, uint32_t* st) {
   const int r = lane >> 2, c = lane & 3;
   const int nch = sz.d / 8;          // whole 16-byte chunks of a row
   const int64_t rs = sz.stride / 8;  // row stride in 16-byte chunks
@@ -210,14 +215,23 @@ __device__ __forceinline__ void group_row_stats(const gpo_batch& b, const Sizes&
     two_sum(P.x, P.y, h, l);
     return make_float2(h, l);
   };
-  for (int blk = wg; blk * 8 < n; blk += kGWarps) {
+  auto claim = [&]() {
+    int k = 0;
+    if (lane == 0) k = atomicAdd(&gs->stats_next, 1);
+    return __shfl_sync(0xffffffffu, k, 0);
+  };
+  for (int blk = claim(); blk * 8 < n; blk = claim()) {
     const int i = blk * 8 + r;  // local row of this lane
     const bool live = i < n;
     // parent: >= 0 a local row, -2 the prompt embedding, -1 none (eta 0)
     int pl = -1;
     if (live) {
-      pl = tree ? gs->par[i] : (gs->dep[i] > 1 ? i - 1 : -1);
-      if (pl < 0) pl = b.root_emb ? -2 : -1;
+      if (early) {
+        pl = i - 1;
+      } else {
+        pl = tree ? gs->par[i] : (gs->dep[i] > 1 ? i - 1 : -1);
+        if (pl < 0) pl = b.root_emb ? -2 : -1;
+      }
     }
     const bool from_left = pl >= 0 && pl == i - 1 && r > 0;
     const uint4* zb = Z + (int64_t)(s0 + (live ? i : 0)) * rs;
@@ -308,14 +322,6 @@ __device__ __forceinline__ void group_row_stats(const gpo_batch& b, const Sizes&
       if (!isfinite(n2.x) || !isfinite(dot.x)) report(st, GPO_ERR_NONFINITE, 3, s0 + i);
       ws.x_n2[s0 + i] = n2;
       ws.x_dot[s0 + i] = dot;
-    }
-  }
-  if (b.root_emb && wg == kGWarps - 1) {  // |prompt embedding|^2, one warp
-    float2 n2, dot;
-    exact_pair_sums<true>(b.root_emb, (int64_t)g * sz.stride, nullptr, 0, false, sz.d, lane, n2, dot);
-    if (lane == 0) {
-      if (!isfinite(n2.x)) report(st, GPO_ERR_NONFINITE, 3, sz.N + g);
-      ws.x_root_n2[g] = n2;
     }
   }
 }
@@ -457,6 +463,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
     mbar_init(&ctl->tempty, kEpiThreads / 32);
     mbar_init(&ctl->drain, 1);
     fence_mbar_init();
+    gs->stats_next = 0;
     tma_prefetch_desc(&zmap);
     tma_prefetch_desc(&zmap32);
   }
@@ -618,24 +625,47 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
         gs->overflow = 0;
       }
 
+      // ---- compensated row statistics of the group (eta needs them; the Gram accumulator
+      //      is too coarse): |z_v|^2 and <z_{p(v)}, z_v> as float pairs into ws.x_n2 / x_dot,
+      //      read from L2 or HBM while the producer streams the same rows, only for each
+      //      CTA's first group (its stream has nothing to overlap before it; later groups'
+      //      come from a launch of their own).  A warp takes 8 rows, lane 4 r + c every fourth
+      //      16-byte chunk of row r starting at chunk c; a parent that is the row before comes
+      //      from the lane 4 below, other parents and the prompt embedding are loaded.  bf16
+      //      products are exact in fp32, every sum is error-free (BiasedSum), the row's 4
+      //      partial pairs are combined in a fixed butterfly.  Chain layout without prompt
+      //      embeddings: the drain warps start at once (every state's parent taken as the
+      //      state before it; a rollout's first state then has eta 0 whatever its dot) while
+      //      warps 2 and 3 lay out the group, then join them; otherwise all group warps
+      //      after the set-up.
+      const bool stats_here = p.mode == 0 && p.stats_in_kernel && g < sz.g0 + (int)gridDim.x;
+      const bool early = stats_here && !tree && b.root_emb == nullptr;
+      if (early && epi) group_row_stats(b, sz, ws, gs, g, s0, n, false, true, lane, st);
+
       if (tree) {
         tree_setup(b, sz, gs, g, r0, nr, s0, n, gt, wg, lane, st);
-      } else {
-      // ---- validate the group and lay out its states (Sec. 4.2 chain layout)
-      for (int r = gt; r <= nr; r += kGThreads) {
+      } else if (!early || !epi) {
+      // ---- validate the group and lay out its states (Sec. 4.2 chain layout): all group
+      //      threads, or warps 2 and 3 alone while the drain warps read the statistics
+      const int tid = gt, nt = early ? 64 : kGThreads;  // warps 2 and 3: gt = 0..63
+      auto sync = [&] {
+        if (early) bar_setup();
+        else bar_group();
+      };
+      for (int r = tid; r <= nr; r += nt) {
         gs->rstart[r] = b.rollout_step_off[r0 + r] - s0;
         gs->tok0[r] = b.rollout_token_off[r0 + r];
       }
-      for (int r = gt; r < nr; r += kGThreads) gs->rew[r] = b.reward[r0 + r];
-      group_scratch_zero(gs->X, n, gt, kGThreads);  // read after the drain
-      for (int i = gt; i < n; i += kGThreads) {
+      for (int r = tid; r < nr; r += nt) gs->rew[r] = b.reward[r0 + r];
+      group_scratch_zero(gs->X, n, tid, nt);  // read after the drain
+      for (int i = tid; i < n; i += nt) {
         gs->lab[i] = i;
         gs->slen[i] = b.step_len[s0 + i];
         gs->roll[i] = 0;
         gs->dep[i] = 1;
       }
-      bar_group();
-      for (int r = gt; r < nr; r += kGThreads) {
+      sync();
+      for (int r = tid; r < nr; r += nt) {
         const int a = gs->rstart[r], e = gs->rstart[r + 1];
         bool bad = !(a >= 0 && e > a && e <= n) || gs->rew[r] > 1;
         if (gs->rew[r] > 1) report(st, GPO_ERR_BAD_REWARD, 2, r0 + r);
@@ -656,21 +686,19 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
           atomicOr(&gs->flags, 1);
         }
       }
-      bar_group();
+      if (early) group_row_stats(b, sz, ws, gs, g, s0, n, false, true, lane, st);  // join the drain warps
       }
+      bar_group();  // set-up (and with `early` the row statistics) complete
       const bool valid = (gs->flags & 1) == 0;
-
-      // ---- compensated row statistics of the group (eta needs them; the Gram accumulator
-      //      is too coarse): |z_v|^2 and <z_{p(v)}, z_v> as float pairs into ws.x_n2 / x_dot,
-      //      by the group warps while the producer streams the same rows (L2 serves the
-      //      second reader; only for each CTA's first group, whose stream has nothing to
-      //      overlap before it, so that the work does not delay the CTA's next groups).  A warp takes 8 rows, lane 4 r + c every fourth 16-byte chunk of
-      //      row r starting at chunk c; a parent that is the row before comes from the lane
-      //      4 below, other parents and the prompt embedding are loaded.  bf16 products are
-      //      exact in fp32, every sum is compensated (TwoSum per element, two fp32 lanes per
-      //      instruction), the row's 4 partial pairs are combined in a fixed butterfly.
-      if (valid && p.mode == 0 && p.stats_in_kernel && g < sz.g0 + (int)gridDim.x)
-        group_row_stats(b, sz, ws, gs, g, s0, n, tree, wg, lane, st);
+      if (!early && valid && stats_here) group_row_stats(b, sz, ws, gs, g, s0, n, tree, false, lane, st);
+      if (valid && stats_here && b.root_emb && wg == 0) {  // |prompt embedding|^2, one warp
+        float2 n2, dot;
+        exact_pair_sums<true>(b.root_emb, (int64_t)g * sz.stride, nullptr, 0, false, sz.d, lane, n2, dot);
+        if (lane == 0) {
+          if (!isfinite(n2.x)) report(st, GPO_ERR_NONFINITE, 3, sz.N + g);
+          ws.x_root_n2[g] = n2;
+        }
+      }
 
       // ---- drain the accumulator pass by pass (warps 4..15)
       bool fail = false;
@@ -941,6 +969,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
           }
         }
       }
+      if (gt == 0) gs->stats_next = 0;  // for the next group's row statistics
       bar_group();
     }
   }
