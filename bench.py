@@ -119,8 +119,9 @@ def algorithmic(b):
         "similarity": (zb + 12 * N, flops),
         "groups": (8 * N + R + 12 * R + 4 * N + 17 * N + 8 * N, 0.0),
         "tokens": (4 * T + 8 * N + 4 * N + 4 * N, 0.0),
-        # the group-resident kernel does the whole path, the compensated statistics included
+        # the group-resident kernels do the whole path, the compensated statistics included
         "fused": (path_bytes, flops, alu_x),
+        "fused_f32": (path_bytes, flops, alu_x),
     }
     return dict(N=N, R=R, G=G, T=T, path_bytes=path_bytes, flops=flops, stages=stages)
 
@@ -209,7 +210,8 @@ def traffic_for(kernel_file, workload):
 
 STAGE_SOURCE = {"prep": "gpo_prep.cu", "tree_prep": "gpo_prep.cu", "exact_stats": "gpo_prep.cu",
                 "row_stats": "gpo_prep.cu", "similarity": "gpo_sim_tc.cu",
-                "groups": "gpo_group.cu", "tokens": "gpo_prep.cu", "fused": "gpo_fused.cu"}
+                "groups": "gpo_group.cu", "tokens": "gpo_prep.cu", "fused": "gpo_fused.cu",
+                "fused_f32": "gpo_fused_f32.cu"}
 
 
 def cpu_baseline(b, budget_s=6.0, max_groups=None):

@@ -109,9 +109,10 @@ typedef struct {
 /* Compute the pairwise similarities of bf16 embeddings on the CUDA cores (fp32
  * FMA) instead of the tcgen05 tensor cores; fp32 embeddings always use them. */
 #define GPO_FLAG_SIMT_SIMILARITY 1
-/* Use the multi-kernel tiled path even when every group fits the fused
- * group-resident kernel (bf16 embeddings, max_states_per_group <= 384);
- * for comparisons and tests. */
+/* Use the multi-kernel tiled path even when every group fits a group-resident
+ * kernel (bf16 embeddings with max_states_per_group <= 384, or fp32 embeddings in
+ * the chain layout with small groups, see gpo_compute_groups); for comparisons
+ * and tests. */
 #define GPO_FLAG_TILED 2
 /* For tests of the failure path only: in every CTA of the tensor-core kernels the MMA warp's
  * first wait runs out (it waits about a millisecond on an mbarrier that nothing arrives on),
@@ -198,8 +199,10 @@ gpo_status gpo_compute(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* 
  * the first error of any.  num_groups = 0 with clear_status = 1 only clears.
  * Calls for disjoint ranges may run concurrently on different streams once the
  * clearing call has completed; they share the workspace's status words only.
- * A range other than the whole batch needs the group-resident path (bf16
- * embeddings, max_states_per_group <= 384, no flags): otherwise
+ * A range other than the whole batch needs a group-resident path -- bf16
+ * embeddings with max_states_per_group <= 384, or fp32 embeddings in the chain
+ * layout with max_states_per_group <= 128 and max_states_per_group x
+ * (d rounded up to 32, plus 4) floats within 160 KiB; no flags -- otherwise
  * GPO_ERR_UNSUPPORTED.  A range outside [0, num_groups] gives
  * GPO_ERR_INVALID_ARG. */
 gpo_status gpo_compute_groups(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs* out, int64_t first_group,

@@ -264,6 +264,7 @@ gpo_status gpo_create(gpo_ctx** out, const gpo_params* params) {
     }
   }
   if (setup_sim_tc() != cudaSuccess || setup_groups() != cudaSuccess || setup_fused() != cudaSuccess ||
+      setup_fused_f32() != cudaSuccess ||
       setup_tree_prep() != cudaSuccess || setup_loss() != cudaSuccess ||
       cudaMallocHost(&c->host_status, sizeof(uint32_t) * kStatusWords) != cudaSuccess) {
     cudaGetLastError();
@@ -366,10 +367,13 @@ gpo_status compute_impl(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs*
 
   const bool use_tc = b.emb_dtype == GPO_EMB_BF16 && !(p.flags & GPO_FLAG_SIMT_SIMILARITY) && sz.N > 0;
   const bool fused = use_tc && !(p.flags & GPO_FLAG_TILED) && sz.G > 0 && sz.maxn <= kFusedMaxStates;
+  // fp32 embeddings, chain layout, small groups: the one-launch CUDA-core path
+  const bool fused32 = b.emb_dtype == GPO_EMB_F32 && !b.parent && !bud && !(p.flags & GPO_FLAG_TILED) && sz.G > 0 &&
+                       sz.N > 0 && fused_f32_fits(sz.d, sz.maxn);
   const bool whole = g0 == 0 && g1 == sz.G;
-  if (!whole && !fused && g1 > g0) {
-    return set_msg(ctx, "a group range needs the group-resident path (bf16, at most %d states per group, no flags)",
-                   kFusedMaxStates), GPO_ERR_UNSUPPORTED;
+  if (!whole && !fused && !fused32 && g1 > g0) {
+    return set_msg(ctx, "a group range needs a group-resident path (bf16 with at most %d states per group, or fp32 "
+                        "chain layout with small groups; no flags)", kFusedMaxStates), GPO_ERR_UNSUPPORTED;
   }
   // embedding tensor maps: boxes of 64 elements x 128 rows and x 32 rows, 128B swizzle
   CUtensorMap map, map32;
@@ -410,6 +414,8 @@ gpo_status compute_impl(gpo_ctx* ctx, const gpo_batch* batch, const gpo_outputs*
   if (e == cudaSuccess && clear) e = cudaMemsetAsync(ws.status, 0, sizeof(uint32_t) * kStatusWords, lc.stream);
   if (g1 <= g0) {
     // nothing to compute (a call that only clears the status words)
+  } else if (fused32) {
+    if (e == cudaSuccess) e = stage("fused_f32", [&] { return launch_fused_f32(lc, b, *out, sz, ws, pp); });
   } else if (fused) {
     // one group per CTA at a time: the group warps compute the compensated statistics of
     // each CTA's first group while it streams in; the groups after those (more groups than

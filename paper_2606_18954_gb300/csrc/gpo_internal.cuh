@@ -663,6 +663,11 @@ int fused_grid(const LaunchCtx& lc, const Sizes& sz);
 cudaError_t launch_fused(const LaunchCtx& lc, const CUtensorMap& map, const CUtensorMap& map32, const gpo_batch& b,
                          const gpo_outputs& o, const Sizes& sz, const Ws& ws, const Params& p);
 cudaError_t setup_fused();
+// fp32 group-resident path (chain layout, small groups whose rows fit in shared memory)
+bool fused_f32_fits(int d, int maxn);
+cudaError_t setup_fused_f32();
+cudaError_t launch_fused_f32(const LaunchCtx& lc, const gpo_batch& b, const gpo_outputs& o, const Sizes& sz,
+                             const Ws& ws, const Params& p);
 cudaError_t setup_sim_tc();
 cudaError_t setup_groups();
 size_t sim_tc_smem_bytes();

@@ -93,8 +93,10 @@ def oracle_run(b, params, threads=8):
 SCALED = [("tiny", 8), ("math", 4), ("agentic", 24), ("full", 3), ("wide", 1)]
 
 
-# fused: the group-resident kernel (bf16, groups <= 384 states); tiled: the
-# multi-kernel tensor-core path; simt: the multi-kernel CUDA-core path
+# fused: a group-resident kernel (bf16 groups <= 384 states on the tensor cores, fp32
+# chain-layout groups <= 128 states on the CUDA cores); tiled: the multi-kernel path
+# (tensor-core similarity for bf16, CUDA-core for fp32); simt: the multi-kernel CUDA-core
+# path for bf16 (fp32 embeddings take the CUDA cores on every path)
 PATH_FLAGS = {"fused": 0, "tiled": 2, "simt": 1}
 
 
@@ -103,8 +105,8 @@ PATH_FLAGS = {"fused": 0, "tiled": 2, "simt": 1}
 @pytest.mark.parametrize("path", ["fused", "tiled", "simt"])
 def test_parity_scaled(gp_mod, name, groups, rule, path):
     b = batch_of(name, groups)
-    if path != "simt" and b["emb_dtype"] != "bf16":
-        pytest.skip("fp32 embeddings always use the CUDA-core similarity kernel")
+    if path == "simt" and b["emb_dtype"] != "bf16":
+        pytest.skip("fp32 embeddings: the simt flag selects nothing new (same path as fused)")
     params = oracle_params(b, merge_rule=rule)
     ref = oracle_run(b, params)
     gpu = run_gpu(gp_mod, b, params, flags=PATH_FLAGS[path])

@@ -35,10 +35,11 @@ def _gp(P, b, flags=0):
     return P.GraphPO(kappa=b["kappa"], w=b["w"], lambda_eff=b["lambda_eff"], flags=flags)
 
 
+@pytest.mark.parametrize("name", ["math", "tiny"])  # bf16 and fp32 group-resident paths
 @pytest.mark.parametrize("cuts", [(0, 3, 5, 8), (0, 1, 8), (0, 8)], ids=["3-2-3", "1-7", "whole"])
-def test_ranges_cover_batch(P, cuts):
+def test_ranges_cover_batch(P, cuts, name):
     import torch
-    b = _batch("math", 8)
+    b = _batch(name, 8)
     gp = _gp(P, b)
     db = P.Batch.from_arrays(b, device="cuda")
     ref = gp(db, components=True, nodes=True, edges=True, efficiency=True)
