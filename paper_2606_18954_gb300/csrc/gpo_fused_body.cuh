@@ -700,6 +700,19 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
         }
       }
 
+      // ---- eta(p(v), v) of every state from the finished statistics, by warps 2 and 3 while
+      //      the drain warps test the pairs (with `early`: no prompt embedding, a rollout's
+      //      first state has eta 0); the group math takes it from ecor / eeff, which it
+      //      overwrites only with its own outputs, state by state, after reading it
+      if (early && valid && !epi) {
+        for (int i = gt; i < n; i += 64) {
+          const float2 e = gs->dep[i] == 1 ? make_float2(0.f, 0.f)
+                                           : ff_eta(ws.x_dot[s0 + i], ws.x_n2[s0 + i - 1], ws.x_n2[s0 + i]);
+          gs->ecor[i] = e.x;
+          gs->eeff[i] = e.y;
+        }
+      }
+
       // ---- drain the accumulator pass by pass (warps 4..15)
       bool fail = false;
       if (epi) {
@@ -887,6 +900,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
       else if (valid) {
         // eta(p(v), v) from the compensated row statistics (pairs; see exact_stats_kernel)
         auto eta = [&](int i) -> float2 {
+          if (early) return make_float2(gs->ecor[i], gs->eeff[i]);
           const float2 z = make_float2(0.f, 0.f);
           const float2 n1 = gs->dep[i] == 1 ? (b.root_emb ? ws.x_root_n2[g] : z) : ws.x_n2[s0 + i - 1];
           return ff_eta(ws.x_dot[s0 + i], n1, ws.x_n2[s0 + i]);
