@@ -84,7 +84,10 @@ typedef enum {
   GPO_ERR_UNSUPPORTED = 5, /* e.g. a group above GPO_MAX_GROUP_STATES, misaligned embeddings */
   GPO_ERR_CUDA = 6,        /* a CUDA runtime call failed; see gpo_last_error */
   GPO_ERR_TIMEOUT = 7,     /* a device-side wait gave up (the kernel returned cleanly) */
-  GPO_ERR_WORKSPACE = 8    /* workspace missing or smaller than gpo_workspace_size */
+  GPO_ERR_WORKSPACE = 8,   /* workspace missing or smaller than gpo_workspace_size */
+  GPO_ERR_BOUNDS = 9       /* debug build only (GPO_DEBUG): an index computed inside a kernel fell
+                              outside its array; the access was skipped (the kernel and index are
+                              in gpo_last_error) */
 } gpo_status;
 
 typedef enum {

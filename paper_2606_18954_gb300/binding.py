@@ -92,7 +92,9 @@ _lock = threading.Lock()
 
 
 def lib_path() -> str:
-    return _build.LIB
+    """The library this process loads: GRAPHPO_LIB if set (e.g. the debug build,
+    buildlib.DEBUG_LIB), else the in-tree release build."""
+    return os.environ.get("GRAPHPO_LIB") or _build.LIB
 
 
 def load(build_if_missing: bool = False):
@@ -101,7 +103,7 @@ def load(build_if_missing: bool = False):
     with _lock:
         if _lib is not None:
             return _lib
-        path = _build.LIB
+        path = lib_path()
         if not os.path.exists(path):
             if not build_if_missing:
                 raise RuntimeError(f"{path} is missing: build it with paper_2606_18954_gb300.build()")

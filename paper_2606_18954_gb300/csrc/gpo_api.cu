@@ -215,7 +215,11 @@ using namespace gpo;
 
 extern "C" {
 
+#ifdef GPO_DEBUG
+const char* gpo_version(void) { return "graphpo-gb300 0.1 (sm_103a, GPO_DEBUG bounds checks)"; }
+#else
 const char* gpo_version(void) { return "graphpo-gb300 0.1 (sm_103a)"; }
+#endif
 
 const char* gpo_status_string(gpo_status s) {
   switch (s) {
@@ -228,6 +232,7 @@ const char* gpo_status_string(gpo_status s) {
     case GPO_ERR_CUDA: return "CUDA runtime error";
     case GPO_ERR_TIMEOUT: return "device-side wait timed out";
     case GPO_ERR_WORKSPACE: return "workspace missing or too small";
+    case GPO_ERR_BOUNDS: return "index out of bounds inside a kernel (debug build)";
   }
   return "unknown status";
 }

@@ -234,6 +234,11 @@ __device__ __forceinline__ void group_row_stats(const gpo_batch& b, const Sizes&
       }
     }
     const bool from_left = pl >= 0 && pl == i - 1 && r > 0;
+    // (debug build) the rows this lane reads; the whole warp skips the block if any is out of
+    // range, since the sums below shuffle across all its lanes
+    const bool rows_ok =
+        GPO_BOUNDS(st, s0 + (live ? i : 0), sz.N, kWhereStats) && GPO_BOUNDS(st, pl >= 0 ? s0 + pl : 0, sz.N, kWhereStats);
+    if (!__all_sync(0xffffffffu, rows_ok)) continue;
     const uint4* zb = Z + (int64_t)(s0 + (live ? i : 0)) * rs;
     const uint4* pb = pl >= 0 ? Z + (int64_t)(s0 + pl) * rs : (pl == -2 ? RZ + (int64_t)g * rs : nullptr);
     // error-free sums of the exact bf16 products (BiasedSum: a plain fp32 bound of each
@@ -318,7 +323,7 @@ __device__ __forceinline__ void group_row_stats(const gpo_batch& b, const Sizes&
     const float2 n2 = finish4(ns, ne);
     float2 dot = finish4(ds, de);
     if (pl == -1) dot = make_float2(0.f, 0.f);
-    if (live && c == 0) {
+    if (live && c == 0 && GPO_BOUNDS(st, s0 + i, sz.N, kWhereStats)) {
       if (!isfinite(n2.x) || !isfinite(dot.x)) report(st, GPO_ERR_NONFINITE, 3, s0 + i);
       ws.x_n2[s0 + i] = n2;
       ws.x_dot[s0 + i] = dot;
@@ -911,6 +916,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
           gs->eeff[i] = E;
           gs->emask[i] = mask;
           const int v = s0 + i;
+          if (!GPO_BOUNDS(st, v, sz.N, kWhereStateOut)) return;
           if (o.edge_adv) o.edge_adv[v] = dual;
           if (o.class_id) o.class_id[v] = s0 + label;
           if (o.node_score) o.node_score[v] = S;
@@ -956,6 +962,8 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks)
           const int64_t t0 = qa <= qb ? 4 * qb : te;  // tail [t0, te)
           const int64_t tp = hl < 4 ? ts + hl : t0 + (hl - 4);
           const bool scal = hl < 4 ? tp < h1 : (hl < 8 && tp < te);
+          // (debug build) every store below lies in the state's span [ts, te)
+          if (!GPO_BOUNDS(st, ts, sz.T, kWhereTokens) || !GPO_BOUNDS(st, te - 1, sz.T, kWhereTokens)) continue;
           {
             const float4 v = make_float4(x, x, x, x);
             for (int64_t c = qa + hl; c < qb; c += 16) reinterpret_cast<float4*>(o.adv)[c] = v;

@@ -183,6 +183,7 @@ __global__ void __launch_bounds__(kF32Threads, 1) fused_f32_kernel(gpo_batch b, 
       const int dv = d / 4;  // whole 16-byte chunks of a row (rows start on 16 bytes)
       for (int e = tid; e < n * dv; e += nt) {
         const int i = e / dv, k4 = e - i * dv;
+        if (!GPO_BOUNDS(st, (int64_t)i * ds + 4 * k4 + 3, (int64_t)kF32MaxN * ds, kWhereSmemRow)) continue;
         const float4 v = *reinterpret_cast<const float4*>(Z + (int64_t)(s0 + i) * sz.stride + 4 * k4);
         *reinterpret_cast<float4*>(Zs + i * ds + 4 * k4) = v;
       }
@@ -265,6 +266,7 @@ __global__ void __launch_bounds__(kF32Threads, 1) fused_f32_kernel(gpo_batch b, 
       gs->eeff[i] = E;
       gs->emask[i] = mask;
       const int v = s0 + i;
+      if (!GPO_BOUNDS(st, v, sz.N, kWhereStateOut)) return;
       if (o.edge_adv) o.edge_adv[v] = dual;
       if (o.class_id) o.class_id[v] = s0 + label;
       if (o.node_score) o.node_score[v] = S;
@@ -293,6 +295,7 @@ __global__ void __launch_bounds__(kF32Threads, 1) fused_f32_kernel(gpo_batch b, 
       const int64_t t0 = qa <= qb ? 4 * qb : te;  // tail [t0, te)
       const int64_t tp = hl < 4 ? ts + hl : t0 + (hl - 4);
       const bool scal = hl < 4 ? tp < h1 : (hl < 8 && tp < te);
+      if (!GPO_BOUNDS(st, te - 1, sz.T, kWhereTokens)) continue;
       auto put = [&](float* dst, float x) {
         const float4 v = make_float4(x, x, x, x);
         for (int64_t c = qa + hl; c < qb; c += 16) reinterpret_cast<float4*>(dst)[c] = v;

@@ -151,6 +151,7 @@ __global__ void __launch_bounds__(1024) groups_kernel(gpo_batch b, gpo_outputs o
   };
   auto out = [&](int i, int label, float S, float acor, float E, float dual, unsigned char mask) {
     const int v = s0 + i;
+    if (!GPO_BOUNDS(st, v, sz.N, kWhereStateOut)) return;
     ws.e_adv[v] = dual;
     ws.e_cor[v] = acor;
     ws.e_eff[v] = E;

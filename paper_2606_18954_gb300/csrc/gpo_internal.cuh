@@ -108,6 +108,34 @@ __device__ __forceinline__ void report(uint32_t* st, int code, int where, int de
   atomicExch(&st[kStAbort], 1u);
 }
 
+// Bounds checks of the debug build (-DGPO_DEBUG, a stand-in for a device memory checker):
+// GPO_BOUNDS(st, i, n, where) is true when 0 <= i < n; otherwise it reports GPO_ERR_BOUNDS
+// with the index and the check's number (kWhere*), and the caller skips the access.  In the
+// release build it is the constant true and costs nothing.
+#ifdef GPO_DEBUG
+__device__ __forceinline__ bool bounds_ok(uint32_t* st, int64_t i, int64_t n, int where) {
+  if (i >= 0 && i < n) return true;
+  if (atomicCAS(&st[kStError], 0u, (uint32_t)GPO_ERR_BOUNDS) == 0u) {
+    st[kStWhere] = (uint32_t)where;
+    st[kStDetail] = (uint32_t)i;
+  }
+  atomicExch(&st[kStAbort], 1u);
+  return false;
+}
+#define GPO_BOUNDS(st, i, n, where) ::gpo::bounds_ok((st), (int64_t)(i), (int64_t)(n), (where))
+#else
+#define GPO_BOUNDS(st, i, n, where) true
+#endif
+// check numbers (the `where` of GPO_ERR_BOUNDS)
+enum : int {
+  kWhereTokens = 100,      // a token output (index of the 16-byte chunk or of the token)
+  kWhereStateOut = 101,    // a per-state output
+  kWhereStats = 102,       // a row of the compensated statistics (read or written)
+  kWhereEdges = 103,       // an item's spanning-forest edge
+  kWhereNorms = 104,       // an fp32 norm of the similarity stage
+  kWhereSmemRow = 105,     // a row of the fp32 group-resident kernel's shared-memory copy
+};
+
 __device__ __forceinline__ bool aborted(const uint32_t* st) {
   return *((volatile const uint32_t*)&st[kStAbort]) != 0u;
 }

@@ -824,7 +824,9 @@ __global__ void __launch_bounds__(256) tokens_kernel(gpo_batch b, gpo_outputs o,
     for (int j = 0; j < cnt; ++j) {
       const int64_t s = __shfl_sync(0xffffffffu, ts, j);
       const int64_t e = s + __shfl_sync(0xffffffffu, L, j);
-      write_span(o.adv, s, e, __shfl_sync(0xffffffffu, va, j), lane);
+      const float a = __shfl_sync(0xffffffffu, va, j);
+      if (!GPO_BOUNDS(ws.status, e - 1, sz.T, kWhereTokens) || !GPO_BOUNDS(ws.status, s, sz.T, kWhereTokens)) continue;
+      write_span(o.adv, s, e, a, lane);
       if (o.adv_cor) write_span(o.adv_cor, s, e, __shfl_sync(0xffffffffu, vc, j), lane);
       if (o.adv_eff) write_span(o.adv_eff, s, e, __shfl_sync(0xffffffffu, ve, j), lane);
       if (o.eff_mask) write_span_u8(o.eff_mask, s, e, (uint8_t)__shfl_sync(0xffffffffu, vm, j), lane);

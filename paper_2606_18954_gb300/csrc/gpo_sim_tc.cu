@@ -300,7 +300,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int k = 0; k < 32; ++k)
             if (k == lane) dg = __uint_as_float(r[k]);
-          if (t < item.ncols) {
+          if (t < item.ncols && GPO_BOUNDS(st, row, sz.N, kWhereNorms)) {
             const float rni = dg > 0.f ? 1.0f / sqrtf(dg) : 0.f;
             ws.nrm2[row] = dg;
             ws.rn[row] = rni;
@@ -423,7 +423,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int k = base + __popc(act & ((1u << lane) - 1u));
           const int gs = sl < kTileM ? item.row0 + sl : item.col0 + (sl - kTileM);
           const int gr = root < kTileM ? item.row0 + root : item.col0 + (root - kTileM);
-          if (k < kEdgeCap) out[k] = make_int2(gr, gs);
+          if (k < kEdgeCap && GPO_BOUNDS(st, gr, sz.N, kWhereEdges) && GPO_BOUNDS(st, gs, sz.N, kWhereEdges))
+            out[k] = make_int2(gr, gs);
         }
       }
       epi_sync();

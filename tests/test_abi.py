@@ -64,7 +64,7 @@ def test_binding_structs_match_header():
 
 def test_status_strings_and_version(lib):
     assert lib.gpo_version().startswith(b"graphpo-gb300")
-    for code in range(9):
+    for code in range(10):
         assert lib.gpo_status_string(code)
     assert lib.gpo_status_string(123) == b"unknown status"
 
@@ -135,3 +135,17 @@ def test_header_is_plain_c_and_links(lib, tmp_path):
     out = subprocess.run([str(exe)], capture_output=True, text=True)
     assert out.returncode == 0, out
     assert out.stdout.startswith("graphpo-gb300") and "inconsistent offsets" in out.stdout
+
+
+def test_debug_build_compiles_and_loads():
+    """The debug build (GPO_DEBUG: index checks in every kernel, GPO_ERR_BOUNDS) compiles for
+    sm_103a, loads, says so in gpo_version and names the extra status."""
+    from paper_2606_18954_gb300 import buildlib
+    path = buildlib.build(debug=True)
+    assert path == buildlib.DEBUG_LIB and path != buildlib.LIB
+    L = ctypes.CDLL(path)
+    L.gpo_version.restype = ctypes.c_char_p
+    L.gpo_status_string.restype = ctypes.c_char_p
+    L.gpo_status_string.argtypes = [ctypes.c_int]
+    assert b"GPO_DEBUG" in L.gpo_version()
+    assert b"debug build" in L.gpo_status_string(9)
