@@ -15,7 +15,8 @@
 //   graph reward, dual-group advantage (gpo_group_math.cuh), exploration efficiency and
 //   the token scatter (Sec. 4.3-4.5)
 // Replaces the tiled path's six launches for such batches (prep, row norms, similarity,
-// statistics, per-group math, tokens).
+// statistics, per-group math, tokens).  Groups of at most 64 states run with 512 threads
+// (the Gram's k range split between the block's halves), larger ones with 256.
 #include "gpo_group_math.cuh"
 
 namespace gpo {
@@ -23,8 +24,13 @@ namespace gpo {
 namespace {
 
 constexpr int kF32MaxN = 128;
-constexpr int kF32Threads = 256;
 constexpr int kF32MaxZBytes = 160 * 1024;  // the group's rows in shared memory
+// Two instances: 256 threads for groups of up to 128 states (TA <= 8 row blocks of 16), and
+// 512 threads for groups of up to 64 (TA <= 4), whose Gram splits k between the two halves
+// of the block (twice the warps to hide the loop's latency; the second half's partial sums
+// pass through shared memory and are added in a fixed order)
+constexpr int kF32SmallN = 64;
+__host__ __device__ constexpr int f32_partial_bytes(int nt, int tamax) { return (nt / 256 - 1) * tamax * tamax * 256 * 4; }
 
 struct __align__(16) F32Smem {
   int lab[kF32MaxN];
@@ -55,18 +61,22 @@ __host__ __device__ inline int f32_row_stride(int d) { return ((d + 31) & ~31) +
 __device__ __forceinline__ bool any_block(bool f) { return __syncthreads_or(f ? 1 : 0) != 0; }
 
 // Gram block of the group's rows in shared memory (row stride ds floats) and its linked
-// pairs.  Thread (ti, tj) = (tid / 16, tid % 16) accumulates rows ti + 16 a and columns
-// tj + 16 c for a, c < TA (TA = ceil(n / 16)): per 4 elements of k, one 16-byte chunk of
-// each of its TA rows and TA columns (a quarter-warp reads 8 consecutive rows: one bank
-// group each) and 4 TA^2 fma.  The diagonal (ti == tj, a == c) gives the squared norms of
-// the threshold test; after a barrier every comparable pair i < j (another rollout: j at or
+// pairs.  Within each 256-thread part q of the block, thread (ti, tj) = (t / 16, t % 16)
+// (t = tid % 256) accumulates rows ti + 16 a and columns tj + 16 c for a, c < TA
+// (TA = ceil(n / 16)) over part q's range of k: per 4 elements, one 16-byte chunk of each of
+// its TA rows and TA columns (a quarter-warp reads 8 consecutive rows: one bank group each)
+// and 4 TA^2 fma.  With NT / 256 > 1 parts, parts 1.. leave their sums in `part` and part 0
+// adds them in part order.  The diagonal (ti == tj, a == c) gives the squared norms of the
+// threshold test; after a barrier every comparable pair i < j (another rollout: j at or
 // after the end of i's rollout; with the same-depth rule also equal depth) with
 // acc / |z_j| - kappa |z_i| >= 0 is united in the label forest.  Ends with the barrier
 // that publishes the forest.
-template <int TA>
+template <int TA, int NT>
 __device__ __forceinline__ void f32_gram_links(F32Smem* gs, const float* Zs, int n, int d, int ds, int s0,
-                                               float kappa, int rule, int tid, uint32_t* st) {
-  const int ti = tid >> 4, tj = tid & 15;
+                                               float kappa, int rule, int tid, float* part, uint32_t* st) {
+  constexpr int KS = NT / 256;  // parts of the block, each a range of k
+  const int t = tid & 255, kq = tid >> 8;
+  const int ti = t >> 4, tj = t & 15;
   float acc[TA][TA];
 #pragma unroll
   for (int a = 0; a < TA; ++a)
@@ -74,10 +84,12 @@ __device__ __forceinline__ void f32_gram_links(F32Smem* gs, const float* Zs, int
     for (int c = 0; c < TA; ++c) acc[a][c] = 0.f;
   const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f);
   const int kend = (d + 3) & ~3;  // zeros from d on
+  const int kh = ((kend / 4 + KS - 1) / KS) * 4;  // elements of k per part
+  const int ka = kq * kh, kb = min(kend, ka + kh);
   // not unrolled: the loop body is fetched once (the instruction cache is cold on every launch
   // after other work has gone through L2)
 #pragma unroll 1
-  for (int k = 0; k < kend; k += 4) {
+  for (int k = ka; k < kb; k += 4) {
     float4 ra4[TA], cb4[TA];
 #pragma unroll
     for (int a = 0; a < TA; ++a) {
@@ -96,7 +108,23 @@ __device__ __forceinline__ void f32_gram_links(F32Smem* gs, const float* Zs, int
         acc[a][c] = s;
       }
   }
-  if (ti == tj) {
+  if (KS > 1) {  // the other parts' sums into part 0's, in part order
+    if (kq > 0) {
+#pragma unroll
+      for (int a = 0; a < TA; ++a)
+#pragma unroll
+        for (int c = 0; c < TA; ++c) part[(((kq - 1) * TA + a) * TA + c) * 256 + t] = acc[a][c];
+    }
+    __syncthreads();
+    if (kq == 0) {
+      for (int q = 1; q < KS; ++q)
+#pragma unroll
+        for (int a = 0; a < TA; ++a)
+#pragma unroll
+          for (int c = 0; c < TA; ++c) acc[a][c] += part[(((q - 1) * TA + a) * TA + c) * 256 + t];
+    }
+  }
+  if (kq == 0 && ti == tj) {
 #pragma unroll
     for (int a = 0; a < TA; ++a) {
       const int i = ti + 16 * a;
@@ -113,7 +141,7 @@ __device__ __forceinline__ void f32_gram_links(F32Smem* gs, const float* Zs, int
 #pragma unroll
   for (int a = 0; a < TA; ++a) {
     const int i = ti + 16 * a;
-    if (i >= n) continue;
+    if (kq != 0 || i >= n) continue;
     const float th = gs->thr[i];
     const int re = gs->rend[i], di = gs->dep[i];
 #pragma unroll
@@ -128,15 +156,16 @@ __device__ __forceinline__ void f32_gram_links(F32Smem* gs, const float* Zs, int
 }
 
 
-__global__ void __launch_bounds__(kF32Threads, 1) fused_f32_kernel(gpo_batch b, gpo_outputs o, Sizes sz, Ws ws,
-                                                                   Params p) {
+template <int NT, int TAMAX>
+__global__ void __launch_bounds__(NT, 1) fused_f32_kernel(gpo_batch b, gpo_outputs o, Sizes sz, Ws ws, Params p) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   F32Smem* gs = reinterpret_cast<F32Smem*>(smem_raw);
   float* Zs = reinterpret_cast<float*>(smem_raw + kF32ZOff);
   uint32_t* st = ws.status;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  constexpr int nt = kF32Threads;
+  constexpr int nt = NT;
   const int d = sz.d, ds = f32_row_stride(d);
+  float* part = Zs + (size_t)sz.maxn * ds;  // Gram partial sums of parts 1.. (f32_partial_bytes)
   const float kappa = p.kappa_f;
   if (blockIdx.x == 0 && tid == 0) {
     if (b.group_rollout_off[0] != 0 || b.group_rollout_off[sz.G] != sz.R) report(st, GPO_ERR_SHAPE, 2, 0);
@@ -220,14 +249,20 @@ __global__ void __launch_bounds__(kF32Threads, 1) fused_f32_kernel(gpo_batch b, 
 
     // ---- Gram block and pair tests (f32_gram_links: TA = ceil(n / 16) row blocks per thread)
     switch ((n + 15) >> 4) {
-      case 1: f32_gram_links<1>(gs, Zs, n, d, ds, s0, kappa, p.rule, tid, st); break;
-      case 2: f32_gram_links<2>(gs, Zs, n, d, ds, s0, kappa, p.rule, tid, st); break;
-      case 3: f32_gram_links<3>(gs, Zs, n, d, ds, s0, kappa, p.rule, tid, st); break;
-      case 4: f32_gram_links<4>(gs, Zs, n, d, ds, s0, kappa, p.rule, tid, st); break;
-      case 5: f32_gram_links<5>(gs, Zs, n, d, ds, s0, kappa, p.rule, tid, st); break;
-      case 6: f32_gram_links<6>(gs, Zs, n, d, ds, s0, kappa, p.rule, tid, st); break;
-      case 7: f32_gram_links<7>(gs, Zs, n, d, ds, s0, kappa, p.rule, tid, st); break;
-      default: f32_gram_links<8>(gs, Zs, n, d, ds, s0, kappa, p.rule, tid, st); break;
+      case 1: f32_gram_links<1, NT>(gs, Zs, n, d, ds, s0, kappa, p.rule, tid, part, st); break;
+      case 2: f32_gram_links<2, NT>(gs, Zs, n, d, ds, s0, kappa, p.rule, tid, part, st); break;
+      case 3: f32_gram_links<3, NT>(gs, Zs, n, d, ds, s0, kappa, p.rule, tid, part, st); break;
+      case 4: f32_gram_links<4, NT>(gs, Zs, n, d, ds, s0, kappa, p.rule, tid, part, st); break;
+      default:
+        if constexpr (TAMAX > 4) {
+          switch ((n + 15) >> 4) {
+            case 5: f32_gram_links<5, NT>(gs, Zs, n, d, ds, s0, kappa, p.rule, tid, part, st); break;
+            case 6: f32_gram_links<6, NT>(gs, Zs, n, d, ds, s0, kappa, p.rule, tid, part, st); break;
+            case 7: f32_gram_links<7, NT>(gs, Zs, n, d, ds, s0, kappa, p.rule, tid, part, st); break;
+            default: f32_gram_links<8, NT>(gs, Zs, n, d, ds, s0, kappa, p.rule, tid, part, st); break;
+          }
+        }
+        break;
     }
     // ---- error-free row statistics for eta (one warp per row, from the rows in shared
     //      memory; the prompt embedding from global memory; TwoProduct for fp32 products)
@@ -317,7 +352,9 @@ __global__ void __launch_bounds__(kF32Threads, 1) fused_f32_kernel(gpo_batch b, 
   }
 }
 
-size_t f32_smem_bytes(int d, int maxn) { return kF32ZOff + (size_t)maxn * f32_row_stride(d) * sizeof(float); }
+size_t f32_smem_bytes(int d, int maxn, int nt, int tamax) {
+  return kF32ZOff + (size_t)maxn * f32_row_stride(d) * sizeof(float) + (size_t)f32_partial_bytes(nt, tamax);
+}
 
 }  // namespace
 
@@ -326,8 +363,12 @@ bool fused_f32_fits(int d, int maxn) {
 }
 
 cudaError_t setup_fused_f32() {
-  return cudaFuncSetAttribute(fused_f32_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              (int)(kF32ZOff + kF32MaxZBytes));
+  cudaError_t e = cudaFuncSetAttribute(fused_f32_kernel<256, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)(kF32ZOff + kF32MaxZBytes));
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(fused_f32_kernel<512, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)(kF32ZOff + kF32MaxZBytes + f32_partial_bytes(512, 4)));
+  return e;
 }
 
 cudaError_t launch_fused_f32(const LaunchCtx& lc, const gpo_batch& b, const gpo_outputs& o, const Sizes& sz,
@@ -335,7 +376,10 @@ cudaError_t launch_fused_f32(const LaunchCtx& lc, const gpo_batch& b, const gpo_
   const int ng = sz.g1 - sz.g0;
   if (ng <= 0) return cudaSuccess;
   const int grid = ng < lc.num_sms ? ng : lc.num_sms;
-  fused_f32_kernel<<<grid, kF32Threads, f32_smem_bytes(sz.d, sz.maxn), lc.stream>>>(b, o, sz, ws, p);
+  if (sz.maxn <= kF32SmallN)
+    fused_f32_kernel<512, 4><<<grid, 512, f32_smem_bytes(sz.d, sz.maxn, 512, 4), lc.stream>>>(b, o, sz, ws, p);
+  else
+    fused_f32_kernel<256, 8><<<grid, 256, f32_smem_bytes(sz.d, sz.maxn, 256, 8), lc.stream>>>(b, o, sz, ws, p);
   return cudaGetLastError();
 }
 

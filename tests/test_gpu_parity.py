@@ -209,6 +209,32 @@ def test_zero_rows_and_f32(gp_mod):
     compare(run_gpu(gp_mod, b, params), oracle_run(b, params), "f32 zero rows")
 
 
+@pytest.mark.parametrize("rollouts,d", [(8, 256), (10, 30), (16, 256), (20, 62)])
+def test_parity_f32_instances(gp_mod, rollouts, d):
+    """The fp32 group-resident kernel's two instances: groups of at most 64 states (48, 60:
+    512 threads, the Gram's k range split between the block's halves, whose partial sums
+    are added in a fixed order) and of 65..128 states (96, 120: 256 threads).  d = 30 and 62
+    are not multiples of 4: those rows sit in a buffer padded to 32 and 64 columns (a row's
+    bytes must be a multiple of 16), and the split range ends ragged."""
+    import dataclasses
+    import torch
+    spec = dataclasses.replace(W.CONFIGS["tiny"], rollouts=rollouts, d=d)
+    b = W.make_batch(spec, seed=101 + rollouts + d)
+    params = oracle_params(b)
+    P = gp_mod
+    gp = P.GraphPO(kappa=params["kappa"], w=params["w"], lambda_eff=params["lambda_eff"])
+    db = P.Batch.from_arrays(b, device="cuda")
+    dp = (d + 3) // 4 * 4
+    padded = torch.full((db.emb.shape[0], dp), float("nan"), dtype=torch.float32, device="cuda")
+    padded[:, :d] = db.emb
+    db.emb = padded[:, :d]  # row stride dp, the padding never read
+    assert db.c_struct().emb_row_stride == dp
+    out = gp(db, components=True, nodes=True)
+    gp.check()
+    gpu = {k: v.cpu().numpy() for k, v in out.items()}
+    compare(gpu, oracle_run(b, params), f"f32 {rollouts}x6 states, d={d}")
+
+
 def test_largest_group(gp_mod):
     """One group at the 4096-state limit (16 x 16 tiles of 128 x 256)."""
     rng = np.random.default_rng(11)
